@@ -1,0 +1,680 @@
+#!/usr/bin/env python3
+"""Benchmark of libmpcomp: compress+decompress GB/s (input bytes) and the fraction of HBM
+bandwidth per operator, on one GB300.
+
+Workload (the CNN stage boundary, [128,128,16,16] fp32 = 128 rows x 32768): one step is
+one boundary crossing of every operator the workload sweeps, on that step's tensors:
+  forward : error-feedback TopK at K = 5, 10, 30 % (one error buffer per K, carried
+            across steps) of the activation ReLU(N(0,1)) drifting by 0.1*N(0,1) per step,
+            each followed by TopK decompression;
+  backward: 2/4/8-bit min-max quantisation of the gradient N(0, sigma=1e-3), round to
+            nearest and stochastic (seed (seed << 32) | step), each followed by
+            dequantisation.
+value = sum over the 9 compress+decompress pairs of the input bytes (4 x 128 x 32768) /
+device time of the step.  Each step is one CUDA graph of the 18 library launches (one
+graph per slot of a pool of 4 pre-drawn steps, so inputs differ from step to step); L2
+is flushed (256 MiB write) before every timed step and the flush is outside the timed
+interval.  `e2e` runs the same steps through the Python API without graphs, with the
+step's inputs copied from pinned host memory and two outputs copied back inside the
+timed region.  `operators` times every operator of the path on its own workload.
+
+`--impl reference` times the CPU oracle (single-threaded C) on a bounded sample of the
+same step: 16 of the 128 rows.
+"""
+
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+METRIC = "compress+decompress GB/s (input bytes) and % of HBM roofline per operator at 1 GB300"
+UNIT = "GB/s"
+WORKLOAD = "CNN stage boundary [128,128,16,16] fp32"
+R, L = 128, 32768
+TOPK_PCTS = (5, 10, 30)
+BITS = (2, 4, 8)
+POOL = 4
+SAMPLE_ROWS = 16
+
+
+def parse_args():
+    p = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=200)
+    p.add_argument("--warmup", type=int, default=10)
+    p.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    p.add_argument("--no-operators", action="store_true", help="skip the per-operator table")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    return p.parse_args()
+
+
+# ---------------------------------------------------------------------------------------
+# process group (one process per GPU; independent replicas, no data exchange)
+# ---------------------------------------------------------------------------------------
+
+def dist_env():
+    return (int(os.environ.get("RANK", "0")), int(os.environ.get("LOCAL_RANK", "0")),
+            int(os.environ.get("WORLD_SIZE", "1")))
+
+
+def init_dist(world: int, backend: str):
+    if world > 1:
+        import torch.distributed as dist
+
+        if not dist.is_initialized():
+            dist.init_process_group(backend=backend)
+
+
+def barrier(world: int):
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.barrier()
+
+
+def aggregate(units: float, seconds: float, world: int, device) -> tuple[float, float]:
+    """Whole-job units (sum over ranks) and time (max over ranks)."""
+    if world == 1:
+        return units, seconds
+    import torch.distributed as dist
+
+    t = torch.tensor([units, seconds], dtype=torch.float64, device=device)
+    u = t[:1].clone()
+    s = t[1:].clone()
+    dist.all_reduce(u, op=dist.ReduceOp.SUM)
+    dist.all_reduce(s, op=dist.ReduceOp.MAX)
+    return float(u.item()), float(s.item())
+
+
+# ---------------------------------------------------------------------------------------
+# peaks, clocks, traffic records
+# ---------------------------------------------------------------------------------------
+
+def hbm_peak():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return 6800.0, "fallback"
+
+
+def source_digest() -> str:
+    import hashlib
+
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2401_07788_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        with open(os.path.join(csrc, name), "rb") as f:
+            h.update(name.encode() + f.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(kernel: str):
+    """DRAM bytes per launch from the committed ncu summary, if taken on this source."""
+    path = os.path.join(ROOT, "profiles", "dram_traffic.txt")
+    try:
+        lines = open(path).read().splitlines()
+    except OSError:
+        return None
+    digest = None
+    table = {}
+    for ln in lines:
+        parts = ln.split()
+        if len(parts) >= 2 and parts[0] == "source_digest":
+            digest = parts[1]
+        elif len(parts) >= 2 and not ln.startswith("#"):
+            try:
+                table[parts[0]] = float(parts[1])
+            except ValueError:
+                pass
+    if digest != source_digest():
+        return None
+    return table.get(kernel)
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons while the benchmark runs."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.proc = None
+        try:
+            bus = torch.cuda.get_device_properties(device_index).pci_bus_id
+        except Exception:
+            bus = None
+        self.target = bus
+        self.out = os.path.join("/tmp", "mpc_clocks_%d.csv" % os.getpid())
+
+    def __enter__(self):
+        cmd = ["nvidia-smi", "--query-gpu=" + self.FIELDS, "--format=csv,noheader,nounits",
+               "-lms", "100"]
+        if self.target:
+            cmd += ["-i", self.target]
+        try:
+            self.fh = open(self.out, "w")
+            self.proc = subprocess.Popen(cmd, stdout=self.fh, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.fh.close()
+
+    def summary(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        sm, mx, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        try:
+            rows = open(self.out).read().splitlines()
+        except OSError:
+            rows = []
+        for row in rows:
+            f = [c.strip() for c in row.split(",")]
+            if len(f) < 6:
+                continue
+            try:
+                sm.append(float(f[0]))
+                mx.append(float(f[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[2:6]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        try:
+            os.remove(self.out)
+        except OSError:
+            pass
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------------------
+# the workload
+# ---------------------------------------------------------------------------------------
+
+def algorithmic_bytes(R_, L_, k=None, bits=None, op=""):
+    """Minimum HBM bytes of one launch: inputs and buffers read once, payload and buffers
+    written once."""
+    N = R_ * L_
+    if op == "ef_topk":
+        return 12 * N + 8 * k * R_
+    if op == "topk":
+        return 4 * N + 8 * k * R_
+    if op == "topk_decompress":
+        return 8 * k * R_ + 4 * N
+    if op == "delta_topk":  # EF21 / AQ-SGD: state written only where kept
+        return 8 * N + 12 * k * R_
+    if op == "aqsgd_decompress":
+        return 8 * k * R_ + 8 * k * R_
+    if op in ("quant", "dequant"):
+        return 4 * N + (N * bits + 7) // 8 + 8 * R_
+    raise ValueError(op)
+
+
+class Step:
+    """Pre-allocated tensors and the launch sequence of one boundary step."""
+
+    def __init__(self, mpc, synth, device, seed: int):
+        self.mpc = mpc
+        gen = synth.generator(seed, device)
+        x = synth.relu_normal((R, L), seed, device, gen=gen)
+        self.xs, self.gs = [], []
+        for t in range(POOL):
+            self.xs.append(x)
+            self.gs.append(synth.normal((R, L), 1000 + 100 * seed + t, device, std=1e-3))
+            x = synth.drift(x, 0.1, gen)
+        self.ks = {p: synth.k_of(L, p) for p in TOPK_PCTS}
+        self.errs = {p: torch.zeros((R, L), device=device) for p in TOPK_PCTS}
+        self.vals = {p: torch.empty((R, self.ks[p]), device=device) for p in TOPK_PCTS}
+        self.idx = {p: torch.empty((R, self.ks[p]), dtype=torch.int32, device=device)
+                    for p in TOPK_PCTS}
+        self.y = torch.empty((R, L), device=device)
+        self.gy = torch.empty((R, L), device=device)
+        W = {b: mpc.mpc_quant_codes_words(R, L, b) // R for b in BITS}
+        self.codes = {b: torch.empty((R, W[b]), dtype=torch.int32, device=device) for b in BITS}
+        self.scale = {b: torch.empty(R, device=device) for b in BITS}
+        self.minv = {b: torch.empty(R, device=device) for b in BITS}
+        self.seed = seed
+        self.ops = []  # (name, bytes) in launch order
+        for p in TOPK_PCTS:
+            self.ops.append(("ef_topk_compress K=%d%%" % p,
+                             algorithmic_bytes(R, L, k=self.ks[p], op="ef_topk")))
+            self.ops.append(("topk_decompress K=%d%%" % p,
+                             algorithmic_bytes(R, L, k=self.ks[p], op="topk_decompress")))
+        for b in BITS:
+            for sr in (False, True):
+                tag = "%d-bit %s" % (b, "stochastic" if sr else "nearest")
+                self.ops.append(("quant_compress " + tag, algorithmic_bytes(R, L, bits=b, op="quant")))
+                self.ops.append(("quant_decompress " + tag, algorithmic_bytes(R, L, bits=b, op="dequant")))
+        self.input_bytes = 9 * 4 * R * L  # 9 compress+decompress pairs
+
+    def launch(self, slot: int, step: int, events=None, x=None, g=None):
+        """Enqueue the step's 18 launches; optionally record an event after each."""
+        m = self.mpc
+        x = self.xs[slot] if x is None else x
+        g = self.gs[slot] if g is None else g
+        e = iter(events) if events is not None else None
+        for p in TOPK_PCTS:
+            m.mpc_ef_topk_compress(x, self.errs[p], self.ks[p], self.vals[p], self.idx[p])
+            if e: next(e).record()
+            m.mpc_topk_decompress(self.vals[p], self.idx[p], L, y=self.y)
+            if e: next(e).record()
+        for b in BITS:
+            for sr in (False, True):
+                m.mpc_quant_compress(g, b, stochastic=sr, seed=(self.seed << 32) | step,
+                                     codes=self.codes[b], scale=self.scale[b], minv=self.minv[b])
+                if e: next(e).record()
+                m.mpc_quant_decompress(self.codes[b], self.scale[b], self.minv[b], L, b, y=self.gy)
+                if e: next(e).record()
+
+
+def make_event(external: bool):
+    if external:
+        try:
+            return torch.cuda.Event(enable_timing=True, external=True)
+        except TypeError:
+            return None
+    return torch.cuda.Event(enable_timing=True)
+
+
+def run_ours(args, rank, local, world):
+    import paper_2401_07788_gb300 as mpc
+    from paper_2401_07788_gb300 import synth
+
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    init_dist(world, "nccl")
+    mpc.lib()
+    seed = rank % 10
+    st = Step(mpc, synth, device, seed)
+    n_ops = len(st.ops)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=device)
+    stream = torch.cuda.Stream(device)
+    torch.cuda.synchronize()
+
+    # eager warm-up (sets kernel attributes) before capture
+    with torch.cuda.stream(stream):
+        for w in range(2):
+            st.launch(w % POOL, w)
+    stream.synchronize()
+    assert mpc.mpc_get_status(stream) == 0, mpc.mpc_last_error()
+
+    # one graph per pool slot, with an event after every launch
+    probe = make_event(external=True)
+    per_op_events = probe is not None
+    graphs, evsets = [], []
+    for slot in range(POOL):
+        evs = [make_event(True) for _ in range(n_ops)] if per_op_events else None
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            st.launch(slot, slot, events=evs)
+        graphs.append(g)
+        evsets.append(evs)
+    torch.cuda.synchronize()
+    for p in TOPK_PCTS:
+        st.errs[p].zero_()
+
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    op_ms = [0.0] * n_ops
+    sampler = ClockSampler(local)
+    with sampler:
+        with torch.cuda.stream(stream):
+            for w in range(args.warmup):
+                flush.fill_(w & 0xff)
+                graphs[w % POOL].replay()
+        stream.synchronize()
+        barrier(world)
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        with torch.cuda.stream(stream):
+            for s in range(args.steps):
+                flush.fill_(s & 0xff)
+                starts[s].record(stream)
+                graphs[s % POOL].replay()
+                ends[s].record(stream)
+                if per_op_events:
+                    # events inside the graph belong to its slot; read them before reuse
+                    if (s + 1) % POOL == 0 or s == args.steps - 1:
+                        stream.synchronize()
+                        base = s - (s % POOL)
+                        for j in range(base, s + 1):
+                            evs = evsets[j % POOL]
+                            prev = starts[j]
+                            for i, ev in enumerate(evs):
+                                op_ms[i] += prev.elapsed_time(ev)
+                                prev = ev
+        stream.synchronize()
+        torch.cuda.synchronize()
+        barrier(world)
+        wall = time.perf_counter() - t0
+    clocks = sampler.summary()
+    step_ms = [starts[s].elapsed_time(ends[s]) for s in range(args.steps)]
+    dev_s = sum(step_ms) / 1e3
+    status = mpc.mpc_get_status(stream)
+    if status != 0:
+        raise RuntimeError("device status %d: %s" % (status, mpc.mpc_last_error()))
+
+    units, secs = aggregate(st.input_bytes * args.steps, dev_s, world, device)
+    value = units / secs / 1e9
+
+    # roofline of the dominant kernel (largest share of the step)
+    peak, peak_kind = hbm_peak()
+    roofline = None
+    if per_op_events and sum(op_ms) > 0:
+        i = max(range(n_ops), key=lambda j: op_ms[j])
+        name, nbytes = st.ops[i]
+        avg_ms = op_ms[i] / args.steps
+        achieved = nbytes / (avg_ms / 1e3) / 1e9
+        kern = "topk_cta_kernel" if "topk_compress" in name else (
+            "topk_decompress_kernel" if "decompress K" in name else (
+                "quant_cta_kernel" if "quant_compress" in name else "dequant_kernel"))
+        traffic = recorded_traffic(kern + ":" + name.replace(" ", "_"))
+        roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                    "frac": round(achieved / peak, 4), "traffic": traffic,
+                    "kernel": kern, "op": name, "algorithmic_bytes": nbytes,
+                    "avg_launch_us": round(avg_ms * 1e3, 2),
+                    "share_of_step": round(op_ms[i] / max(sum(op_ms), 1e-9), 4),
+                    "peak_source": peak_kind}
+        per_op = {st.ops[j][0]: {"avg_us": round(op_ms[j] / args.steps * 1e3, 2),
+                                 "GBps": round(st.ops[j][1] / (op_ms[j] / args.steps / 1e3) / 1e9, 1)}
+                  for j in range(n_ops)}
+    else:
+        per_op = None
+
+    # end to end through the Python API: host inputs in, two outputs back, no graphs
+    e2e = run_e2e(args, st, stream, world, device)
+
+    operators = None
+    if not args.no_operators and rank == 0:
+        operators = measure_operators(mpc, synth, device, stream, peak)
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(budget_s=10.0)
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": round(value, 2), "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(secs * 1e3 / args.steps, 4), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": {"workload": WORKLOAD, "rows": R, "row_len": L,
+                       "topk_percents": list(TOPK_PCTS), "bits": list(BITS),
+                       "rounding": ["nearest", "stochastic"], "launches_per_step": n_ops,
+                       "step": "one CUDA graph per step", "l2": "256 MiB flush before each "
+                       "timed step, outside the timed interval", "parallelism":
+                       "replicas" if world > 1 else "single GPU"},
+            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
+            "gpu_launches": n_ops * args.steps, "clocks": clocks,
+            "wall_s": round(wall, 3), "per_op": per_op, "operators": operators,
+        }
+        print(json.dumps(line), flush=True)
+
+
+def run_e2e(args, st, stream, world, device):
+    mpc = st.mpc
+    hx = [t.cpu().pin_memory() for t in st.xs]
+    hg = [t.cpu().pin_memory() for t in st.gs]
+    dx = torch.empty_like(st.xs[0])
+    dg = torch.empty_like(st.gs[0])
+    hy = torch.empty((R, L), pin_memory=True)
+    hgy = torch.empty((R, L), pin_memory=True)
+    k10 = 10
+
+    def one(s):
+        dx.copy_(hx[s % POOL], non_blocking=True)
+        dg.copy_(hg[s % POOL], non_blocking=True)
+        st.launch(0, s, x=dx, g=dg)
+        # outputs read back: the K=10% decompressed activation and the 8-bit gradient
+        mpc.mpc_topk_decompress(st.vals[k10], st.idx[k10], L, y=st.y)
+        hy.copy_(st.y, non_blocking=True)
+        hgy.copy_(st.gy, non_blocking=True)
+
+    steps = max(3, min(args.steps, 50))
+    with torch.cuda.stream(stream):
+        for s in range(3):
+            one(s)
+    stream.synchronize()
+    barrier(world)
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for s in range(steps):
+            one(s)
+        e1.record(stream)
+    stream.synchronize()
+    barrier(world)
+    secs = e0.elapsed_time(e1) / 1e3
+    units, secs = aggregate(st.input_bytes * steps, secs, world, device)
+    return {"value": round(units / secs / 1e9, 2), "unit": UNIT,
+            "h2d_bytes_per_step": 2 * 4 * R * L, "d2h_bytes_per_step": 2 * 4 * R * L,
+            "steps": steps, "api": "python binding, no graphs"}
+
+
+def time_op(fn, stream, flush, reps=5):
+    """Median device time (ms) of fn over reps, L2 flushed before each."""
+    ts = []
+    with torch.cuda.stream(stream):
+        fn()
+        for r in range(reps):
+            flush.fill_(r)
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            fn()
+            b.record(stream)
+            stream.synchronize()
+            ts.append(a.elapsed_time(b))
+    return statistics.median(ts)
+
+
+def measure_operators(mpc, synth, device, stream, peak):
+    """Every operator of the path on its own workload: GB/s of algorithmic bytes and the
+    fraction of HBM bandwidth."""
+    out = {}
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=device)
+
+    def rec(name, ms, nbytes):
+        gbs = nbytes / (ms / 1e3) / 1e9
+        out[name] = {"us": round(ms * 1e3, 2), "GBps": round(gbs, 1), "frac": round(gbs / peak, 4),
+                     "MB": round(nbytes / 1e6, 2)}
+
+    # small CNN boundary: Top10% and 8-bit
+    x = synth.relu_normal((32, 16384), 0, device)
+    k = synth.k_of(16384, 10)
+    v, i = mpc.mpc_topk_compress(x, k)
+    y = torch.empty_like(x)
+    rec("topk_compress 32x16384 K=10%", time_op(lambda: mpc.mpc_topk_compress(x, k, v, i), stream, flush),
+        algorithmic_bytes(32, 16384, k=k, op="topk"))
+    rec("topk_decompress 32x16384 K=10%", time_op(lambda: mpc.mpc_topk_decompress(v, i, 16384, y=y), stream, flush),
+        algorithmic_bytes(32, 16384, k=k, op="topk_decompress"))
+    # LM boundary: EF21 Top10% per token, 4-bit
+    xl = synth.lm_hidden(0, device)
+    gl = torch.zeros_like(xl)
+    kl = synth.k_of(768, 10)
+    vl, il = mpc.mpc_ef21_topk_compress(xl, gl, kl)
+    rec("ef21_topk_compress 8192x768 K=10%", time_op(lambda: mpc.mpc_ef21_topk_compress(xl, gl, kl, vl, il), stream, flush),
+        algorithmic_bytes(8192, 768, k=kl, op="delta_topk"))
+    cq, sq, mq = mpc.mpc_quant_compress(xl, 4)
+    yl = torch.empty_like(xl)
+    rec("quant_compress 8192x768 4-bit", time_op(lambda: mpc.mpc_quant_compress(xl, 4, codes=cq, scale=sq, minv=mq), stream, flush),
+        algorithmic_bytes(8192, 768, bits=4, op="quant"))
+    rec("quant_decompress 8192x768 4-bit", time_op(lambda: mpc.mpc_quant_decompress(cq, sq, mq, 768, 4, y=yl), stream, flush),
+        algorithmic_bytes(8192, 768, bits=4, op="dequant"))
+    del xl, gl, yl
+    # AQ-SGD boundary: 8 GiB buffer, 16 ids, Top30%
+    S, rps, La = 4096, 512, 1024
+    buf = synth.normal((S, rps, La), 0, device)
+    ids = synth.sample_ids(S, 16, 1, device)
+    xa = buf[ids] + 0.05 * torch.randn((16, rps, La), device=device)
+    ka = synth.k_of(La, 30)
+    va, ia = mpc.mpc_aqsgd_compress(xa, buf, ids, ka)
+    rec("aqsgd_compress 16x512x1024 K=30%", time_op(lambda: mpc.mpc_aqsgd_compress(xa, buf, ids, ka, va, ia), stream, flush),
+        algorithmic_bytes(16 * rps, La, k=ka, op="delta_topk"))
+    rec("aqsgd_decompress 16x512x1024 K=30%", time_op(lambda: mpc.mpc_aqsgd_decompress(va, ia, buf, ids), stream, flush),
+        algorithmic_bytes(16 * rps, La, k=ka, op="aqsgd_decompress"))
+    del buf, xa
+    torch.cuda.empty_cache()
+    # bandwidth sweep point: one 1 GiB tensor
+    N = 1 << 28
+    xs = synth.normal((N,), 28, device)
+    for Ls in (768, 4096, 65536):
+        Rs = N // Ls
+        xv = xs[: Rs * Ls].view(Rs, Ls)
+        for pct in (1, 10, 50):
+            ks = synth.k_of(Ls, pct)
+            vs, is_ = mpc.mpc_topk_compress(xv, ks)
+            rec("topk_compress 2^28 L=%d K=%d%%" % (Ls, pct), time_op(lambda: mpc.mpc_topk_compress(xv, ks, vs, is_), stream, flush, 3),
+                algorithmic_bytes(Rs, Ls, k=ks, op="topk"))
+            if pct == 10:
+                ys = torch.empty_like(xv)
+                rec("topk_decompress 2^28 L=%d K=10%%" % Ls, time_op(lambda: mpc.mpc_topk_decompress(vs, is_, Ls, y=ys), stream, flush, 3),
+                    algorithmic_bytes(Rs, Ls, k=ks, op="topk_decompress"))
+                es = torch.zeros_like(xv)
+                rec("ef_topk_compress 2^28 L=%d K=10%%" % Ls, time_op(lambda: mpc.mpc_ef_topk_compress(xv, es, ks, vs, is_), stream, flush, 3),
+                    algorithmic_bytes(Rs, Ls, k=ks, op="ef_topk"))
+                del ys, es
+            del vs, is_
+        for b in BITS:
+            cq, sq, mq = mpc.mpc_quant_compress(xv, b)
+            rec("quant_compress 2^28 L=%d %d-bit" % (Ls, b), time_op(lambda: mpc.mpc_quant_compress(xv, b, codes=cq, scale=sq, minv=mq), stream, flush, 3),
+                algorithmic_bytes(Rs, Ls, bits=b, op="quant"))
+            if b == 4:
+                rec("quant_compress 2^28 L=%d 4-bit stochastic" % Ls, time_op(lambda: mpc.mpc_quant_compress(xv, 4, True, 7, codes=cq, scale=sq, minv=mq), stream, flush, 3),
+                    algorithmic_bytes(Rs, Ls, bits=4, op="quant"))
+                ys = torch.empty_like(xv)
+                rec("quant_decompress 2^28 L=%d 4-bit" % Ls, time_op(lambda: mpc.mpc_quant_decompress(cq, sq, mq, Ls, 4, y=ys), stream, flush, 3),
+                    algorithmic_bytes(Rs, Ls, bits=4, op="dequant"))
+                del ys
+    del xs
+    torch.cuda.empty_cache()
+    st = mpc.mpc_get_status(stream)
+    if st != 0:
+        raise RuntimeError("device status %d: %s" % (st, mpc.mpc_last_error()))
+    return out
+
+
+# ---------------------------------------------------------------------------------------
+# CPU oracle (the reference arm and the cpu_baseline key)
+# ---------------------------------------------------------------------------------------
+
+class OracleStep:
+    """The same boundary step on SAMPLE_ROWS of the 128 rows, computed by the oracle."""
+
+    def __init__(self, seed: int = 0):
+        import oracle
+        from paper_2401_07788_gb300 import synth
+
+        self.oracle = oracle
+        self.lib = oracle.load()
+        x = synth.relu_normal((R, L), seed, "cpu")[:SAMPLE_ROWS].numpy().copy()
+        g = synth.normal((R, L), 1000 + 100 * seed, "cpu", std=1e-3)[:SAMPLE_ROWS].numpy().copy()
+        self.x, self.g = x, g
+        self.ks = {p: synth.k_of(L, p) for p in TOPK_PCTS}
+        self.errs = {p: np.zeros_like(x) for p in TOPK_PCTS}
+        self.seed = seed
+        self.input_bytes = 9 * 4 * SAMPLE_ROWS * L
+
+    def run(self, step: int):
+        o = self.oracle
+        for p in TOPK_PCTS:
+            v, i = o.ef_topk_compress(self.x, self.errs[p], self.ks[p], self.lib)
+            o.topk_decompress(v, i, L, self.lib)
+        for b in BITS:
+            for sr in (False, True):
+                c, s, m = o.quant_compress(self.g, b, sr, (self.seed << 32) | step, self.lib)
+                o.quant_decompress(c, s, m, L, b, self.lib)
+
+
+def cpu_baseline(budget_s: float = 10.0):
+    st = OracleStep(0)
+    st.run(0)
+    n, t0 = 0, time.perf_counter()
+    while time.perf_counter() - t0 < budget_s or n < 2:
+        st.run(n)
+        n += 1
+    secs = time.perf_counter() - t0
+    return {"value": round(st.input_bytes * n / secs / 1e9, 4), "unit": UNIT, "cores": 1,
+            "kind": "oracle", "sample": "%d of %d rows of the step, %d steps in %.1f s"
+            % (SAMPLE_ROWS, R, n, secs), "cpu": cpu_name()}
+
+
+def cpu_name():
+    try:
+        for ln in open("/proc/cpuinfo"):
+            if ln.lower().startswith(("model name", "cpu part")):
+                return ln.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    return os.uname().machine
+
+
+def run_reference(args, rank, world):
+    if rank != 0:
+        return
+    st = OracleStep(0)
+    for w in range(args.warmup):
+        st.run(w)
+    t0 = time.perf_counter()
+    for s in range(args.steps):
+        st.run(s)
+    secs = time.perf_counter() - t0
+    value = st.input_bytes * args.steps / secs / 1e9
+    line = {
+        "impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": UNIT,
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(secs * 1e3 / args.steps, 3), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "rows": R, "row_len": L,
+                   "topk_percents": list(TOPK_PCTS), "bits": list(BITS),
+                   "sample_rows": SAMPLE_ROWS},
+        "cpu_baseline": {"value": round(value, 4), "unit": UNIT, "cores": 1, "kind": "oracle",
+                         "sample": "%d of %d rows of each step" % (SAMPLE_ROWS, R),
+                         "cpu": cpu_name()},
+        "e2e": {"value": round(value, 4), "unit": UNIT, "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse_args()
+    rank, local, world = dist_env()
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+        return
+    run_ours(args, rank, local, world)
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

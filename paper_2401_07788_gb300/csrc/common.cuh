@@ -1,0 +1,175 @@
+// common.cuh -- device helpers shared by the libmpcomp kernels (sm_103a).
+//
+// Inline PTX wrappers for the Blackwell data-movement path (bulk asynchronous
+// copies completing on an mbarrier, thread-block clusters and distributed
+// shared memory), exact fp32 arithmetic helpers, the magnitude keys used by
+// TopK selection and the device status word.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace mpc {
+
+// ---------------------------------------------------------------------------
+// Device status word (read and cleared by mpc_get_status on the host).
+// ---------------------------------------------------------------------------
+enum : unsigned {
+  STATUS_TIMEOUT = 1u,     // a bounded wait on an mbarrier gave up
+  STATUS_BAD_SAMPLE = 2u,  // an AQ-SGD sample id was out of range
+};
+// Kernels receive the address of the library's status word (one per device)
+// and OR their error bits into it.
+__device__ __forceinline__ void set_status(unsigned* status, unsigned bits) {
+  if (status != nullptr) atomicOr(status, bits);
+}
+
+// ---------------------------------------------------------------------------
+// Exact fp32 arithmetic: every call is one IEEE round-to-nearest-even
+// operation and is never contracted into a fused multiply-add.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float fadd(float a, float b) { return __fadd_rn(a, b); }
+__device__ __forceinline__ float fsub(float a, float b) { return __fsub_rn(a, b); }
+__device__ __forceinline__ float fmul(float a, float b) { return __fmul_rn(a, b); }
+__device__ __forceinline__ float fdiv(float a, float b) { return __fdiv_rn(a, b); }
+
+// Magnitude key of a float: its bit pattern without the sign.  For
+// non-negative floats the integer order of the bit patterns is the numeric
+// order, so comparing keys compares |x| (and +0, -0 share key 0).
+__device__ __forceinline__ int mag_key(float v) {
+  return static_cast<int>(__float_as_uint(v) & 0x7fffffffu);
+}
+
+// ---------------------------------------------------------------------------
+// Shared-memory addresses, mbarriers and bulk copies.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_addr(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(count)
+               : "memory");
+}
+
+// Make mbarrier initialisation visible to the async proxy and the cluster.
+__device__ __forceinline__ void fence_mbar_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+// Order this thread's earlier generic-proxy shared-memory accesses before
+// later async-proxy (bulk copy) accesses to the same memory.
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)),
+               "r"(bytes)
+               : "memory");
+}
+
+// Non-blocking test of phase `parity` of `bar` (returns at once).
+__device__ __forceinline__ bool mbar_test_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(smem_addr(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Wait for phase `parity` of `bar` to complete, testing at most `limit`
+// times (a short sleep between tests after the first few, so every test
+// costs a bounded time).  Returns false, and records STATUS_TIMEOUT, if it
+// gave up.
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity,
+                                                  uint32_t limit, unsigned* status) {
+  for (uint32_t i = 0; i < limit; ++i) {
+    if (mbar_test_wait(bar, parity)) return true;
+    if (i >= 16) __nanosleep(64);
+  }
+  set_status(status, STATUS_TIMEOUT);
+  return false;
+}
+
+// Bulk copy of `bytes` (multiple of 16, both addresses 16-byte aligned) from
+// global to this CTA's shared memory; completion is counted on `bar`.
+__device__ __forceinline__ void bulk_g2s(void* dst_smem, const void* src_gmem, uint32_t bytes,
+                                         uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cta.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          smem_addr(dst_smem)),
+      "l"(src_gmem), "r"(bytes), "r"(smem_addr(bar))
+      : "memory");
+}
+
+// The number of polls a drain wait (after a timed-out wait, before the CTA
+// may exit with a copy still in flight) makes before giving up for good.
+constexpr uint32_t kDrainPolls = 1u << 22;
+
+// ---------------------------------------------------------------------------
+// Thread-block clusters and distributed shared memory.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ uint32_t cluster_size() {
+  uint32_t n;
+  asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(n));
+  return n;
+}
+// Cluster-wide barrier with release/acquire semantics for shared memory.
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::
+                   : "memory");
+}
+// Address of the same shared variable in CTA `rank` of this cluster.
+__device__ __forceinline__ uint32_t dsmem_addr(const void* local, uint32_t rank) {
+  uint32_t out;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(out) : "r"(smem_addr(local)), "r"(rank));
+  return out;
+}
+__device__ __forceinline__ uint32_t dsmem_ld_u32(uint32_t addr) {
+  uint32_t v;
+  asm volatile("ld.shared::cluster.u32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
+  return v;
+}
+__device__ __forceinline__ int dsmem_ld_s32(uint32_t addr) {
+  return static_cast<int>(dsmem_ld_u32(addr));
+}
+__device__ __forceinline__ uint2 dsmem_ld_u32x2(uint32_t addr) {
+  uint2 v;
+  asm volatile("ld.shared::cluster.v2.u32 {%0, %1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(addr) : "memory");
+  return v;
+}
+
+__host__ __device__ __forceinline__ int64_t min64(int64_t a, int64_t b) { return a < b ? a : b; }
+__host__ __device__ __forceinline__ int64_t max64(int64_t a, int64_t b) { return a > b ? a : b; }
+
+// ---------------------------------------------------------------------------
+// Warp helpers.
+// ---------------------------------------------------------------------------
+constexpr unsigned kFull = 0xffffffffu;
+
+__device__ __forceinline__ unsigned lanemask_lt() {
+  unsigned m;
+  asm("mov.u32 %0, %%lanemask_lt;" : "=r"(m));
+  return m;
+}
+
+// Inclusive prefix sum across the warp.
+__device__ __forceinline__ unsigned warp_inclusive_scan(unsigned v, int lane) {
+#pragma unroll
+  for (int d = 1; d < 32; d <<= 1) {
+    unsigned o = __shfl_up_sync(kFull, v, d);
+    if (lane >= d) v += o;
+  }
+  return v;
+}
+
+}  // namespace mpc

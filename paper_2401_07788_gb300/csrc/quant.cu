@@ -1,0 +1,496 @@
+// quant.cu -- min-max quantisation and dequantisation (§2.2).
+//
+// Per row: mn, mx (in the total order with -0 below +0, reduced as
+// order-preserving integer keys), scale = (mx - mn) / L, inv = L / (mx - mn)
+// with L = 2^bits - 1, then for each entry t = (x - mn) * inv and
+// q = round_half_even(t) or floor(t + u), clamped to [0, L], each step one
+// fp32 round-to-nearest operation.  Codes are packed LSB-first into 32-bit
+// words; rows of codes are padded to 16 bytes.
+//
+// Kernels:
+//  * quant_warp_kernel: one warp per row (rows <= 2048 entries), row held in
+//    registers, min/max by warp reductions, codes packed with shuffles.
+//  * quant_cta_kernel: one cluster of CTAs per row; each CTA stages its slice
+//    with one bulk asynchronous copy on an mbarrier and the cluster merges
+//    min/max through distributed shared memory.  With a workspace it instead
+//    takes min/max from a preceding pass (rows too long for a cluster).
+//  * quant_minmax_kernel: that preceding pass (long rows).
+//  * dequant_kernel: grid-stride over code words, 16-byte stores.
+#include "common.cuh"
+#include "kernels.h"
+#include "launch_util.h"
+
+namespace mpc {
+namespace {
+
+constexpr int kQWarps = 8;
+constexpr int kQNT = 256;
+constexpr int kQNV = 8;
+constexpr int kQSCAP = 4 * kQNT * kQNV;  // 8192 entries per CTA slice
+
+// Order-preserving map of float bits to unsigned: -0 below +0, negatives
+// reversed.  Its inverse recovers the exact float.
+__device__ __forceinline__ uint32_t ord_key(float v) {
+  const uint32_t u = __float_as_uint(v);
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+__device__ __forceinline__ float ord_value(uint32_t k) {
+  return __uint_as_float((k & 0x80000000u) ? (k & 0x7fffffffu) : ~k);
+}
+
+// splitmix64 (Steele, Lea & Flood, OOPSLA 2014) at counter c: the finaliser
+// applied to seed + (c + 1) * golden-ratio increment.
+__device__ __forceinline__ uint64_t splitmix64_at(uint64_t seed, uint64_t c) {
+  uint64_t z = seed + (c + 1u) * 0x9E3779B97F4A7C15ull;
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+// u for 4 consecutive flat indices i0..i0+3: 24 bits of the low (even i) or
+// high (odd i) half of splitmix64 at counter i >> 1, times 2^-24.
+__device__ __forceinline__ void uniform4(uint64_t seed, uint64_t i0, float u[4]) {
+  const uint64_t c0 = i0 >> 1;
+  const uint64_t z0 = splitmix64_at(seed, c0);
+  const uint64_t z1 = splitmix64_at(seed, c0 + 1);
+  uint64_t z[4];
+  if ((i0 & 1u) == 0) {
+    z[0] = z0; z[1] = z0; z[2] = z1; z[3] = z1;
+  } else {
+    const uint64_t z2 = splitmix64_at(seed, c0 + 2);
+    z[0] = z0; z[1] = z1; z[2] = z1; z[3] = z2;
+  }
+#pragma unroll
+  for (int t = 0; t < 4; ++t) {
+    const uint64_t i = i0 + t;
+    const uint32_t h = (i & 1u) ? static_cast<uint32_t>(z[t] >> 32) : static_cast<uint32_t>(z[t]);
+    u[t] = fmul(__uint2float_rn(h >> 8), 0x1p-24f);
+  }
+}
+
+struct RowParams {
+  float mn;
+  float inv;
+  float levels;
+  bool degenerate;
+};
+
+__device__ __forceinline__ RowParams row_params(uint32_t kmin, uint32_t kmax, int bits,
+                                                float* scale_out, float* minv_out) {
+  RowParams p;
+  p.mn = ord_value(kmin);
+  const float mx = ord_value(kmax);
+  p.levels = static_cast<float>((1u << bits) - 1u);
+  const float range = fsub(mx, p.mn);
+  p.inv = fdiv(p.levels, range);
+  p.degenerate = (range == 0.0f) || isinf(range) || isinf(p.inv);
+  if (scale_out) *scale_out = p.degenerate ? 0.0f : fdiv(range, p.levels);
+  if (minv_out) *minv_out = p.mn;
+  return p;
+}
+
+// Code of one entry.
+__device__ __forceinline__ uint32_t code_of(float x, const RowParams& p, bool stochastic, float u) {
+  const float t = fmul(fsub(x, p.mn), p.inv);
+  float q = stochastic ? floorf(fadd(t, u)) : rintf(t);
+  q = fminf(fmaxf(q, 0.0f), p.levels);
+  return static_cast<uint32_t>(q);
+}
+
+// Codes of the 4 entries e0..e0+3 of a row (entries at or past n give 0).
+template <int BITS>
+__device__ __forceinline__ uint32_t codes4(const float xs[4], int64_t e0, int64_t n,
+                                           const RowParams& p, bool stochastic, uint64_t seed,
+                                           uint64_t flat0) {
+  uint32_t packed = 0;
+  if (p.degenerate) return 0;
+  float u[4] = {0.f, 0.f, 0.f, 0.f};
+  if (stochastic) uniform4(seed, flat0, u);
+#pragma unroll
+  for (int t = 0; t < 4; ++t)
+    if (e0 + t < n) packed |= code_of(xs[t], p, stochastic, u[t]) << (BITS * t);
+  return packed;
+}
+
+// Assemble 32-bit words from 4*BITS-bit pieces held by consecutive lanes;
+// returns true on the lane that stores the word.
+template <int BITS>
+__device__ __forceinline__ bool assemble_word(uint32_t& piece, int lane) {
+  if (BITS == 8) return true;
+  if (BITS == 4) {
+    const uint32_t hi = __shfl_down_sync(kFull, piece, 1);
+    piece |= hi << 16;
+    return (lane & 1) == 0;
+  }
+  // BITS == 2
+  const uint32_t p1 = __shfl_down_sync(kFull, piece, 1);
+  const uint32_t p2 = __shfl_down_sync(kFull, piece, 2);
+  const uint32_t p3 = __shfl_down_sync(kFull, piece, 3);
+  piece |= (p1 << 8) | (p2 << 16) | (p3 << 24);
+  return (lane & 3) == 0;
+}
+
+// ---------------------------------------------------------------------------
+// One warp per row
+// ---------------------------------------------------------------------------
+template <int BITS, int NVW>
+__global__ void __launch_bounds__(32 * kQWarps) quant_warp_kernel(const QuantArgs a) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int64_t L = a.L;
+  const int64_t data_words = (L * BITS + 31) / 32;
+  for (int64_t row = static_cast<int64_t>(blockIdx.x) * kQWarps + warp; row < a.rows;
+       row += static_cast<int64_t>(gridDim.x) * kQWarps) {
+    const float* xr = a.x + row * L;
+    float xs[NVW][4];
+    uint32_t kmin = 0xffffffffu, kmax = 0u;
+#pragma unroll
+    for (int v = 0; v < NVW; ++v) {
+      const int64_t e0 = 4 * (v * 32 + lane);
+      if (a.aligned && e0 + 4 <= L) {
+        const float4 f = *reinterpret_cast<const float4*>(xr + e0);
+        xs[v][0] = f.x; xs[v][1] = f.y; xs[v][2] = f.z; xs[v][3] = f.w;
+      } else {
+#pragma unroll
+        for (int t = 0; t < 4; ++t) xs[v][t] = (e0 + t < L) ? xr[e0 + t] : 0.0f;
+      }
+#pragma unroll
+      for (int t = 0; t < 4; ++t)
+        if (e0 + t < L) {
+          const uint32_t ok = ord_key(xs[v][t]);
+          kmin = min(kmin, ok);
+          kmax = max(kmax, ok);
+        }
+    }
+    kmin = __reduce_min_sync(kFull, kmin);
+    kmax = __reduce_max_sync(kFull, kmax);
+    const RowParams p = row_params(kmin, kmax, BITS, lane == 0 ? a.scale + row : nullptr,
+                                   lane == 0 ? a.minv + row : nullptr);
+    uint32_t* cr = a.codes + row * a.W;
+#pragma unroll
+    for (int v = 0; v < NVW; ++v) {
+      const int64_t e0 = 4 * (v * 32 + lane);
+      uint32_t piece = codes4<BITS>(xs[v], e0, L, p, a.stochastic, a.seed,
+                                    static_cast<uint64_t>(row * L + e0));
+      const bool store = assemble_word<BITS>(piece, lane);
+      const int64_t w = e0 * BITS / 32;
+      if (store && w < data_words) cr[w] = piece;
+    }
+    if (lane < a.W - data_words) cr[data_words + lane] = 0u;  // row padding
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Cluster of CTAs per row (or, with a workspace, CTAs over one row's chunks)
+// ---------------------------------------------------------------------------
+struct QuantShared {
+  uint32_t redmin[kQNT / 32];
+  uint32_t redmax[kQNT / 32];
+  uint32_t pub_min, pub_max;
+  uint64_t bar;
+};
+
+template <int BITS>
+__global__ void __launch_bounds__(kQNT) quant_cta_kernel(const QuantArgs a, int spr) {
+  __shared__ QuantShared sh;
+  extern __shared__ __align__(16) float sx[];  // kQSCAP floats
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const bool from_ws = a.ws != nullptr;
+  const uint32_t C = from_ws ? 1u : cluster_size();
+  const int64_t row = blockIdx.x / spr;
+  const int64_t sidx = blockIdx.x % spr;  // slice index within the row (= cluster rank)
+  const int64_t L = a.L;
+  const int64_t c0 = sidx * a.slice;
+  const int n = static_cast<int>(max64(0, min64(a.slice, L - c0)));
+  const float* xr = a.x + row * L;
+
+  bool failed = false;
+  if (a.aligned) {
+    if (tid == 0) {
+      mbar_init(&sh.bar, 1);
+      fence_mbar_init();
+    }
+    __syncthreads();
+    if (n > 0) {
+      if (tid == 0) {
+        mbar_arrive_expect_tx(&sh.bar, static_cast<uint32_t>(n) * 4u);
+        bulk_g2s(sx, xr + c0, static_cast<uint32_t>(n) * 4u, &sh.bar);
+      }
+      if (!mbar_wait_bounded(&sh.bar, 0, a.spin_limit, a.status)) {
+        mbar_wait_bounded(&sh.bar, 0, kDrainPolls, nullptr);
+        failed = true;
+      }
+    }
+    failed = __syncthreads_or(failed);
+  } else {
+    for (int e = tid; e < n; e += kQNT) sx[e] = xr[c0 + e];
+    __syncthreads();
+  }
+  const int nv = failed ? 0 : n;
+
+  uint32_t kmin, kmax;
+  if (from_ws) {
+    const uint32_t* mm = static_cast<const uint32_t*>(a.ws) + 2 * row;
+    kmin = mm[0];
+    kmax = mm[1];
+  } else {
+    kmin = 0xffffffffu;
+    kmax = 0u;
+    for (int e = tid; e < nv; e += kQNT) {
+      const uint32_t ok = ord_key(sx[e]);
+      kmin = min(kmin, ok);
+      kmax = max(kmax, ok);
+    }
+    kmin = __reduce_min_sync(kFull, kmin);
+    kmax = __reduce_max_sync(kFull, kmax);
+    if (lane == 0) {
+      sh.redmin[warp] = kmin;
+      sh.redmax[warp] = kmax;
+    }
+    __syncthreads();
+    if (tid == 0) {
+      uint32_t a0 = 0xffffffffu, a1 = 0u;
+      for (int w = 0; w < kQNT / 32; ++w) {
+        a0 = min(a0, sh.redmin[w]);
+        a1 = max(a1, sh.redmax[w]);
+      }
+      sh.pub_min = a0;
+      sh.pub_max = a1;
+    }
+    if (C > 1) {
+      cluster_sync();
+      kmin = 0xffffffffu;
+      kmax = 0u;
+      for (uint32_t r = 0; r < C; ++r) {
+        kmin = min(kmin, dsmem_ld_u32(dsmem_addr(&sh.pub_min, r)));
+        kmax = max(kmax, dsmem_ld_u32(dsmem_addr(&sh.pub_max, r)));
+      }
+    } else {
+      __syncthreads();
+      kmin = sh.pub_min;
+      kmax = sh.pub_max;
+    }
+  }
+  const bool writer = sidx == 0 && tid == 0 && !failed;
+  const RowParams p = row_params(kmin, kmax, BITS, writer ? a.scale + row : nullptr,
+                                 writer ? a.minv + row : nullptr);
+
+  uint32_t* cr = a.codes + row * a.W;
+  const int64_t data_words = (L * BITS + 31) / 32;
+  if (!failed) {
+#pragma unroll
+    for (int v = 0; v < kQNV; ++v) {
+      const int q = v * kQNT + tid;
+      const int64_t e0 = 4 * q;  // slice-relative
+      const float4 f = reinterpret_cast<const float4*>(sx)[q];
+      const float xs[4] = {f.x, f.y, f.z, f.w};
+      uint32_t piece = codes4<BITS>(xs, e0, nv, p, a.stochastic, a.seed,
+                                    static_cast<uint64_t>(row * L + c0 + e0));
+      const bool store = assemble_word<BITS>(piece, lane);
+      const int64_t w = (c0 + e0) * BITS / 32;
+      if (store && e0 < nv && w < data_words) cr[w] = piece;
+    }
+    if (c0 + n >= L && tid < a.W - data_words) cr[data_words + tid] = 0u;  // row padding
+  }
+  if (C > 1) cluster_sync();
+}
+
+// Long rows, first pass: per-row min/max keys into the workspace (which the
+// launcher initialises to {0xffffffff, 0}).
+__global__ void __launch_bounds__(kQNT) quant_minmax_kernel(const float* x, int64_t L, int spr,
+                                                            int64_t slice, uint32_t* mm) {
+  const int64_t row = blockIdx.x / spr;
+  const int64_t c0 = (blockIdx.x % spr) * slice;
+  const int64_t n = max64(0, min64(slice, L - c0));
+  const float* xr = x + row * L + c0;
+  uint32_t kmin = 0xffffffffu, kmax = 0u;
+  for (int64_t e = threadIdx.x; e < n; e += kQNT) {
+    const uint32_t ok = ord_key(xr[e]);
+    kmin = min(kmin, ok);
+    kmax = max(kmax, ok);
+  }
+  kmin = __reduce_min_sync(kFull, kmin);
+  kmax = __reduce_max_sync(kFull, kmax);
+  if ((threadIdx.x & 31) == 0) {
+    atomicMin(mm + 2 * row, kmin);
+    atomicMax(mm + 2 * row + 1, kmax);
+  }
+}
+
+__global__ void minmax_init_kernel(uint32_t* mm, int64_t rows) {
+  for (int64_t r = blockIdx.x * blockDim.x + threadIdx.x; r < rows;
+       r += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    mm[2 * r] = 0xffffffffu;
+    mm[2 * r + 1] = 0u;
+  }
+}
+
+// bits = 32: raw passthrough of the fp32 bits.
+__global__ void passthrough_kernel(const float* __restrict__ x, int64_t rows, int64_t L,
+                                   int64_t W, uint32_t* __restrict__ codes, float* scale,
+                                   float* minv) {
+  const int64_t total = rows * W;
+  for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int64_t r = i / W, j = i % W;
+    codes[i] = j < L ? __float_as_uint(x[r * L + j]) : 0u;
+    if (j == 0) {
+      scale[r] = 0.0f;
+      minv[r] = 0.0f;
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Dequantisation: y = minv + float(q) * scale
+// ---------------------------------------------------------------------------
+template <int BITS>
+__global__ void __launch_bounds__(256)
+    dequant_kernel(const uint32_t* __restrict__ codes, const float* __restrict__ scale,
+                   const float* __restrict__ minv, int64_t rows, int64_t L, int64_t W,
+                   int64_t wpr, float* __restrict__ y, int aligned) {
+  constexpr int PER = 32 / BITS;  // codes per word
+  const int64_t total = rows * wpr;
+  for (int64_t g = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; g < total;
+       g += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int64_t r = g / wpr, w = g % wpr;
+    const uint32_t word = codes[r * W + w];
+    const float s = scale[r], m = minv[r];
+    float out[PER];
+#pragma unroll
+    for (int t = 0; t < PER; ++t) {
+      const uint32_t q = (word >> (BITS * t)) & ((1u << BITS) - 1u);
+      out[t] = fadd(m, fmul(static_cast<float>(q), s));
+    }
+    const int64_t e0 = w * PER;
+    float* yr = y + r * L;
+    if (aligned && e0 + PER <= L) {
+#pragma unroll
+      for (int t = 0; t < PER; t += 4)
+        *reinterpret_cast<float4*>(yr + e0 + t) = make_float4(out[t], out[t + 1], out[t + 2], out[t + 3]);
+    } else {
+#pragma unroll
+      for (int t = 0; t < PER; ++t)
+        if (e0 + t < L) yr[e0 + t] = out[t];
+    }
+  }
+}
+
+__global__ void dequant_passthrough_kernel(const uint32_t* __restrict__ codes, int64_t rows,
+                                           int64_t L, int64_t W, float* __restrict__ y) {
+  const int64_t total = rows * L;
+  for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int64_t r = i / L, j = i % L;
+    y[i] = __uint_as_float(codes[r * W + j]);
+  }
+}
+
+template <int BITS, int NVW>
+cudaError_t run_quant_warp(const QuantArgs& a, int num_sms, cudaStream_t s) {
+  auto kernel = quant_warp_kernel<BITS, NVW>;
+  const int occ = resident_blocks(kernel, 32 * kQWarps, 0);
+  const int64_t want = (a.rows + kQWarps - 1) / kQWarps;
+  const int64_t cap = static_cast<int64_t>(num_sms) * occ;
+  kernel<<<static_cast<unsigned>(want < cap ? want : cap), 32 * kQWarps, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+template <int BITS>
+cudaError_t run_quant_bits(const QuantArgs& a0, int num_sms, cudaStream_t s) {
+  QuantArgs a = a0;
+  const int64_t L = a.L;
+  if (a.ws == nullptr && L <= 2048) {
+    if (L <= 256) return run_quant_warp<BITS, 2>(a, num_sms, s);
+    if (L <= 512) return run_quant_warp<BITS, 4>(a, num_sms, s);
+    if (L <= 768) return run_quant_warp<BITS, 6>(a, num_sms, s);
+    if (L <= 1024) return run_quant_warp<BITS, 8>(a, num_sms, s);
+    return run_quant_warp<BITS, 16>(a, num_sms, s);
+  }
+  auto kernel = quant_cta_kernel<BITS>;
+  const int smem = kQSCAP * 4;
+  cudaError_t err = ensure_dynamic_smem(kernel, smem);
+  if (err != cudaSuccess) return err;
+  int64_t spr;
+  if (a.ws == nullptr) {
+    spr = (L + kQSCAP - 1) / kQSCAP;
+    while (a.rows * spr < 2 * num_sms && spr < 8 && L / (2 * spr) >= 1024) spr *= 2;
+    if (spr > 8) return cudaErrorInvalidValue;
+    a.slice = ((L + spr - 1) / spr + 127) / 128 * 128;
+  } else {
+    a.slice = kQSCAP;
+    spr = (L + kQSCAP - 1) / kQSCAP;
+    uint32_t* mm = static_cast<uint32_t*>(a.ws);
+    minmax_init_kernel<<<static_cast<unsigned>(min64((a.rows + 255) / 256, 1024)), 256, 0, s>>>(mm, a.rows);
+    quant_minmax_kernel<<<static_cast<unsigned>(a.rows * spr), kQNT, 0, s>>>(a.x, L, static_cast<int>(spr), a.slice, mm);
+    err = cudaGetLastError();
+    if (err != cudaSuccess) return err;
+  }
+  const int64_t blocks = a.rows * spr;
+  if (blocks > 0x7fffffffLL) return cudaErrorInvalidValue;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(blocks), 1, 1);
+  cfg.blockDim = dim3(kQNT, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = (a.ws == nullptr) ? static_cast<unsigned>(spr) : 1u;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, a, static_cast<int>(spr));
+}
+
+unsigned grid_for(int64_t work, int num_sms) {
+  const int64_t cap = static_cast<int64_t>(num_sms) * 16;
+  const int64_t b = (work + 255) / 256;
+  return static_cast<unsigned>(b < 1 ? 1 : (b < cap ? b : cap));
+}
+
+}  // namespace
+
+size_t quant_workspace_bytes(int64_t rows, int64_t L, int bits) {
+  if (bits == 32 || L <= kQuantRowPathMaxLen) return 0;
+  return static_cast<size_t>(rows) * 8u;
+}
+
+cudaError_t launch_quant_compress(const QuantArgs& a, int num_sms, cudaStream_t s) {
+  if (a.rows <= 0) return cudaSuccess;
+  switch (a.bits) {
+    case 2: return run_quant_bits<2>(a, num_sms, s);
+    case 4: return run_quant_bits<4>(a, num_sms, s);
+    case 8: return run_quant_bits<8>(a, num_sms, s);
+    case 32:
+      passthrough_kernel<<<grid_for(a.rows * a.W, num_sms), 256, 0, s>>>(a.x, a.rows, a.L, a.W,
+                                                                          a.codes, a.scale, a.minv);
+      return cudaGetLastError();
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+cudaError_t launch_quant_decompress(const uint32_t* codes, const float* scale,
+                                    const float* minv, int64_t rows, int64_t L, int bits,
+                                    int64_t W, float* y, int aligned, int num_sms,
+                                    cudaStream_t s) {
+  if (rows <= 0) return cudaSuccess;
+  const int64_t wpr = (L * bits + 31) / 32;
+  switch (bits) {
+    case 2:
+      dequant_kernel<2><<<grid_for(rows * wpr, num_sms), 256, 0, s>>>(codes, scale, minv, rows, L, W, wpr, y, aligned);
+      break;
+    case 4:
+      dequant_kernel<4><<<grid_for(rows * wpr, num_sms), 256, 0, s>>>(codes, scale, minv, rows, L, W, wpr, y, aligned);
+      break;
+    case 8:
+      dequant_kernel<8><<<grid_for(rows * wpr, num_sms), 256, 0, s>>>(codes, scale, minv, rows, L, W, wpr, y, aligned);
+      break;
+    case 32:
+      dequant_passthrough_kernel<<<grid_for(rows * L, num_sms), 256, 0, s>>>(codes, rows, L, W, y);
+      break;
+    default: return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
+}
+
+}  // namespace mpc

@@ -1,0 +1,150 @@
+// topk_decompress.cu -- TopK decompression (§2.3: the kept values are put back
+// at their indices and every other entry is zero) and the AQ-SGD receiver's
+// buffer update (§2.5).
+//
+// Decompression builds each output tile in shared memory (zero fill, scatter
+// of the tile's kept entries) and writes it to HBM once with 16-byte stores.
+// A tile is either several whole rows (short rows) or a column range of one
+// row (long rows); for a column range the kept entries are found by a
+// block-parallel search of the row's ascending indices.
+#include "common.cuh"
+#include "kernels.h"
+#include "launch_util.h"
+
+namespace mpc {
+namespace {
+
+constexpr int kTile = 16384;  // floats per output tile (64 KiB of shared memory)
+constexpr int kDecThreads = 256;
+
+// Number of entries of idx[0..n) that are < target, for ascending idx;
+// every thread of the block returns the same value.
+__device__ int64_t block_lower_bound(const int32_t* idx, int64_t n, int64_t target) {
+  int64_t lo = 0, hi = n;
+  while (lo < hi) {
+    const int64_t span = hi - lo;
+    const int64_t stride = (span + kDecThreads - 1) / kDecThreads;
+    const int64_t p = lo + static_cast<int64_t>(threadIdx.x) * stride;
+    const bool pred = p < hi && static_cast<int64_t>(idx[p]) < target;
+    const int c = __syncthreads_count(pred);
+    if (c == 0) {
+      hi = lo;
+    } else {
+      const int64_t last = lo + static_cast<int64_t>(c - 1) * stride;
+      hi = min(hi, lo + static_cast<int64_t>(c) * stride);
+      lo = last + 1;
+    }
+  }
+  return lo;
+}
+
+// rpc rows per CTA when tpr == 1; tpr column tiles per row when rpc == 1.
+__global__ void __launch_bounds__(kDecThreads)
+    topk_decompress_kernel(const float* __restrict__ vals, const int32_t* __restrict__ idx,
+                           int64_t rows, int64_t L, int64_t k, float* __restrict__ y,
+                           int64_t rpc, int64_t tpr, int aligned) {
+  extern __shared__ __align__(16) float tile[];  // kTile floats
+  const int tid = threadIdx.x;
+  const int64_t g = blockIdx.x;
+  int64_t r0, nrows, c0, ncols, e_begin, e_end;
+  if (tpr == 1) {
+    r0 = g * rpc;
+    nrows = min(rpc, rows - r0);
+    c0 = 0;
+    ncols = L;
+    e_begin = r0 * k;
+    e_end = (r0 + nrows) * k;
+  } else {
+    r0 = g / tpr;
+    nrows = 1;
+    c0 = (g % tpr) * kTile;
+    ncols = min64(kTile, L - c0);
+    const int32_t* ri = idx + r0 * k;
+    const int64_t lb0 = block_lower_bound(ri, k, c0);
+    const int64_t lb1 = block_lower_bound(ri, k, c0 + ncols);
+    e_begin = r0 * k + lb0;
+    e_end = r0 * k + max(lb0, lb1);
+  }
+  const int64_t cells = nrows * ncols;  // <= kTile
+  for (int64_t i = tid; i < (cells + 3) / 4; i += kDecThreads)
+    reinterpret_cast<float4*>(tile)[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+  __syncthreads();
+  for (int64_t e = e_begin + tid; e < e_end; e += kDecThreads) {
+    // rpc * k <= kTile, so the 32-bit quotient is exact
+    const int64_t lr =
+        (tpr == 1) ? static_cast<uint32_t>(e - e_begin) / static_cast<uint32_t>(k) : 0u;
+    const int64_t col = static_cast<int64_t>(idx[e]) - c0;
+    if (col >= 0 && col < ncols) tile[lr * ncols + col] = vals[e];
+  }
+  __syncthreads();
+  float* dst = y + r0 * L + c0;
+  if (aligned) {
+    const int64_t n4 = cells / 4;
+    for (int64_t i = tid; i < n4; i += kDecThreads)
+      reinterpret_cast<float4*>(dst)[i] = reinterpret_cast<const float4*>(tile)[i];
+    for (int64_t i = n4 * 4 + tid; i < cells; i += kDecThreads) dst[i] = tile[i];
+  } else {
+    for (int64_t i = tid; i < cells; i += kDecThreads) dst[i] = tile[i];
+  }
+}
+
+// One CTA per logical payload row: buf_recv[s][r][idx] += vals.
+__global__ void __launch_bounds__(kDecThreads)
+    aqsgd_decompress_kernel(const float* __restrict__ vals, const int32_t* __restrict__ idx,
+                            float* __restrict__ buf, int64_t num_samples,
+                            const int64_t* __restrict__ ids, int64_t rps, int64_t L, int64_t k,
+                            unsigned* status) {
+  const int64_t lr = blockIdx.x;
+  const int64_t sid = ids[lr / rps];
+  if (sid < 0 || sid >= num_samples) {
+    if (threadIdx.x == 0) set_status(status, STATUS_BAD_SAMPLE);
+    return;
+  }
+  float* brow = buf + (sid * rps + lr % rps) * L;
+  const float* v = vals + lr * k;
+  const int32_t* ix = idx + lr * k;
+  for (int64_t i = threadIdx.x; i < k; i += kDecThreads) {
+    const int64_t c = ix[i];
+    if (c >= 0 && c < L) brow[c] = fadd(brow[c], v[i]);
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_topk_decompress(const float* vals, const int32_t* idx, int64_t rows,
+                                   int64_t L, int64_t k, float* y, int aligned, int num_sms,
+                                   cudaStream_t s) {
+  (void)num_sms;
+  if (rows <= 0) return cudaSuccess;
+  int64_t rpc = 1, tpr = 1, blocks;
+  if (L <= kTile) {
+    rpc = kTile / L;
+    if (rpc > rows) rpc = rows;
+    blocks = (rows + rpc - 1) / rpc;
+  } else {
+    tpr = (L + kTile - 1) / kTile;
+    blocks = rows * tpr;
+  }
+  if (blocks > 0x7fffffffLL) return cudaErrorInvalidValue;
+  const int smem = kTile * 4;
+  cudaError_t err = ensure_dynamic_smem(topk_decompress_kernel, smem);
+  if (err != cudaSuccess) return err;
+  topk_decompress_kernel<<<static_cast<unsigned>(blocks), kDecThreads, smem, s>>>(
+      vals, idx, rows, L, k, y, rpc, tpr, aligned);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_aqsgd_decompress(const float* vals, const int32_t* idx, float* buf,
+                                    int64_t num_samples, const int64_t* ids, int64_t n_ids,
+                                    int64_t rps, int64_t L, int64_t k, unsigned* status,
+                                    int num_sms, cudaStream_t s) {
+  (void)num_sms;
+  const int64_t rows = n_ids * rps;
+  if (rows <= 0) return cudaSuccess;
+  if (rows > 0x7fffffffLL) return cudaErrorInvalidValue;
+  aqsgd_decompress_kernel<<<static_cast<unsigned>(rows), kDecThreads, 0, s>>>(
+      vals, idx, buf, num_samples, ids, rps, L, k, status);
+  return cudaGetLastError();
+}
+
+}  // namespace mpc

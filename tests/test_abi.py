@@ -1,0 +1,98 @@
+"""The C-ABI library loads on the CPU and exports every symbol its header declares, and
+its host-side argument validation rejects bad calls before any launch (no GPU needed:
+validation returns before any CUDA call)."""
+
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "mpcomp.h")
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(mpc_\w+)\s*\(", text)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    import __graft_entry__ as g
+
+    g.build()
+    import paper_2401_07788_gb300 as mpc
+
+    return mpc.lib()
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for want in ("mpc_topk_compress", "mpc_topk_decompress", "mpc_ef_topk_compress",
+                 "mpc_ef21_topk_compress", "mpc_aqsgd_compress", "mpc_aqsgd_decompress",
+                 "mpc_quant_compress", "mpc_quant_decompress", "mpc_get_status",
+                 "mpc_last_error", "mpc_topk_workspace_bytes", "mpc_quant_codes_words"):
+        assert want in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+
+
+def test_version(lib):
+    assert lib.mpc_version() >= 100
+
+
+def test_sizes(lib):
+    # W = roundup4(ceil(L*b/32)) words per row
+    assert lib.mpc_quant_codes_words(3, 768, 4) == 3 * 96
+    assert lib.mpc_quant_codes_words(1, 31, 2) == 4
+    assert lib.mpc_quant_codes_words(2, 16384, 8) == 2 * 4096
+    assert lib.mpc_quant_codes_words(1, 5, 32) == 8
+    assert lib.mpc_quant_codes_words(1, 5, 6) == 0  # unsupported width
+    assert lib.mpc_topk_workspace_bytes(128, 32768, 3276) == 0  # on-chip path
+    assert lib.mpc_quant_workspace_bytes(128, 32768, 4) == 0
+
+
+@pytest.mark.parametrize("args,code", [
+    ((0x1000, 4, 16, 0), 1),        # k = 0
+    ((0x1000, 4, 16, 17), 1),       # k > row_len
+    ((0x1000, 4, 0, 1), 1),         # row_len = 0
+    ((0x1000, -1, 16, 1), 1),       # rows < 0
+    ((0, 4, 16, 2), 1),             # x NULL
+    ((0x1002, 4, 16, 2), 1),        # x misaligned
+])
+def test_topk_validation(lib, args, code):
+    x, rows, L, k = args
+    st = lib.mpc_topk_compress(ctypes.c_void_p(x), rows, L, k, ctypes.c_void_p(0x2000),
+                               ctypes.c_void_p(0x3000), None, 0, None)
+    assert st == code
+    assert lib.mpc_last_error()
+
+
+def test_zero_rows_is_a_noop(lib):
+    assert lib.mpc_topk_compress(None, 0, 16, 2, None, None, None, 0, None) == 0
+
+
+def test_quant_validation(lib):
+    p = ctypes.c_void_p(0x1000)
+    assert lib.mpc_quant_compress(p, 2, 16, 3, 0, 0, p, p, p, None, 0, None) == 1  # bits
+    assert lib.mpc_quant_compress(p, 2, 16, 4, 7, 0, p, p, p, None, 0, None) == 1  # mode
+    assert lib.mpc_quant_decompress(p, p, p, 2, 16, 5, p, None) == 1
+
+
+def test_aqsgd_validation(lib):
+    p = ctypes.c_void_p(0x1000)
+    # sample_ids misaligned
+    assert lib.mpc_aqsgd_compress(p, p, 10, ctypes.c_void_p(0x1004), 2, 3, 16, 2, p, p, None, 0,
+                                  None) == 1
+    assert lib.mpc_aqsgd_compress(p, p, 0, p, 2, 3, 16, 2, p, p, None, 0, None) == 1
+
+
+def test_knobs(lib):
+    assert lib.mpc_set_knob(99, 0) == 1
+    assert lib.mpc_set_knob(2, 5) == 1
+    assert lib.mpc_set_knob(2, 0) == 0

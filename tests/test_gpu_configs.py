@@ -1,0 +1,183 @@
+"""The five stage-boundary workloads at their full sizes, in the launch configuration the
+benchmark uses, against the CPU oracle: every output where the oracle finishes in seconds,
+sampled rows (recomputed one by one by the oracle) where it does not."""
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from gpu_cases import assert_bits_equal
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def mpc():
+    import __graft_entry__ as g
+
+    g.build()
+    import paper_2401_07788_gb300 as m
+
+    torch.cuda.set_device(0)
+    return m
+
+
+@pytest.fixture(scope="module")
+def synth():
+    from paper_2401_07788_gb300 import synth as s
+
+    return s
+
+
+def ok(mpc):
+    assert mpc.mpc_get_status() == 0, mpc.mpc_last_error()
+
+
+def test_cnn_small_boundary(mpc, synth):
+    """ResNet-18 boundary [32,64,16,16]: Top10% of the activation, 8-bit gradient."""
+    c = synth.CNN_SMALL
+    x = synth.relu_normal(c["shape"], 0, "cuda").view(c["rows"], c["row_len"])
+    g = synth.normal(c["shape"], 1, "cuda", std=1e-3).view(c["rows"], c["row_len"])
+    k = synth.k_of(c["row_len"], c["topk_percent"])
+    v, i = mpc.mpc_topk_compress(x, k)
+    y = mpc.mpc_topk_decompress(v, i, c["row_len"])
+    cq, sq, mq = mpc.mpc_quant_compress(g, 8)
+    gy = mpc.mpc_quant_decompress(cq, sq, mq, c["row_len"], 8)
+    ok(mpc)
+    xn, gn = x.cpu().numpy(), g.cpu().numpy()
+    ov, oi = oracle.topk_compress(xn, k)
+    assert_bits_equal(i.cpu().numpy(), oi, "idx")
+    assert_bits_equal(v.cpu().numpy(), ov, "vals")
+    assert_bits_equal(y.cpu().numpy(), oracle.topk_decompress(ov, oi, c["row_len"]), "y")
+    oc, os_, om = oracle.quant_compress(gn, 8)
+    assert_bits_equal(cq.cpu().numpy().view(np.uint32), oc, "codes")
+    assert_bits_equal(gy.cpu().numpy(), oracle.quant_decompress(oc, os_, om, c["row_len"], 8),
+                      "dequant")
+
+
+@pytest.mark.parametrize("seed", [0, 9])
+def test_cnn_boundary_ef_and_quant(mpc, synth, seed):
+    """[128,128,16,16]: EF-TopK at 5/10/30% with the error carried over drifting steps;
+    2/4/8-bit gradients, nearest and stochastic (seed (config_seed << 32) | step)."""
+    c = synth.CNN
+    R, L = c["rows"], c["row_len"]
+    gen = synth.generator(seed, "cuda")
+    x = synth.relu_normal(c["shape"], seed, "cuda", gen=gen).view(R, L)
+    errs = {p: torch.zeros((R, L), device="cuda") for p in c["topk_percents"]}
+    errs_host = {p: np.zeros((R, L), np.float32) for p in c["topk_percents"]}
+    for step in range(3):
+        xn = x.cpu().numpy()
+        for p in c["topk_percents"]:
+            k = synth.k_of(L, p)
+            v, i = mpc.mpc_ef_topk_compress(x, errs[p], k)
+            ok(mpc)
+            ov, oi = oracle.ef_topk_compress(xn, errs_host[p], k)
+            assert_bits_equal(i.cpu().numpy(), oi, "idx K=%d step %d" % (p, step))
+            assert_bits_equal(v.cpu().numpy(), ov, "vals K=%d step %d" % (p, step))
+            assert_bits_equal(errs[p].cpu().numpy(), errs_host[p], "err K=%d step %d" % (p, step))
+        g = synth.normal((R, L), 1000 * seed + step, "cuda", std=1e-3)
+        gn = g.cpu().numpy()
+        for bits in c["bits"]:
+            for sr in (False, True):
+                sd = (seed << 32) | step
+                cq, sq, mq = mpc.mpc_quant_compress(g, bits, stochastic=sr, seed=sd)
+                ok(mpc)
+                oc, os_, om = oracle.quant_compress(gn, bits, sr, sd)
+                assert_bits_equal(cq.cpu().numpy().view(np.uint32), oc, "codes b=%d" % bits)
+                assert_bits_equal(sq.cpu().numpy(), os_, "scale b=%d" % bits)
+                assert_bits_equal(mq.cpu().numpy(), om, "minv b=%d" % bits)
+        x = synth.drift(x, c["drift"], gen)
+
+
+def test_lm_boundary_ef21_and_quant(mpc, synth):
+    """GPT-2 boundary [8,1024,768] with outlier channels: EF21-TopK 10% per token, g_0 = 0,
+    over drifting steps; 4-bit per-token gradient quantisation."""
+    c = synth.LM
+    R, L = c["rows"], c["row_len"]
+    k = synth.k_of(L, c["topk_percent"])
+    x = synth.lm_hidden(0, "cuda")
+    gen = synth.generator(1, "cuda")
+    g_dev = torch.zeros((R, L), device="cuda")
+    g_host = np.zeros((R, L), np.float32)
+    for step in range(3):
+        xn = x.cpu().numpy()
+        v, i = mpc.mpc_ef21_topk_compress(x, g_dev, k)
+        ok(mpc)
+        ov, oi = oracle.ef21_topk_compress(xn, g_host, k)
+        assert_bits_equal(i.cpu().numpy(), oi, "idx step %d" % step)
+        assert_bits_equal(v.cpu().numpy(), ov, "vals step %d" % step)
+        assert_bits_equal(g_dev.cpu().numpy(), g_host, "g step %d" % step)
+        x = synth.drift(x, c["drift"], gen)
+    gr = synth.normal((R, L), 2, "cuda", std=1e-4)
+    cq, sq, mq = mpc.mpc_quant_compress(gr, 4)
+    y = mpc.mpc_quant_decompress(cq, sq, mq, L, 4)
+    ok(mpc)
+    oc, os_, om = oracle.quant_compress(gr.cpu().numpy(), 4)
+    assert_bits_equal(cq.cpu().numpy().view(np.uint32), oc, "codes")
+    assert_bits_equal(y.cpu().numpy(), oracle.quant_decompress(oc, os_, om, L, 4), "dequant")
+
+
+def test_aqsgd_boundary_full_buffer(mpc, synth):
+    """Per-sample buffer [4096,512,1024] (2^31 entries, 64-bit offsets): 16 ids per step,
+    Top30% of the change; the gathered rows are checked against the oracle and rows of
+    samples not drawn stay bit-identical."""
+    c = synth.AQSGD
+    S, rps, L = c["num_samples"], c["rows_per_sample"], c["row_len"]
+    k = synth.k_of(L, c["topk_percent"])
+    buf = synth.normal((S, rps, L), 0, "cuda")
+    watch = torch.tensor([0, 1, S // 2, S - 1], device="cuda")
+    gen = synth.generator(5, "cuda")
+    for step in range(2):
+        ids = synth.sample_ids(S, c["ids_per_step"], 100 + step, "cuda")
+        x = buf[ids] + c["noise"] * torch.randn((ids.numel(), rps, L), generator=gen, device="cuda")
+        rows_before = buf[ids].cpu().numpy()
+        untouched = watch[~torch.isin(watch, ids)]
+        keep = buf[untouched].clone()
+        v, i = mpc.mpc_aqsgd_compress(x, buf, ids, k)
+        ok(mpc)
+        local = rows_before.copy()
+        ov, oi = oracle.aqsgd_compress(x.cpu().numpy(), local, np.arange(ids.numel()), k)
+        assert_bits_equal(i.cpu().numpy(), oi, "idx step %d" % step)
+        assert_bits_equal(v.cpu().numpy(), ov, "vals step %d" % step)
+        assert_bits_equal(buf[ids].cpu().numpy(), local, "buffer rows step %d" % step)
+        assert torch.equal(buf[untouched], keep)
+    del buf
+    torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("log2n", [20, 26, 30])
+@pytest.mark.parametrize("L", [768, 4096, 65536])
+def test_sweep_sampled_rows(mpc, synth, log2n, L):
+    """Single N(0,1) tensors of 2^20..2^30 entries as rows of L: TopK 1/10/50% plain and
+    with error feedback, 2/4/8-bit quantisation; 8 sampled rows recomputed by the oracle."""
+    N = 1 << log2n
+    R = N // L
+    x = synth.normal((R * L,), log2n, "cuda").view(R, L)
+    rows = np.unique(np.random.default_rng(log2n + L).integers(0, R, 8))
+    rows = np.unique(np.concatenate([rows, [0, R - 1]]))
+    xs = x[torch.from_numpy(rows).cuda()].cpu().numpy()
+    for pct in (1, 10, 50):
+        k = synth.k_of(L, pct)
+        v, i = mpc.mpc_topk_compress(x, k)
+        ok(mpc)
+        ov, oi = oracle.topk_compress(xs, k)
+        assert_bits_equal(i[rows].cpu().numpy(), oi, "idx K=%d" % pct)
+        assert_bits_equal(v[rows].cpu().numpy(), ov, "vals K=%d" % pct)
+        del v, i
+        err = torch.full_like(x, 0.25)
+        v, i = mpc.mpc_ef_topk_compress(x, err, k)
+        ok(mpc)
+        eh = np.full_like(xs, 0.25)
+        ov, oi = oracle.ef_topk_compress(xs, eh, k)
+        assert_bits_equal(i[rows].cpu().numpy(), oi, "EF idx K=%d" % pct)
+        assert_bits_equal(err[rows].cpu().numpy(), eh, "EF err K=%d" % pct)
+        del v, i, err
+    for bits in (2, 4, 8):
+        cq, sq, mq = mpc.mpc_quant_compress(x, bits)
+        ok(mpc)
+        oc, os_, om = oracle.quant_compress(xs, bits)
+        assert_bits_equal(cq[rows].cpu().numpy().view(np.uint32), oc, "codes b=%d" % bits)
+        assert_bits_equal(sq[rows].cpu().numpy(), os_, "scale b=%d" % bits)
+    del x
+    torch.cuda.empty_cache()

@@ -1,0 +1,52 @@
+"""Device-side waits give up cleanly: with the spin limit at 0 every first wait on a bulk
+copy gives up, the kernel records a timeout in the status word, drains its copy and
+returns; the context stays usable.  No fault, trap or hang is involved."""
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from gpu_cases import assert_bits_equal, rows_of
+
+pytestmark = pytest.mark.gpu
+
+DEFAULT_SPIN = 1 << 20
+
+
+@pytest.fixture(scope="module")
+def mpc():
+    import __graft_entry__ as g
+
+    g.build()
+    import paper_2401_07788_gb300 as m
+
+    torch.cuda.set_device(0)
+    yield m
+    m.mpc_set_knob(m.MPC_KNOB_SPIN_LIMIT, DEFAULT_SPIN)
+
+
+@pytest.mark.parametrize("op,L", [("ef", 4096), ("ef", 32768), ("plain", 768), ("quant", 32768)])
+def test_timeout_is_reported_and_context_survives(mpc, op, L):
+    x = torch.from_numpy(rows_of("normal", 6, L, seed=1)).cuda()
+    err = torch.zeros_like(x)
+    mpc.mpc_set_knob(mpc.MPC_KNOB_SPIN_LIMIT, 0)
+    try:
+        if op == "ef":
+            mpc.mpc_ef_topk_compress(x, err, L // 10)
+        elif op == "plain":
+            mpc.mpc_topk_compress(x, L // 10)
+        else:
+            mpc.mpc_quant_compress(x, 4)
+        assert mpc.mpc_get_status() == 5  # MPC_ERR_TIMEOUT
+        assert "wait" in mpc.mpc_last_error()
+    finally:
+        mpc.mpc_set_knob(mpc.MPC_KNOB_SPIN_LIMIT, DEFAULT_SPIN)
+    assert mpc.mpc_get_status() == 0
+    # the same call now succeeds and matches the oracle
+    xn = x.cpu().numpy()
+    v, i = mpc.mpc_topk_compress(x, L // 10)
+    ov, oi = oracle.topk_compress(xn, L // 10)
+    assert mpc.mpc_get_status() == 0
+    assert_bits_equal(i.cpu().numpy(), oi, "idx after timeout")
+    assert_bits_equal(v.cpu().numpy(), ov, "vals after timeout")
