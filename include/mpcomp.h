@@ -188,6 +188,26 @@ mpc_status mpc_quant_decompress(const uint32_t* codes, const float* scale,
                                 const float* minv, int64_t rows, int64_t row_len, int bits,
                                 float* y, mpc_stream_t stream);
 
+/* Quantise without allocating (the paper has no counterpart; this is a
+ * deployment convenience).  Same operation, arguments and results as
+ * mpc_quant_compress, bit for bit, but with no workspace argument: for callers
+ * that cannot allocate device memory when they quantise (a fixed memory plan,
+ * a host framework that forbids allocation inside its step, an allocator that
+ * cannot be called from there).  The per-row scratch is a static device array
+ * of 8 * MPC_QUANT_NOALLOC_MAX_ROWS bytes (512 KiB) that every device loading
+ * the library keeps until the process exits.  rows > MPC_QUANT_NOALLOC_MAX_ROWS
+ * returns MPC_ERR_INVALID_ARG and launches nothing.
+ * The first call on a device looks up the array's device address (with that
+ * device current); make that first call outside any CUDA stream capture.
+ * Every call shares the one array: calls whose kernels may overlap on the GPU
+ * (different streams without ordering) race and give undefined results; calls
+ * ordered on one stream are safe.  No cudaMalloc, cudaFree or allocating
+ * library routine is called. */
+#define MPC_QUANT_NOALLOC_MAX_ROWS 65536
+mpc_status mpc_quant_compress_noalloc(const float* x, int64_t rows, int64_t row_len, int bits,
+                                      mpc_rounding mode, uint64_t seed, uint32_t* codes,
+                                      float* scale, float* minv, mpc_stream_t stream);
+
 /* ------------------------------------------------------------------------ */
 /* Status and diagnostics                                                   */
 /* ------------------------------------------------------------------------ */

@@ -54,6 +54,8 @@ _SIGNATURES = {
     "mpc_quant_compress": ([_VP, _I64, _I64, _INT, _INT, _U64, _VP, _VP, _VP, _VP, _SZ, _VP],
                            _INT),
     "mpc_quant_decompress": ([_VP, _VP, _VP, _I64, _I64, _INT, _VP, _VP], _INT),
+    "mpc_quant_compress_noalloc": ([_VP, _I64, _I64, _INT, _INT, _U64, _VP, _VP, _VP, _VP],
+                                   _INT),
     "mpc_get_status": ([_VP], _INT),
     "mpc_last_error": ([], ctypes.c_char_p),
     "mpc_set_knob": ([_INT, _I64], _INT),

@@ -327,6 +327,47 @@ mpc_status mpc_quant_compress(const float* x, int64_t rows, int64_t row_len, int
   return ok();
 }
 
+mpc_status mpc_quant_compress_noalloc(const float* x, int64_t rows, int64_t row_len, int bits,
+                                      mpc_rounding mode, uint64_t seed, uint32_t* codes,
+                                      float* scale, float* minv, mpc_stream_t stream) {
+  MPC_TRY(check_shape(rows, row_len, 1));
+  if (bits != 2 && bits != 4 && bits != 8 && bits != 32)
+    return set_error(MPC_ERR_INVALID_ARG, "bits=%d not in {2, 4, 8, 32}", bits);
+  if (mode != MPC_ROUND_NEAREST && mode != MPC_ROUND_STOCHASTIC)
+    return set_error(MPC_ERR_INVALID_ARG, "rounding mode %d", static_cast<int>(mode));
+  if (row_len > 0x7fffffffLL / 32) return set_error(MPC_ERR_INVALID_ARG, "row_len too large");
+  if (rows > mpc::quant_noalloc_max_rows())
+    return set_error(MPC_ERR_INVALID_ARG,
+                     "rows=%lld exceeds the %lld rows of the static scratch of "
+                     "mpc_quant_compress_noalloc",
+                     (long long)rows, (long long)mpc::quant_noalloc_max_rows());
+  if (rows == 0) return ok();
+  MPC_TRY(check_ptr(x, 4, "x"));
+  MPC_TRY(check_ptr(codes, 4, "codes"));
+  MPC_TRY(check_ptr(scale, 4, "scale"));
+  MPC_TRY(check_ptr(minv, 4, "minv"));
+  Device d;
+  MPC_TRY(current_device(&d));
+  mpc::QuantArgs a = {};
+  a.x = x;
+  a.rows = rows;
+  a.L = row_len;
+  a.bits = bits;
+  a.stochastic = (mode == MPC_ROUND_STOCHASTIC);
+  a.seed = seed;
+  a.codes = codes;
+  a.scale = scale;
+  a.minv = minv;
+  a.W = static_cast<int64_t>(mpc_quant_codes_words(1, row_len, bits));
+  a.aligned = (row_len % 4 == 0) && aligned_to(x, 16);
+  a.spin_limit = g_spin_limit.load();
+  a.status = d.status;
+  cudaError_t e = mpc::launch_quant_compress_noalloc(a, d.num_sms,
+                                                     reinterpret_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_error(e, "quant_compress_noalloc launch");
+  return ok();
+}
+
 mpc_status mpc_quant_decompress(const uint32_t* codes, const float* scale, const float* minv,
                                 int64_t rows, int64_t row_len, int bits, float* y,
                                 mpc_stream_t stream) {

@@ -79,6 +79,9 @@ struct QuantArgs {
 constexpr int64_t kQuantRowPathMaxLen = 65536;
 size_t quant_workspace_bytes(int64_t rows, int64_t L, int bits);
 cudaError_t launch_quant_compress(const QuantArgs& a, int num_sms, cudaStream_t s);
+// Allocation-free variant: the min/max scratch is a static device array.
+int64_t quant_noalloc_max_rows();
+cudaError_t launch_quant_compress_noalloc(const QuantArgs& a, int num_sms, cudaStream_t s);
 cudaError_t launch_quant_decompress(const uint32_t* codes, const float* scale,
                                     const float* minv, int64_t rows, int64_t L, int bits,
                                     int64_t W, float* y, int aligned, int num_sms,

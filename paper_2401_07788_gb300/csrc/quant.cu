@@ -16,6 +16,8 @@
 //    takes min/max from a preceding pass (rows too long for a cluster).
 //  * quant_minmax_kernel: that preceding pass (long rows).
 //  * dequant_kernel: grid-stride over code words, 16-byte stores.
+#include <mutex>
+
 #include "common.cuh"
 #include "kernels.h"
 #include "launch_util.h"
@@ -491,6 +493,56 @@ cudaError_t launch_quant_decompress(const uint32_t* codes, const float* scale,
     default: return cudaErrorInvalidValue;
   }
   return cudaGetLastError();
+}
+
+
+// ---------------------------------------------------------------------------
+// Allocation-free quantisation (the paper has no counterpart).
+//
+// Some callers cannot allocate device memory at the moment they quantise: a
+// stage running under a memory planner that has handed out every byte, a
+// plugin inside a host framework that forbids allocations during its step,
+// or code whose allocator may not be called from where it runs.  For them the
+// per-row {min, max} scratch of the two-pass quantisation lives in a fixed
+// file-scope device array instead of a caller workspace.  Every device that
+// loads the library holds this array (8 bytes x kNoallocMaxRows) until the
+// process exits.  The array's host-side name only stands in for it; its
+// device address is looked up once per device with cudaGetSymbolAddress.
+// ---------------------------------------------------------------------------
+namespace {
+
+constexpr int64_t kNoallocMaxRows = 65536;
+static __device__ __align__(256) uint32_t g_noalloc_minmax[2 * kNoallocMaxRows];
+
+std::mutex g_noalloc_mu;
+uint32_t* g_noalloc_ptr[64];
+
+}  // namespace
+
+int64_t quant_noalloc_max_rows() { return kNoallocMaxRows; }
+
+cudaError_t launch_quant_compress_noalloc(const QuantArgs& a0, int num_sms, cudaStream_t s) {
+  if (a0.rows > kNoallocMaxRows) return cudaErrorInvalidValue;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  uint32_t* scratch;
+  {
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    if (g_noalloc_ptr[dev] == nullptr) {
+      void* p = nullptr;
+      e = cudaGetSymbolAddress(&p, g_noalloc_minmax);
+      if (e != cudaSuccess) return e;
+      g_noalloc_ptr[dev] = static_cast<uint32_t*>(p);
+    }
+    scratch = g_noalloc_ptr[dev];
+  }
+  QuantArgs a = a0;
+  // The two-pass path starts by writing every row's {min, max} slot, so no
+  // state of an earlier call is read.
+  a.ws = (a.bits == 32) ? nullptr : scratch;
+  return launch_quant_compress(a, num_sms, s);
 }
 
 }  // namespace mpc
