@@ -142,6 +142,9 @@ __device__ __forceinline__ uint32_t dsmem_ld_u32(uint32_t addr) {
 __device__ __forceinline__ int dsmem_ld_s32(uint32_t addr) {
   return static_cast<int>(dsmem_ld_u32(addr));
 }
+__device__ __forceinline__ void dsmem_st_u32(uint32_t addr, uint32_t v) {
+  asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
+}
 __device__ __forceinline__ uint2 dsmem_ld_u32x2(uint32_t addr) {
   uint2 v;
   asm volatile("ld.shared::cluster.v2.u32 {%0, %1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(addr) : "memory");

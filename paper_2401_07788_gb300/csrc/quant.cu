@@ -187,7 +187,8 @@ __global__ void __launch_bounds__(32 * kQWarps) quant_warp_kernel(const QuantArg
 struct QuantShared {
   uint32_t redmin[kQNT / 32];
   uint32_t redmax[kQNT / 32];
-  uint32_t pub_min, pub_max;
+  uint32_t mm_min[8];  // per-CTA extrema of the row, pushed by every CTA of the cluster
+  uint32_t mm_max[8];
   uint64_t bar;
 };
 
@@ -255,21 +256,18 @@ __global__ void __launch_bounds__(kQNT) quant_cta_kernel(const QuantArgs a, int 
         a0 = min(a0, sh.redmin[w]);
         a1 = max(a1, sh.redmax[w]);
       }
-      sh.pub_min = a0;
-      sh.pub_max = a1;
-    }
-    if (C > 1) {
-      cluster_sync();
-      kmin = 0xffffffffu;
-      kmax = 0u;
+      // push this slice's extrema into every CTA of the cluster (itself included)
       for (uint32_t r = 0; r < C; ++r) {
-        kmin = min(kmin, dsmem_ld_u32(dsmem_addr(&sh.pub_min, r)));
-        kmax = max(kmax, dsmem_ld_u32(dsmem_addr(&sh.pub_max, r)));
+        dsmem_st_u32(dsmem_addr(&sh.mm_min[sidx], r), a0);
+        dsmem_st_u32(dsmem_addr(&sh.mm_max[sidx], r), a1);
       }
-    } else {
-      __syncthreads();
-      kmin = sh.pub_min;
-      kmax = sh.pub_max;
+    }
+    if (C > 1) cluster_sync(); else __syncthreads();
+    kmin = 0xffffffffu;
+    kmax = 0u;
+    for (uint32_t r = 0; r < C; ++r) {
+      kmin = min(kmin, sh.mm_min[r]);
+      kmax = max(kmax, sh.mm_max[r]);
     }
   }
   const bool writer = sidx == 0 && tid == 0 && !failed;
@@ -293,7 +291,6 @@ __global__ void __launch_bounds__(kQNT) quant_cta_kernel(const QuantArgs a, int 
     }
     if (c0 + n >= L && tid < a.W - data_words) cr[data_words + tid] = 0u;  // row padding
   }
-  if (C > 1) cluster_sync();
 }
 
 // Long rows, first pass: per-row min/max keys into the workspace (which the
@@ -345,17 +342,17 @@ __global__ void passthrough_kernel(const float* __restrict__ x, int64_t rows, in
 // ---------------------------------------------------------------------------
 // Dequantisation: y = minv + float(q) * scale
 // ---------------------------------------------------------------------------
-template <int BITS>
+template <int BITS, class Index>
 __global__ void __launch_bounds__(256)
     dequant_kernel(const uint32_t* __restrict__ codes, const float* __restrict__ scale,
-                   const float* __restrict__ minv, int64_t rows, int64_t L, int64_t W,
-                   int64_t wpr, float* __restrict__ y, int aligned) {
+                   const float* __restrict__ minv, Index rows, int64_t L, int64_t W, Index wpr,
+                   float* __restrict__ y, int aligned) {
   constexpr int PER = 32 / BITS;  // codes per word
-  const int64_t total = rows * wpr;
-  for (int64_t g = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; g < total;
-       g += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    const int64_t r = g / wpr, w = g % wpr;
-    const uint32_t word = codes[r * W + w];
+  const Index total = rows * wpr;
+  for (Index g = static_cast<Index>(blockIdx.x) * blockDim.x + threadIdx.x; g < total;
+       g += static_cast<Index>(gridDim.x) * blockDim.x) {
+    const Index r = g / wpr, w = g - r * wpr;
+    const uint32_t word = codes[static_cast<int64_t>(r) * W + w];
     const float s = scale[r], m = minv[r];
     float out[PER];
 #pragma unroll
@@ -363,8 +360,8 @@ __global__ void __launch_bounds__(256)
       const uint32_t q = (word >> (BITS * t)) & ((1u << BITS) - 1u);
       out[t] = fadd(m, fmul(static_cast<float>(q), s));
     }
-    const int64_t e0 = w * PER;
-    float* yr = y + r * L;
+    const int64_t e0 = static_cast<int64_t>(w) * PER;
+    float* yr = y + static_cast<int64_t>(r) * L;
     if (aligned && e0 + PER <= L) {
 #pragma unroll
       for (int t = 0; t < PER; t += 4)
@@ -375,6 +372,18 @@ __global__ void __launch_bounds__(256)
         if (e0 + t < L) yr[e0 + t] = out[t];
     }
   }
+}
+
+// 32-bit word indexing whenever the code array allows it (cheaper division).
+template <int BITS>
+void launch_dequant(const uint32_t* codes, const float* scale, const float* minv, int64_t rows,
+                    int64_t L, int64_t W, int64_t wpr, float* y, int aligned, unsigned grid,
+                    cudaStream_t s) {
+  if (rows * wpr < (int64_t{1} << 31))
+    dequant_kernel<BITS, uint32_t><<<grid, 256, 0, s>>>(codes, scale, minv, static_cast<uint32_t>(rows),
+                                                        L, W, static_cast<uint32_t>(wpr), y, aligned);
+  else
+    dequant_kernel<BITS, int64_t><<<grid, 256, 0, s>>>(codes, scale, minv, rows, L, W, wpr, y, aligned);
 }
 
 __global__ void dequant_passthrough_kernel(const uint32_t* __restrict__ codes, int64_t rows,
@@ -479,13 +488,13 @@ cudaError_t launch_quant_decompress(const uint32_t* codes, const float* scale,
   const int64_t wpr = (L * bits + 31) / 32;
   switch (bits) {
     case 2:
-      dequant_kernel<2><<<grid_for(rows * wpr, num_sms), 256, 0, s>>>(codes, scale, minv, rows, L, W, wpr, y, aligned);
+      launch_dequant<2>(codes, scale, minv, rows, L, W, wpr, y, aligned, grid_for(rows * wpr, num_sms), s);
       break;
     case 4:
-      dequant_kernel<4><<<grid_for(rows * wpr, num_sms), 256, 0, s>>>(codes, scale, minv, rows, L, W, wpr, y, aligned);
+      launch_dequant<4>(codes, scale, minv, rows, L, W, wpr, y, aligned, grid_for(rows * wpr, num_sms), s);
       break;
     case 8:
-      dequant_kernel<8><<<grid_for(rows * wpr, num_sms), 256, 0, s>>>(codes, scale, minv, rows, L, W, wpr, y, aligned);
+      launch_dequant<8>(codes, scale, minv, rows, L, W, wpr, y, aligned, grid_for(rows * wpr, num_sms), s);
       break;
     case 32:
       dequant_passthrough_kernel<<<grid_for(rows * L, num_sms), 256, 0, s>>>(codes, rows, L, W, y);

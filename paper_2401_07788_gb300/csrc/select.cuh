@@ -8,8 +8,9 @@
 // It narrows T down in rounds, each a histogram over bins that are monotone
 // in the key, so that every bin above the chosen one is kept whole and every
 // bin below it is dropped whole:
-//   1. bins linear in |x| between 0 and the row's largest magnitude, which
-//      spreads typical activations over many bins;
+//   1. bins linear in |x| between 0 and the row's largest magnitude (or the
+//      largest of a fixed sample of the row), which spreads typical
+//      activations over many bins; magnitudes above the scale share the top bin;
 //   2. then bins of equal width over the key range [lo, hi] that is left,
 //      256 per round, until one key remains or a bin is taken whole.
 // Keys are int: |x| bit pattern (>= 0), or -1 for a slot past the row end.
@@ -92,6 +93,49 @@ struct Threshold {
   uint32_t need;
 };
 
+// One warp, m <= 64 keys (>= 0) in shared memory: the kr-th largest by
+// counting, for each key, how many keys are larger and how many are at least
+// as large (T is the key with #greater < kr <= #at-least).
+__device__ __forceinline__ Threshold warp_small_select(const int* keys, uint32_t m, uint32_t kr,
+                                                       int lane) {
+  const int k0 = static_cast<uint32_t>(lane) < m ? keys[lane] : -1;
+  const int k1 = static_cast<uint32_t>(lane) + 32u < m ? keys[lane + 32] : -1;
+  uint32_t gt0 = 0, ge0 = 0, gt1 = 0, ge1 = 0;
+  if (m <= 32) {
+#pragma unroll 8
+    for (int j = 0; j < 32; ++j) {
+      const int a = __shfl_sync(kFull, k0, j);
+      gt0 += a > k0;
+      ge0 += a >= k0;
+    }
+  } else {
+#pragma unroll 4
+    for (int j = 0; j < 32; ++j) {
+      const int a = __shfl_sync(kFull, k0, j);
+      const int b = __shfl_sync(kFull, k1, j);
+      gt0 += (a > k0) + (b > k0);
+      ge0 += (a >= k0) + (b >= k0);
+      gt1 += (a > k1) + (b > k1);
+      ge1 += (a >= k1) + (b >= k1);
+    }
+  }
+  const bool ok0 = static_cast<uint32_t>(lane) < m && gt0 < kr && kr <= ge0;
+  const bool ok1 = static_cast<uint32_t>(lane) + 32u < m && gt1 < kr && kr <= ge1;
+  const unsigned b0 = __ballot_sync(kFull, ok0);
+  const unsigned b1 = __ballot_sync(kFull, ok1);
+  Threshold t;
+  if (b0) {
+    const int src = __ffs(b0) - 1;
+    t.T = __shfl_sync(kFull, k0, src);
+    t.need = kr - __shfl_sync(kFull, gt0, src);
+  } else {
+    const int src = b1 ? __ffs(b1) - 1 : 0;
+    t.T = __shfl_sync(kFull, k1, src);
+    t.need = kr - __shfl_sync(kFull, gt1, src);
+  }
+  return t;
+}
+
 // One warp: among m keys (>= 0) in shared memory, find the kr-th largest
 // (1 <= kr <= m) by integer rounds.  whist: 256 words of warp-private scratch.
 __device__ __forceinline__ Threshold warp_list_select(const int* keys, uint32_t m, uint32_t kr,
@@ -134,6 +178,13 @@ __device__ __forceinline__ Threshold warp_list_select(const int* keys, uint32_t 
     lo = nlo;
     hi = nhi;
   }
+}
+
+// One warp: the kr-th largest of m keys in shared memory.
+__device__ __forceinline__ Threshold warp_select(const int* keys, uint32_t m, uint32_t kr,
+                                                 uint32_t* whist, int lane) {
+  if (m <= 64) return warp_small_select(keys, m, kr, lane);
+  return warp_list_select(keys, m, kr, whist, lane);
 }
 
 }  // namespace mpc

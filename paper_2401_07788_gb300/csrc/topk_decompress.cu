@@ -2,11 +2,12 @@
 // at their indices and every other entry is zero) and the AQ-SGD receiver's
 // buffer update (§2.5).
 //
-// Decompression builds each output tile in shared memory (zero fill, scatter
-// of the tile's kept entries) and writes it to HBM once with 16-byte stores.
-// A tile is either several whole rows (short rows) or a column range of one
-// row (long rows); for a column range the kept entries are found by a
-// block-parallel search of the row's ascending indices.
+// Rows of up to 65536 entries: one CTA owns whole rows, zero-fills them with
+// 16-byte stores and, after a block barrier, stores the kept values over the
+// zeros; both writes of a line meet in L2, so HBM sees each output byte once.
+// Longer rows: each output tile is built in shared memory (zero fill, scatter
+// of the tile's kept entries, found by a block-parallel search of the row's
+// ascending indices) and written once.
 #include "common.cuh"
 #include "kernels.h"
 #include "launch_util.h"
@@ -88,6 +89,37 @@ __global__ void __launch_bounds__(kDecThreads)
   }
 }
 
+// Whole rows [r0, r0 + nrows) per CTA (rpc * row_len <= kRowsPerCta entries).
+constexpr int64_t kRowsPerCta = 16384;
+
+__global__ void __launch_bounds__(kDecThreads)
+    topk_decompress_rows_kernel(const float* __restrict__ vals, const int32_t* __restrict__ idx,
+                                int64_t rows, int64_t L, int64_t k, float* __restrict__ y,
+                                int64_t rpc, int aligned) {
+  const int tid = threadIdx.x;
+  const int64_t r0 = static_cast<int64_t>(blockIdx.x) * rpc;
+  const int64_t nrows = min64(rpc, rows - r0);
+  const int64_t cells = nrows * L;
+  float* dst = y + r0 * L;
+  if (aligned) {
+    const int64_t n4 = cells / 4;
+    float4* d4 = reinterpret_cast<float4*>(dst);
+    for (int64_t i = tid; i < n4; i += kDecThreads) d4[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int64_t i = n4 * 4 + tid; i < cells; i += kDecThreads) dst[i] = 0.0f;
+  } else {
+    for (int64_t i = tid; i < cells; i += kDecThreads) dst[i] = 0.0f;
+  }
+  __syncthreads();  // the zeros of this block precede its kept values
+  const int64_t e_begin = r0 * k;
+  const uint32_t nk = static_cast<uint32_t>(nrows * k);  // <= rpc * L <= 65536
+  const uint32_t k32 = static_cast<uint32_t>(k);
+  for (uint32_t e = tid; e < nk; e += kDecThreads) {
+    const uint32_t lr = e / k32;
+    const int64_t col = idx[e_begin + e];
+    if (col >= 0 && col < L) dst[static_cast<int64_t>(lr) * L + col] = vals[e_begin + e];
+  }
+}
+
 // One CTA per logical payload row: buf_recv[s][r][idx] += vals.
 __global__ void __launch_bounds__(kDecThreads)
     aqsgd_decompress_kernel(const float* __restrict__ vals, const int32_t* __restrict__ idx,
@@ -116,6 +148,14 @@ cudaError_t launch_topk_decompress(const float* vals, const int32_t* idx, int64_
                                    cudaStream_t s) {
   (void)num_sms;
   if (rows <= 0) return cudaSuccess;
+  if (L <= 65536) {
+    const int64_t rpc = max64(1, min64(rows, kRowsPerCta / L));
+    const int64_t blocks = (rows + rpc - 1) / rpc;
+    if (blocks > 0x7fffffffLL) return cudaErrorInvalidValue;
+    topk_decompress_rows_kernel<<<static_cast<unsigned>(blocks), kDecThreads, 0, s>>>(
+        vals, idx, rows, L, k, y, rpc, aligned);
+    return cudaGetLastError();
+  }
   int64_t rpc = 1, tpr = 1, blocks;
   if (L <= kTile) {
     rpc = kTile / L;
