@@ -37,6 +37,9 @@ constexpr int64_t kRowPathMaxLen = 65536;
 
 // Launch the on-chip row TopK path.  Returns a CUDA error code.
 cudaError_t launch_topk_rows(int mode, const TopkRowArgs& a, int num_sms, cudaStream_t s);
+cudaError_t launch_topk_rows_plain(const TopkRowArgs& a, int num_sms, cudaStream_t s);
+cudaError_t launch_topk_rows_ef(const TopkRowArgs& a, int num_sms, cudaStream_t s);
+cudaError_t launch_topk_rows_delta(const TopkRowArgs& a, int num_sms, cudaStream_t s);
 
 struct TopkGridArgs {
   const float* x;

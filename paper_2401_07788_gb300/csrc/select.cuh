@@ -93,49 +93,6 @@ struct Threshold {
   uint32_t need;
 };
 
-// One warp, m <= 64 keys (>= 0) in shared memory: the kr-th largest by
-// counting, for each key, how many keys are larger and how many are at least
-// as large (T is the key with #greater < kr <= #at-least).
-__device__ __forceinline__ Threshold warp_small_select(const int* keys, uint32_t m, uint32_t kr,
-                                                       int lane) {
-  const int k0 = static_cast<uint32_t>(lane) < m ? keys[lane] : -1;
-  const int k1 = static_cast<uint32_t>(lane) + 32u < m ? keys[lane + 32] : -1;
-  uint32_t gt0 = 0, ge0 = 0, gt1 = 0, ge1 = 0;
-  if (m <= 32) {
-#pragma unroll 8
-    for (int j = 0; j < 32; ++j) {
-      const int a = __shfl_sync(kFull, k0, j);
-      gt0 += a > k0;
-      ge0 += a >= k0;
-    }
-  } else {
-#pragma unroll 4
-    for (int j = 0; j < 32; ++j) {
-      const int a = __shfl_sync(kFull, k0, j);
-      const int b = __shfl_sync(kFull, k1, j);
-      gt0 += (a > k0) + (b > k0);
-      ge0 += (a >= k0) + (b >= k0);
-      gt1 += (a > k1) + (b > k1);
-      ge1 += (a >= k1) + (b >= k1);
-    }
-  }
-  const bool ok0 = static_cast<uint32_t>(lane) < m && gt0 < kr && kr <= ge0;
-  const bool ok1 = static_cast<uint32_t>(lane) + 32u < m && gt1 < kr && kr <= ge1;
-  const unsigned b0 = __ballot_sync(kFull, ok0);
-  const unsigned b1 = __ballot_sync(kFull, ok1);
-  Threshold t;
-  if (b0) {
-    const int src = __ffs(b0) - 1;
-    t.T = __shfl_sync(kFull, k0, src);
-    t.need = kr - __shfl_sync(kFull, gt0, src);
-  } else {
-    const int src = b1 ? __ffs(b1) - 1 : 0;
-    t.T = __shfl_sync(kFull, k1, src);
-    t.need = kr - __shfl_sync(kFull, gt1, src);
-  }
-  return t;
-}
-
 // One warp: among m keys (>= 0) in shared memory, find the kr-th largest
 // (1 <= kr <= m) by integer rounds.  whist: 256 words of warp-private scratch.
 __device__ __forceinline__ Threshold warp_list_select(const int* keys, uint32_t m, uint32_t kr,
@@ -180,10 +137,55 @@ __device__ __forceinline__ Threshold warp_list_select(const int* keys, uint32_t 
   }
 }
 
+// Rank test of one candidate key ki against the m keys: it is T when fewer than
+// kr keys are larger and at least kr are at least as large; then `need` is
+// kr minus the number larger.
+__device__ __forceinline__ bool rank_is_threshold(const int* keys, uint32_t m, uint32_t kr, int ki,
+                                                  uint32_t* need) {
+  uint32_t gt = 0, ge = 0;
+  uint32_t j = 0;
+  for (; j + 4 <= m; j += 4) {
+    const int a0 = keys[j], a1 = keys[j + 1], a2 = keys[j + 2], a3 = keys[j + 3];
+    gt += (a0 > ki) + (a1 > ki) + (a2 > ki) + (a3 > ki);
+    ge += (a0 >= ki) + (a1 >= ki) + (a2 >= ki) + (a3 >= ki);
+  }
+  for (; j < m; ++j) {
+    const int a0 = keys[j];
+    gt += a0 > ki;
+    ge += a0 >= ki;
+  }
+  *need = kr - gt;
+  return gt < kr && kr <= ge;
+}
+
+// One warp, m <= 64 keys in shared memory: each lane ranks its candidates
+// against all m keys (a loop of length m); the lane holding T reports it.
+__device__ __forceinline__ Threshold warp_rank_select(const int* keys, uint32_t m, uint32_t kr,
+                                                      int lane) {
+  int T = -1;
+  uint32_t need = 0;
+  bool found = false;
+  for (uint32_t i = lane; i < m; i += 32) {
+    uint32_t nd;
+    const int ki = keys[i];
+    if (rank_is_threshold(keys, m, kr, ki, &nd)) {
+      T = ki;
+      need = nd;
+      found = true;
+    }
+  }
+  const unsigned who = __ballot_sync(kFull, found);
+  const int src = who ? __ffs(who) - 1 : 0;
+  Threshold t;
+  t.T = __shfl_sync(kFull, T, src);
+  t.need = __shfl_sync(kFull, need, src);
+  return t;
+}
+
 // One warp: the kr-th largest of m keys in shared memory.
 __device__ __forceinline__ Threshold warp_select(const int* keys, uint32_t m, uint32_t kr,
                                                  uint32_t* whist, int lane) {
-  if (m <= 64) return warp_small_select(keys, m, kr, lane);
+  if (m <= 64) return warp_rank_select(keys, m, kr, lane);
   return warp_list_select(keys, m, kr, whist, lane);
 }
 

@@ -1,0 +1,1064 @@
+// topk_rows.cuh -- exact per-row TopK (§2.3) for rows that fit on chip, fused
+// with error feedback (§2.4, Seide et al.) and with the EF21 / AQ-SGD buffer
+// update (§2.4, §2.5).  Kernel templates; topk_rows_{plain,ef,delta}.cu
+// instantiate them, one fused variant per translation unit.
+//
+// Two kernels share the selection of select.cuh.  Both read x (and the error
+// or state row) from HBM once, keep the ranked values (x, x + err or
+// x - state) in shared memory, write the payload once, write err once (error
+// feedback) or the state at the kept entries only (EF21 / AQ-SGD).
+//
+//  * topk_cta_kernel: rows longer than 1024 entries.  One thread-block cluster
+//    of C CTAs per row, each CTA holding a slice of up to SCAP entries.  The
+//    slice of x arrives by one bulk asynchronous copy completing on an
+//    mbarrier; the error / state slice by 16-byte loads issued at the same
+//    time.  Passes over the slice: ranked values with the histogram, count-and-collect
+//    (entries above the chosen bin are counted per 128-entry chunk, entries in
+//    it are appended to a candidate list), write.  The CTAs of a cluster push
+//    histogram group sums, candidate lists and counts into each other's shared
+//    memory (st.shared::cluster) before a cluster barrier and pull only the few
+//    bins of the chosen group: two cluster barriers per row, none at exit.  The
+//    bin scale comes from a sample of the row that every CTA of the cluster
+//    reads identically, so the histogram is built in the same pass that forms
+//    the ranked values and no barrier is spent on the row maximum.
+//  * topk_warp_kernel: one warp per row for rows of at most 1024 entries,
+//    persistent over rows; each warp double-buffers its rows with its own bulk
+//    copies and mbarriers, so the next row loads while this one is selected.
+//
+// FULL instantiations drop the per-entry end-of-slice checks; they run when
+// every 4-entry slot a thread processes lies inside the slice.
+#pragma once
+
+#include "common.cuh"
+#include "kernels.h"
+#include "launch_util.h"
+#include "select.cuh"
+
+namespace mpc {
+namespace rows {
+
+constexpr int kNB = 2048;     // bins of the first histogram, CTA kernel
+constexpr int kLCAP = 256;    // candidate keys per row, CTA kernel (whole cluster)
+constexpr int kLCAPW = 256;   // candidate keys per row, warp kernel
+constexpr int kMaxCluster = 8;
+constexpr int kSampleThreads = 64;  // threads that read the row sample (4 entries each)
+
+// The value the selection ranks, for each fused variant.
+template <int MODE>
+__device__ __forceinline__ float ranked_value(float x, float a) {
+  if (MODE == kEF) return fadd(x, a);     // s = x + err
+  if (MODE == kDelta) return fsub(x, a);  // d = x - state
+  return x;
+}
+
+template <int MODE>
+__device__ __forceinline__ float4 ranked4(float4 x, float4 a) {
+  return make_float4(ranked_value<MODE>(x.x, a.x), ranked_value<MODE>(x.y, a.y),
+                     ranked_value<MODE>(x.z, a.z), ranked_value<MODE>(x.w, a.w));
+}
+
+// Keys of the 4 entries base..base+3 (-1 past the slice end n, unless FULL).
+template <bool FULL>
+__device__ __forceinline__ void keys4(const float4 v, int base, int n, int k[4]) {
+  if (FULL) {
+    k[0] = mag_key(v.x);
+    k[1] = mag_key(v.y);
+    k[2] = mag_key(v.z);
+    k[3] = mag_key(v.w);
+  } else {
+    k[0] = (base + 0 < n) ? mag_key(v.x) : -1;
+    k[1] = (base + 1 < n) ? mag_key(v.y) : -1;
+    k[2] = (base + 2 < n) ? mag_key(v.z) : -1;
+    k[3] = (base + 3 < n) ? mag_key(v.w) : -1;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Block-level reductions and scans (NT threads)
+// ---------------------------------------------------------------------------
+template <int NT>
+__device__ __forceinline__ int block_max(int v, int* red, int lane, int warp) {
+  v = __reduce_max_sync(kFull, v);
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  int r = red[0];
+#pragma unroll
+  for (int i = 1; i < NT / 32; ++i) r = max(r, red[i]);
+  __syncthreads();
+  return r;
+}
+
+template <int NT>
+__device__ __forceinline__ int block_min(int v, int* red, int lane, int warp) {
+  v = __reduce_min_sync(kFull, v);
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  int r = red[0];
+#pragma unroll
+  for (int i = 1; i < NT / 32; ++i) r = min(r, red[i]);
+  __syncthreads();
+  return r;
+}
+
+template <int NT>
+__device__ __forceinline__ uint32_t block_excl_scan(uint32_t v, uint32_t* red, int lane, int warp) {
+  const uint32_t inc = warp_inclusive_scan(v, lane);
+  if (lane == 31) red[warp] = inc;
+  __syncthreads();
+  uint32_t base = 0;
+#pragma unroll
+  for (int i = 0; i < NT / 32; ++i)
+    if (i < warp) base += red[i];
+  __syncthreads();
+  return base + inc - v;
+}
+
+// ---------------------------------------------------------------------------
+// CTA / cluster kernel
+// ---------------------------------------------------------------------------
+template <int NT, int SCAP>
+struct CtaShared {
+  static constexpr int NW = NT / 32;
+  static constexpr int NCH = SCAP / 128;  // chunks of 128 consecutive entries
+  uint32_t hist[kNB];
+  uint32_t rhist[2][kRoundBins];
+  int lkey[kLCAP];       // this CTA's candidate keys
+  uint16_t lch[kLCAP];   // and their chunks
+  int sel[kLCAP];        // the row's candidate keys (all CTAs), contiguous
+  uint32_t cgt[NCH];     // per chunk: entries kept for being above T
+  uint32_t ceq[NCH];     // per chunk: entries equal to T
+  uint32_t gbins[128];
+  uint32_t tot_gt[kMaxCluster];  // pushed by the lower ranks of the cluster
+  uint32_t tot_eq[kMaxCluster];
+  uint32_t gcnt[kMaxCluster];    // candidates of each CTA (pushed)
+  uint32_t gcab[kMaxCluster];    // entries above the chosen bin in each CTA (pushed)
+  int red[NW];
+  uint32_t ured[NW];
+  int sample_max[2];
+  uint32_t lcount;
+  uint32_t pick_t, pick_excl;
+  uint32_t before_gt, before_eq;
+  int pub_lo, pub_hi;
+  BinPick pick;
+  Threshold thr;
+  uint64_t bar;
+};
+
+// The bin holding the kr-th element of an NBINS-bin histogram (bins ranked
+// high to low) summed over the cluster's C CTAs.  Each thread owns a group of
+// G consecutive bins; group sums are pushed to every CTA (table `gsum`,
+// C x NT words), scanned locally, and only the chosen group's bins are pulled
+// from the other CTAs.
+template <int NT, int NBINS, class Sh>
+__device__ __forceinline__ BinPick cluster_pick(const uint32_t* hist, uint32_t* gsum, uint32_t C,
+                                                uint32_t crank, uint32_t kr, Sh& sh, int tid,
+                                                int lane, int warp) {
+  constexpr int G = NBINS / NT;
+  static_assert(G * NT == NBINS && G * kMaxCluster <= 128, "bin groups");
+  uint32_t gs = 0;
+#pragma unroll
+  for (int b = 0; b < G; ++b) gs += hist[NBINS - 1 - (tid * G + b)];
+  uint32_t total = gs;
+  if (C > 1) {
+    uint32_t* mine = gsum + crank * NT + tid;
+    for (uint32_t r = 0; r < C; ++r) dsmem_st_u32(dsmem_addr(mine, r), gs);
+    cluster_sync();
+    total = 0;
+    for (uint32_t r = 0; r < C; ++r) total += gsum[r * NT + tid];
+  }
+  if (tid == 0) {
+    sh.pick_t = 0;
+    sh.pick_excl = 0;
+  }
+  const uint32_t excl = block_excl_scan<NT>(total, sh.ured, lane, warp);
+  if (excl < kr && kr <= excl + total) {
+    sh.pick_t = tid;
+    sh.pick_excl = excl;
+  }
+  __syncthreads();
+  const uint32_t tg = sh.pick_t;
+  if (tid < G * static_cast<int>(C)) {
+    const int r = tid / G, b = tid % G;
+    const uint32_t* p = &hist[NBINS - 1 - (tg * G + b)];
+    sh.gbins[tid] = (C > 1) ? dsmem_ld_u32(dsmem_addr(p, r)) : *p;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    uint32_t run = sh.pick_excl;
+    BinPick pk = {NBINS - 1 - static_cast<int>(tg * G), run, 0};
+    for (int b = 0; b < G; ++b) {
+      uint32_t cnt = 0;
+      for (uint32_t r = 0; r < C; ++r) cnt += sh.gbins[r * G + b];
+      pk = BinPick{NBINS - 1 - static_cast<int>(tg * G + b), run, cnt};
+      if (run + cnt >= kr) break;
+      run += cnt;
+    }
+    sh.pick = pk;
+  }
+  __syncthreads();
+  return sh.pick;
+}
+
+// Warp 0: exclusive scan of the per-chunk counts in place; returns the totals
+// on lane 31.
+template <int NCH>
+__device__ __forceinline__ void scan_chunks(uint32_t* cgt, uint32_t* ceq, int lane,
+                                            uint32_t* tot_g, uint32_t* tot_e) {
+  constexpr int PER = (NCH + 31) / 32;
+  uint32_t g[PER], e[PER], tg = 0, te = 0;
+#pragma unroll
+  for (int j = 0; j < PER; ++j) {
+    const int ch = lane * PER + j;
+    g[j] = ch < NCH ? cgt[ch] : 0u;
+    e[j] = ch < NCH ? ceq[ch] : 0u;
+    tg += g[j];
+    te += e[j];
+  }
+  uint32_t eg = warp_inclusive_scan(tg, lane) - tg;
+  uint32_t ee = warp_inclusive_scan(te, lane) - te;
+#pragma unroll
+  for (int j = 0; j < PER; ++j) {
+    const int ch = lane * PER + j;
+    if (ch < NCH) {
+      cgt[ch] = eg;
+      ceq[ch] = ee;
+    }
+    eg += g[j];
+    ee += e[j];
+  }
+  *tot_g = eg;
+  *tot_e = ee;
+}
+
+// Bytes of dynamic shared memory of the CTA kernel for cluster size C.
+constexpr int cta_smem_bytes(int NT, int SCAP, int C) {
+  return SCAP * 4 + C * NT * 4 + C * (kLCAP > NT ? kLCAP : NT) * 4;
+}
+
+template <int MODE, int NT, int SCAP, bool FULL>
+__global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const TopkRowArgs a) {
+  constexpr int NW = NT / 32;
+  constexpr int NQ = SCAP / 4;     // float4 slots per slice
+  constexpr int QPT = NQ / NT;     // float4 slots per thread
+  constexpr int NCH = SCAP / 128;  // 128-entry chunks per slice
+  constexpr int GB = kLCAP > NT ? kLCAP : NT;
+  using Sh = CtaShared<NT, SCAP>;
+  __shared__ Sh sh;
+  extern __shared__ __align__(16) float4 dyn4[];
+
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const uint32_t C = cluster_size();
+  const uint32_t crank = cluster_rank();
+  float4* s4 = dyn4;                                         // NQ float4: ranked values
+  uint32_t* gsumA = reinterpret_cast<uint32_t*>(dyn4 + NQ);  // C x NT group sums
+  uint32_t* gB = gsumA + C * NT;  // C x GB: pushed candidate lists, or group sums of a round
+  const int64_t row = blockIdx.x / C;
+  const int64_t L = a.L;
+  const int64_t k = a.k;
+  const int64_t c0 = static_cast<int64_t>(crank) * a.slice;
+  const int n = static_cast<int>(max64(0, min64(a.slice, L - c0)));
+
+  // Row of the error (EF) or state (EF21 / AQ-SGD) buffer.  Every CTA of the
+  // cluster reads the same id, so all of them leave together, before any
+  // cluster barrier.
+  float* arow = nullptr;
+  if (MODE != kPlain) {
+    int64_t srow = row;
+    if (MODE == kDelta && a.ids != nullptr) {
+      const int64_t sid = a.ids[row / a.rps];
+      if (sid < 0 || sid >= a.num_samples) {
+        if (tid == 0 && crank == 0) set_status(a.status, STATUS_BAD_SAMPLE);
+        return;
+      }
+      srow = sid * a.rps + row % a.rps;
+    }
+    arow = a.aux + srow * L;
+  }
+  const float* xrow = a.x + row * L;
+
+  // ---- issue the loads: x by bulk copy, a sample of the row, err / state ----
+  bool failed = false;
+  if (a.aligned) {
+    if (tid == 0) {
+      mbar_init(&sh.bar, 1);
+      fence_mbar_init();
+    }
+    __syncthreads();
+    if (tid == 0 && n > 0) {
+      const uint32_t bytes = static_cast<uint32_t>(n) * 4u;
+      mbar_arrive_expect_tx(&sh.bar, bytes);
+      bulk_g2s(s4, xrow + c0, bytes, &sh.bar);
+    }
+  }
+  // The bin scale comes from a sample of the row, entries [p, p+4) spread over
+  // it, read identically by every CTA of the cluster.
+  float smp[4] = {0.f, 0.f, 0.f, 0.f};
+  const int64_t sp = (L / kSampleThreads) * tid / 4 * 4;
+  if (tid < kSampleThreads) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+      if (sp + i < L)
+        smp[i] = ranked_value<MODE>(xrow[sp + i], (MODE != kPlain) ? arow[sp + i] : 0.0f);
+  }
+  float4 av[QPT];
+  if (a.aligned && MODE != kPlain) {
+#pragma unroll
+    for (int j = 0; j < QPT; ++j) {
+      const int q = j * NT + tid;
+      av[j] = (4 * q < n) ? *reinterpret_cast<const float4*>(arow + c0 + 4 * q)
+                          : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+  }
+  for (int i = tid; i < kNB; i += NT) sh.hist[i] = 0;
+  if (tid == 0) {
+    sh.lcount = 0;
+    sh.thr = Threshold{0x7fffffff, 0};
+  }
+  if (tid < kSampleThreads) {
+    int smax = -1;
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+      if (sp + i < L) smax = max(smax, mag_key(smp[i]));
+    smax = __reduce_max_sync(kFull, smax);
+    if (lane == 0) sh.sample_max[warp] = smax;
+  }
+
+  if (a.aligned) {
+    if (n > 0 && !mbar_wait_bounded(&sh.bar, 0, a.spin_limit, a.status)) {
+      mbar_wait_bounded(&sh.bar, 0, kDrainPolls, nullptr);
+      failed = true;
+    }
+    failed = __syncthreads_or(failed);
+  } else {
+    float* s = reinterpret_cast<float*>(s4);
+    for (int e = tid; e < n; e += NT)
+      s[e] = ranked_value<MODE>(xrow[c0 + e], (MODE != kPlain) ? arow[c0 + e] : 0.0f);
+    __syncthreads();
+  }
+  const int nv = failed ? 0 : n;  // a failed slice takes part as an empty one
+  const int jmax = (nv + 4 * NT - 1) / (4 * NT);  // float4 slots of each thread in use
+  const float scale = bucket_scale(max(sh.sample_max[0], sh.sample_max[1]), kNB);
+  const bool binned = k < L && scale > 0.0f;
+
+  // ---- ranked values into shared memory and the first histogram -------------
+  uint32_t zc = 0;
+#pragma unroll
+  for (int j = 0; j < QPT; ++j) {
+    if (j < jmax) {
+      const int q = j * NT + tid;
+      float4 v = s4[q];
+      if (MODE != kPlain && a.aligned) {
+        v = ranked4<MODE>(v, av[j]);
+        s4[q] = v;
+      }
+      if (binned) {
+        int kk[4];
+        keys4<FULL>(v, 4 * q, nv, kk);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          if (kk[i] == 0) ++zc;
+          else if (kk[i] > 0) atomicAdd(&sh.hist[bucket_of(kk[i], scale, kNB)], 1u);
+        }
+      }
+    }
+  }
+  if (binned) {
+    zc = __reduce_add_sync(kFull, zc);
+    if (lane == 0 && zc) atomicAdd(&sh.hist[0], zc);
+  }
+  __syncthreads();
+
+  // ---- select T and need -----------------------------------------------------
+  int T = -1;
+  uint32_t need = 0;
+  bool counted = false;  // per-chunk counts and the counts of earlier CTAs are in place
+  uint32_t gt_before = 0, eq_before = 0;
+  if (k < L) {
+    uint32_t kr = static_cast<uint32_t>(k);
+    int B = 0;
+    uint32_t m = static_cast<uint32_t>(L);  // with scale 0 every entry is a candidate
+    if (scale > 0.0f) {
+      const BinPick p = cluster_pick<NT, kNB>(sh.hist, gsumA, C, crank, kr, sh, tid, lane, warp);
+      B = p.bin;
+      kr -= p.above;
+      m = p.count;
+    }
+
+    if (scale > 0.0f && m <= static_cast<uint32_t>(kLCAP)) {
+      // ---- count and collect: entries above bin B are kept; the m entries
+      // in it are the candidates for T ---------------------------------------
+#pragma unroll 2
+      for (int j = 0; j < QPT; ++j) {
+        uint32_t ab = 0;
+        if (j < jmax) {
+          const int q = j * NT + tid;
+          int kk[4];
+          keys4<FULL>(s4[q], 4 * q, nv, kk);
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            if (FULL || kk[i] >= 0) {
+              const int b = bucket_of(kk[i], scale, kNB);
+              ab += b > B;
+              if (b == B) {
+                const uint32_t at = atomicAdd(&sh.lcount, 1u);
+                if (at < kLCAP) {
+                  sh.lkey[at] = kk[i];
+                  sh.lch[at] = static_cast<uint16_t>(j * NW + warp);
+                }
+              }
+            }
+          }
+          ab = __reduce_add_sync(kFull, ab);
+        }
+        if (lane == 0) {
+          sh.cgt[j * NW + warp] = ab;
+          sh.ceq[j * NW + warp] = 0;
+        }
+      }
+      __syncthreads();
+      const uint32_t lc = min(sh.lcount, static_cast<uint32_t>(kLCAP));
+      const int* list = sh.lkey;
+      uint32_t mt = lc;
+      if (C > 1) {
+        // push this CTA's candidates and its above-bin count to every CTA
+        if (warp == 0) {
+          uint32_t cab = 0;
+          for (int ch = lane; ch < NCH; ch += 32) cab += sh.cgt[ch];
+          cab = __reduce_add_sync(kFull, cab);
+          if (lane == 0)
+            for (uint32_t r = 0; r < C; ++r) {
+              dsmem_st_u32(dsmem_addr(&sh.gcnt[crank], r), lc);
+              dsmem_st_u32(dsmem_addr(&sh.gcab[crank], r), cab);
+            }
+        }
+        for (uint32_t p = tid; p < lc; p += NT) {
+          const uint32_t key = static_cast<uint32_t>(sh.lkey[p]);
+          uint32_t* slot = gB + crank * GB + p;
+          for (uint32_t r = 0; r < C; ++r) dsmem_st_u32(dsmem_addr(slot, r), key);
+        }
+        cluster_sync();  // the last cluster barrier: nothing is read remotely after it
+        uint32_t off = 0;
+        for (uint32_t r = 0; r < C; ++r) {
+          const uint32_t cnt = sh.gcnt[r];
+          for (uint32_t p = tid; p < cnt && off + p < kLCAP; p += NT)
+            sh.sel[off + p] = static_cast<int>(gB[r * GB + p]);
+          off += cnt;
+        }
+        __syncthreads();
+        list = sh.sel;
+        mt = min(off, static_cast<uint32_t>(kLCAP));
+      }
+      // every thread ranks its candidates against the whole list; the
+      // thread holding T reports it (all such threads report the same values)
+      for (uint32_t i = tid; i < mt; i += NT) {
+        uint32_t nd;
+        const int ki = list[i];
+        if (rank_is_threshold(list, mt, kr, ki, &nd)) sh.thr = Threshold{ki, nd};
+      }
+      __syncthreads();
+      T = sh.thr.T;
+      need = sh.thr.need;
+      // candidates above T, or equal to it, join their chunks' counts
+      for (uint32_t p = tid; p < lc; p += NT) {
+        const int key = sh.lkey[p];
+        if (key > T) atomicAdd(&sh.cgt[sh.lch[p]], 1u);
+        else if (key == T) atomicAdd(&sh.ceq[sh.lch[p]], 1u);
+      }
+      if (C > 1 && warp == 0) {
+        // kept entries of the earlier CTAs of the row
+        uint32_t gb = 0, eb = 0;
+        for (uint32_t r = 0; r < crank; ++r) {
+          if (lane == 0) gb += sh.gcab[r];
+          const uint32_t cnt = sh.gcnt[r];
+          for (uint32_t p = lane; p < cnt; p += 32) {
+            const int key = static_cast<int>(gB[r * GB + p]);
+            gb += key > T;
+            eb += key == T;
+          }
+        }
+        gb = __reduce_add_sync(kFull, gb);
+        eb = __reduce_add_sync(kFull, eb);
+        if (lane == 0) {
+          sh.before_gt = gb;
+          sh.before_eq = eb;
+        }
+      }
+      __syncthreads();
+      if (warp == 0) {
+        uint32_t tg, te;
+        scan_chunks<NCH>(sh.cgt, sh.ceq, lane, &tg, &te);
+      }
+      __syncthreads();
+      if (C > 1) {
+        gt_before = sh.before_gt;
+        eq_before = sh.before_eq;
+      }
+      counted = true;
+    } else {
+      // ---- too many candidates for the list: integer rounds over the slice --
+      int lo = 0x7fffffff, hi = -1;
+#pragma unroll 2
+      for (int j = 0; j < jmax; ++j) {
+        const int q = j * NT + tid;
+        int kk[4];
+        keys4<FULL>(s4[q], 4 * q, nv, kk);
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+          if (kk[i] >= 0 && (scale == 0.0f || bucket_of(kk[i], scale, kNB) == B)) {
+            lo = min(lo, kk[i]);
+            hi = max(hi, kk[i]);
+          }
+      }
+      lo = block_min<NT>(lo, sh.red, lane, warp);
+      hi = block_max<NT>(hi, sh.red, lane, warp);
+      if (C > 1) {
+        if (tid == 0) {
+          sh.pub_lo = lo;
+          sh.pub_hi = hi;
+        }
+        cluster_sync();
+        for (uint32_t r = 0; r < C; ++r) {
+          lo = min(lo, dsmem_ld_s32(dsmem_addr(&sh.pub_lo, r)));
+          hi = max(hi, dsmem_ld_s32(dsmem_addr(&sh.pub_hi, r)));
+        }
+      }
+      int p = 0;
+      for (;;) {
+        if (lo >= hi) {
+          T = lo;
+          need = kr;
+          break;
+        }
+        const int sft = round_shift(lo, hi);
+        for (int i = tid; i < kRoundBins; i += NT) sh.rhist[p][i] = 0;
+        __syncthreads();
+#pragma unroll 2
+        for (int j = 0; j < jmax; ++j) {
+          const int q = j * NT + tid;
+          int kk[4];
+          keys4<FULL>(s4[q], 4 * q, nv, kk);
+#pragma unroll
+          for (int i = 0; i < 4; ++i)
+            if (kk[i] >= lo && kk[i] <= hi)
+              atomicAdd(&sh.rhist[p][static_cast<uint32_t>(kk[i] - lo) >> sft], 1u);
+        }
+        __syncthreads();
+        // the group-sum table alternates from round to round, so a push never
+        // lands on sums another CTA may still be reading
+        const BinPick q = cluster_pick<NT, kRoundBins>(sh.rhist[p], p == 0 ? gB : gsumA, C,
+                                                       crank, kr, sh, tid, lane, warp);
+        kr -= q.above;
+        const int nlo = lo + (q.bin << sft);
+        const int nhi = static_cast<int>(
+            min(static_cast<uint32_t>(hi), static_cast<uint32_t>(nlo) + ((1u << sft) - 1u)));
+        if (q.count == kr) {
+          T = nlo - 1;
+          need = 0;
+          break;
+        }
+        lo = nlo;
+        hi = nhi;
+        p ^= 1;
+      }
+    }
+  }
+
+  if (!counted) {
+    // ---- count kept entries per 128-entry chunk ------------------------------
+#pragma unroll 2
+    for (int j = 0; j < QPT; ++j) {
+      uint32_t g = 0, e = 0;
+      if (j < jmax) {
+        const int q = j * NT + tid;
+        int kk[4];
+        keys4<FULL>(s4[q], 4 * q, nv, kk);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          g += kk[i] > T;
+          e += kk[i] == T;
+        }
+        g = __reduce_add_sync(kFull, g);
+        e = need ? __reduce_add_sync(kFull, e) : 0u;
+      }
+      if (lane == 0) {
+        sh.cgt[j * NW + warp] = g;
+        sh.ceq[j * NW + warp] = e;
+      }
+    }
+    __syncthreads();
+    if (warp == 0) {
+      uint32_t tg, te;
+      scan_chunks<NCH>(sh.cgt, sh.ceq, lane, &tg, &te);
+      if (C > 1 && lane == 31) {
+        // push this slice's totals to every later CTA of the row
+        for (uint32_t r = crank + 1; r < C; ++r) {
+          dsmem_st_u32(dsmem_addr(&sh.tot_gt[crank], r), tg);
+          dsmem_st_u32(dsmem_addr(&sh.tot_eq[crank], r), te);
+        }
+      }
+    }
+    if (C > 1) {
+      cluster_sync();  // the last cluster barrier: nothing is read remotely after it
+      for (uint32_t r = 0; r < crank; ++r) {
+        gt_before += sh.tot_gt[r];
+        eq_before += sh.tot_eq[r];
+      }
+    } else {
+      __syncthreads();
+    }
+  }
+
+  // ---- write the payload (ascending column) and the buffers -----------------
+  float* vrow = a.vals + row * k;
+  int32_t* irow = a.idx + row * k;
+  const unsigned lt = lanemask_lt();
+#pragma unroll 2
+  for (int j = 0; j < jmax; ++j) {
+    const int ch = j * NW + warp;
+    const int q = j * NT + tid;
+    const float4 v4 = s4[q];
+    int kk[4];
+    keys4<FULL>(v4, 4 * q, nv, kk);
+    const uint32_t eqt = eq_before + sh.ceq[ch];
+    uint32_t pos = gt_before + sh.cgt[ch] + min(need, eqt);
+    bool kp[4];
+    if (need) {
+      uint32_t r = eqt;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) r += __popc(__ballot_sync(kFull, kk[i] == T) & lt);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const bool e = kk[i] == T;
+        kp[i] = kk[i] > T || (e && r < need);
+        r += e;
+      }
+    } else {
+#pragma unroll
+      for (int i = 0; i < 4; ++i) kp[i] = kk[i] > T;
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) pos += __popc(__ballot_sync(kFull, kp[i]) & lt);
+    const int e0 = 4 * q;
+    if (!FULL && e0 >= nv) continue;
+    const float val[4] = {v4.x, v4.y, v4.z, v4.w};
+    const int col = static_cast<int>(c0) + e0;
+    for (uint32_t bits = (kp[0] ? 1u : 0u) | (kp[1] ? 2u : 0u) | (kp[2] ? 4u : 0u) |
+                         (kp[3] ? 8u : 0u);
+         bits; bits &= bits - 1u, ++pos) {
+      const int i = __ffs(bits) - 1;
+      const float vi = i == 0 ? val[0] : i == 1 ? val[1] : i == 2 ? val[2] : val[3];
+      if (pos < static_cast<uint64_t>(k)) {
+        vrow[pos] = vi;
+        irow[pos] = col + i;
+      }
+      if (MODE == kDelta) {
+        // state + d, against the same state value d was formed from
+        float* sp = arow + col + i;
+        *sp = fadd(*sp, vi);
+      }
+    }
+    if (MODE == kEF) {
+      const float ne[4] = {kp[0] ? 0.0f : val[0], kp[1] ? 0.0f : val[1], kp[2] ? 0.0f : val[2],
+                           kp[3] ? 0.0f : val[3]};
+      if (a.aligned && (FULL || e0 + 4 <= nv)) {
+        *reinterpret_cast<float4*>(arow + col) = make_float4(ne[0], ne[1], ne[2], ne[3]);
+      } else {
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+          if (e0 + i < nv) arow[col + i] = ne[i];
+      }
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Warp-per-row kernel (rows of at most 128 * NVW entries, WPC warps per CTA)
+// ---------------------------------------------------------------------------
+struct WarpShared {
+  uint32_t hist[kRoundBins];
+  int lkey[kLCAPW];
+  uint32_t lcount;
+  uint64_t bar[2];
+};
+
+// Row of the error / state buffer for a logical row (nullptr for plain TopK);
+// *ok = false for an AQ-SGD sample id out of range.
+template <int MODE>
+__device__ __forceinline__ float* state_row(const TopkRowArgs& a, int64_t row, bool* ok) {
+  *ok = true;
+  if (MODE == kPlain) return nullptr;
+  int64_t srow = row;
+  if (MODE == kDelta && a.ids != nullptr) {
+    const int64_t sid = a.ids[row / a.rps];
+    if (sid < 0 || sid >= a.num_samples) {
+      *ok = false;
+      return nullptr;
+    }
+    srow = sid * a.rps + row % a.rps;
+  }
+  return a.aux + srow * a.L;
+}
+
+template <int MODE, int NVW, int WPC, bool FULL>
+__global__ void __launch_bounds__(32 * WPC) topk_warp_kernel(const TopkRowArgs a) {
+  constexpr int RCAP = 128 * NVW;
+  constexpr int NBUF = (MODE == kPlain) ? 1 : 2;  // x (+ err / state) per row
+  __shared__ WarpShared wsh[WPC];
+  extern __shared__ __align__(16) float dyn[];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  WarpShared& sh = wsh[warp];
+  float* wbase = dyn + warp * (2 * RCAP * NBUF);  // two row buffers (double buffering)
+  const int64_t L = a.L;
+  const int64_t k = a.k;
+  const int n = static_cast<int>(L);
+  const unsigned lt = lanemask_lt();
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * WPC;
+  const uint32_t bytes = static_cast<uint32_t>(n) * 4u;
+
+  if (a.aligned && lane == 0) {
+    mbar_init(&sh.bar[0], 1);
+    mbar_init(&sh.bar[1], 1);
+    fence_mbar_init();
+  }
+  __syncwarp();
+
+  // Start the bulk copies of one row into buffer b; returns false (and does
+  // nothing) for a row whose sample id is out of range.
+  auto issue = [&](int64_t r, int b) -> bool {
+    bool ok;
+    float* ar = state_row<MODE>(a, r, &ok);
+    if (!ok) return false;
+    if (lane == 0) {
+      float* buf = wbase + b * (RCAP * NBUF);
+      fence_proxy_async_smem();
+      mbar_arrive_expect_tx(&sh.bar[b], bytes * NBUF);
+      bulk_g2s(buf, a.x + r * L, bytes, &sh.bar[b]);
+      if (MODE != kPlain) bulk_g2s(buf + RCAP, ar, bytes, &sh.bar[b]);
+    }
+    return true;
+  };
+
+  int64_t row = static_cast<int64_t>(blockIdx.x) * WPC + warp;
+  uint32_t phases = 0u;  // bit b: parity of buffer b's next phase
+  uint32_t live = 0u;    // bit b: a copy into buffer b is in flight
+  int b = 0;
+  if (a.aligned && row < a.rows && issue(row, 0)) live |= 1u;
+  for (; row < a.rows; row += stride, b ^= 1) {
+    const int64_t next = row + stride;
+    if (a.aligned && next < a.rows) {
+      if (issue(next, b ^ 1)) live |= 2u >> b;
+      else live &= ~(2u >> b);
+    }
+    bool ok;
+    float* arow = state_row<MODE>(a, row, &ok);
+    if (!ok) {
+      if (lane == 0) set_status(a.status, STATUS_BAD_SAMPLE);
+      continue;
+    }
+    float* xs = wbase + b * (RCAP * NBUF);
+    float* as = xs + RCAP;
+    if (a.aligned) {
+      const uint32_t par = (phases >> b) & 1u;
+      const bool got = mbar_wait_bounded(&sh.bar[b], par, a.spin_limit, a.status);
+      if (__any_sync(kFull, !got)) {
+        // give up on the remaining rows; drain the copies this warp started
+        mbar_wait_bounded(&sh.bar[b], par, kDrainPolls, nullptr);
+        if (next < a.rows && ((live >> (b ^ 1)) & 1u))
+          mbar_wait_bounded(&sh.bar[b ^ 1], (phases >> (b ^ 1)) & 1u, kDrainPolls, nullptr);
+        break;
+      }
+      phases ^= 1u << b;
+    } else {
+      const float* xrow = a.x + row * L;
+      for (int e = lane; e < n; e += 32) {
+        xs[e] = xrow[e];
+        if (MODE != kPlain) as[e] = arow[e];
+      }
+      __syncwarp();
+    }
+    float4* x4 = reinterpret_cast<float4*>(xs);
+    const float4* a4 = reinterpret_cast<const float4*>(as);
+
+    // ---- ranked values (in place) and the row maximum ----------------------
+    int kmax = -1;
+#pragma unroll
+    for (int v = 0; v < NVW; ++v) {
+      const int q = v * 32 + lane;
+      float4 val = x4[q];
+      if (MODE != kPlain) {
+        val = ranked4<MODE>(val, a4[q]);
+        x4[q] = val;
+      }
+      int kk[4];
+      keys4<FULL>(val, 4 * q, n, kk);
+      kmax = max(kmax, max(max(kk[0], kk[1]), max(kk[2], kk[3])));
+    }
+    kmax = __reduce_max_sync(kFull, kmax);
+
+    // ---- select ---------------------------------------------------------------
+    Threshold t;
+    if (k >= L) {
+      t.T = -1;
+      t.need = 0;
+    } else {
+      const float scale = bucket_scale(kmax, kRoundBins);
+      uint32_t kr = static_cast<uint32_t>(k);
+      int B = 0;
+      uint32_t m = static_cast<uint32_t>(n);  // with scale 0 every entry is a candidate
+      if (scale > 0.0f) {
+#pragma unroll
+        for (int j = 0; j < 8; ++j) sh.hist[lane * 8 + j] = 0;
+        if (lane == 0) sh.lcount = 0;
+        __syncwarp();
+        uint32_t zc = 0;
+#pragma unroll
+        for (int v = 0; v < NVW; ++v) {
+          const int q = v * 32 + lane;
+          int kk[4];
+          keys4<FULL>(x4[q], 4 * q, n, kk);
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            if (kk[i] == 0) ++zc;
+            else if (kk[i] > 0) atomicAdd(&sh.hist[bucket_of(kk[i], scale, kRoundBins)], 1u);
+          }
+        }
+        zc = __reduce_add_sync(kFull, zc);
+        if (lane == 0 && zc) atomicAdd(&sh.hist[0], zc);
+        __syncwarp();
+        const BinPick p = warp_pick_bin(sh.hist, kr, lane);
+        __syncwarp();
+        B = p.bin;
+        kr -= p.above;
+        m = p.count;
+      }
+      if (scale > 0.0f && m <= static_cast<uint32_t>(kLCAPW)) {
+        // the candidates are the m entries in bin B, appended where they occur
+#pragma unroll
+        for (int v = 0; v < NVW; ++v) {
+          const int q = v * 32 + lane;
+          int kk[4];
+          keys4<FULL>(x4[q], 4 * q, n, kk);
+#pragma unroll
+          for (int i = 0; i < 4; ++i)
+            if ((FULL || kk[i] >= 0) && bucket_of(kk[i], scale, kRoundBins) == B) {
+              const uint32_t at = atomicAdd(&sh.lcount, 1u);
+              if (at < kLCAPW) sh.lkey[at] = kk[i];
+            }
+        }
+        __syncwarp();
+        t = warp_select(sh.lkey, min(sh.lcount, static_cast<uint32_t>(kLCAPW)), kr, sh.hist, lane);
+      } else {
+        int lo = 0x7fffffff, hi = -1;
+#pragma unroll
+        for (int v = 0; v < NVW; ++v) {
+          const int q = v * 32 + lane;
+          int kk[4];
+          keys4<FULL>(x4[q], 4 * q, n, kk);
+#pragma unroll
+          for (int i = 0; i < 4; ++i)
+            if (kk[i] >= 0 && (scale == 0.0f || bucket_of(kk[i], scale, kRoundBins) == B)) {
+              lo = min(lo, kk[i]);
+              hi = max(hi, kk[i]);
+            }
+        }
+        lo = __reduce_min_sync(kFull, lo);
+        hi = __reduce_max_sync(kFull, hi);
+        for (;;) {
+          if (lo >= hi) {
+            t.T = lo;
+            t.need = kr;
+            break;
+          }
+          const int sft = round_shift(lo, hi);
+#pragma unroll
+          for (int j = 0; j < 8; ++j) sh.hist[lane * 8 + j] = 0;
+          __syncwarp();
+#pragma unroll
+          for (int v = 0; v < NVW; ++v) {
+            const int q = v * 32 + lane;
+            int kk[4];
+            keys4<FULL>(x4[q], 4 * q, n, kk);
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+              if (kk[i] >= lo && kk[i] <= hi)
+                atomicAdd(&sh.hist[static_cast<uint32_t>(kk[i] - lo) >> sft], 1u);
+          }
+          __syncwarp();
+          const BinPick q = warp_pick_bin(sh.hist, kr, lane);
+          __syncwarp();
+          kr -= q.above;
+          const int nlo = lo + (q.bin << sft);
+          const int nhi = static_cast<int>(
+              min(static_cast<uint32_t>(hi), static_cast<uint32_t>(nlo) + ((1u << sft) - 1u)));
+          if (q.count == kr) {
+            t.T = nlo - 1;
+            t.need = 0;
+            break;
+          }
+          lo = nlo;
+          hi = nhi;
+        }
+      }
+    }
+    const int T = t.T;
+    const uint32_t need = t.need;
+
+    // ---- write (one pass: the warp owns the whole row) ------------------------
+    float* vrow = a.vals + row * k;
+    int32_t* irow = a.idx + row * k;
+    uint32_t pos = 0, eq_seen = 0;
+#pragma unroll
+    for (int v = 0; v < NVW; ++v) {
+      const int q = v * 32 + lane;
+      const float4 v4 = x4[q];
+      int kk[4];
+      keys4<FULL>(v4, 4 * q, n, kk);
+      bool kp[4];
+      if (need) {
+        uint32_t r = eq_seen;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const unsigned be = __ballot_sync(kFull, kk[i] == T);
+          r += __popc(be & lt);
+          eq_seen += __popc(be);
+        }
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const bool e = kk[i] == T;
+          kp[i] = kk[i] > T || (e && r < need);
+          r += e;
+        }
+      } else {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) kp[i] = kk[i] > T;
+      }
+      uint32_t p = pos;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const unsigned bk = __ballot_sync(kFull, kp[i]);
+        p += __popc(bk & lt);
+        pos += __popc(bk);
+      }
+      const int e0 = 4 * q;
+      if (FULL || e0 < n) {
+        const float val[4] = {v4.x, v4.y, v4.z, v4.w};
+        float st[4] = {0.f, 0.f, 0.f, 0.f};
+        if (MODE == kDelta) {
+          const float4 sv = a4[q];
+          st[0] = sv.x;
+          st[1] = sv.y;
+          st[2] = sv.z;
+          st[3] = sv.w;
+        }
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          if (kp[i]) {
+            if (p < static_cast<uint64_t>(k)) {
+              vrow[p] = val[i];
+              irow[p] = e0 + i;
+            }
+            if (MODE == kDelta) arow[e0 + i] = fadd(st[i], val[i]);
+            ++p;
+          }
+        }
+        if (MODE == kEF) {
+          const float ne[4] = {kp[0] ? 0.0f : val[0], kp[1] ? 0.0f : val[1],
+                               kp[2] ? 0.0f : val[2], kp[3] ? 0.0f : val[3]};
+          if (a.aligned && (FULL || e0 + 4 <= n)) {
+            *reinterpret_cast<float4*>(arow + e0) = make_float4(ne[0], ne[1], ne[2], ne[3]);
+          } else {
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+              if (e0 + i < n) arow[e0 + i] = ne[i];
+          }
+        }
+      }
+    }
+    __syncwarp();  // this buffer is free for the bulk copy of a later row
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Host-side launch
+// ---------------------------------------------------------------------------
+template <int MODE, int NVW, bool FULL>
+cudaError_t run_warp(const TopkRowArgs& a, int num_sms, cudaStream_t s) {
+  // Eight warps per CTA, four when a warp's two row buffers exceed 12 KiB.
+  constexpr int NBUF = (MODE == kPlain) ? 1 : 2;
+  constexpr int WBYTES = 2 * 128 * NVW * 4 * NBUF;
+  constexpr int WPC = WBYTES > 12 * 1024 ? 4 : 8;
+  auto kernel = topk_warp_kernel<MODE, NVW, WPC, FULL>;
+  const int smem = WPC * WBYTES;
+  cudaError_t err = ensure_dynamic_smem(kernel, smem);
+  if (err != cudaSuccess) return err;
+  const int occ = resident_blocks(kernel, 32 * WPC, smem);
+  const int64_t want = (a.rows + WPC - 1) / WPC;
+  const int64_t cap = static_cast<int64_t>(num_sms) * occ;
+  const int blocks = static_cast<int>(want < cap ? want : cap);
+  kernel<<<blocks, 32 * WPC, smem, s>>>(a);
+  return cudaGetLastError();
+}
+
+template <int MODE, int NVW>
+cudaError_t run_warp_any(const TopkRowArgs& a, int num_sms, cudaStream_t s) {
+  if (a.L == 128 * NVW) return run_warp<MODE, NVW, true>(a, num_sms, s);
+  return run_warp<MODE, NVW, false>(a, num_sms, s);
+}
+
+template <int MODE, int NT, int SCAP, bool FULL>
+cudaError_t run_cta(const TopkRowArgs& a, int C, cudaStream_t s) {
+  auto kernel = topk_cta_kernel<MODE, NT, SCAP, FULL>;
+  const int smem = cta_smem_bytes(NT, SCAP, C);
+  cudaError_t err = ensure_dynamic_smem(kernel, cta_smem_bytes(NT, SCAP, kMaxCluster));
+  if (err != cudaSuccess) return err;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(a.rows * C), 1, 1);
+  cfg.blockDim = dim3(NT, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = C;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, a);
+}
+
+// FULL when every CTA's slice is a whole number of NT x 4-entry slots.
+template <int MODE, int NT, int SCAP>
+cudaError_t run_cta_any(const TopkRowArgs& a, int C, cudaStream_t s) {
+  const bool full = (a.slice % (4 * NT) == 0) && (a.slice * C == a.L);
+  if (full) return run_cta<MODE, NT, SCAP, true>(a, C, s);
+  return run_cta<MODE, NT, SCAP, false>(a, C, s);
+}
+
+template <int MODE>
+cudaError_t run_mode(const TopkRowArgs& a0, int num_sms, cudaStream_t s) {
+  TopkRowArgs a = a0;
+  const int64_t L = a.L;
+  if (L <= 256) return run_warp_any<MODE, 2>(a, num_sms, s);
+  if (L <= 512) return run_warp_any<MODE, 4>(a, num_sms, s);
+  if (L <= 768) return run_warp_any<MODE, 6>(a, num_sms, s);
+  if (L <= 1024) return run_warp_any<MODE, 8>(a, num_sms, s);
+  // One CTA of 128 threads for rows up to 4096 entries, else clusters of
+  // 256-thread CTAs holding up to 8192 entries each, split further (slices of
+  // at least 2048 entries) while the grid has fewer than 2 CTAs per SM.
+  if (L <= 2048) {
+    a.slice = (L + 3) / 4 * 4;
+    return run_cta_any<MODE, 128, 2048>(a, 1, s);
+  }
+  if (L <= 4096) {
+    a.slice = (L + 3) / 4 * 4;
+    return run_cta_any<MODE, 128, 4096>(a, 1, s);
+  }
+  int64_t C = (L + 8191) / 8192;
+  while (a.rows * C < 2 * num_sms && C < kMaxCluster && L / (2 * C) >= 2048) C *= 2;
+  if (C > kMaxCluster) return cudaErrorInvalidValue;
+  a.slice = ((L + C - 1) / C + 3) / 4 * 4;
+  return run_cta_any<MODE, 256, 8192>(a, static_cast<int>(C), s);
+}
+
+}  // namespace rows
+}  // namespace mpc
