@@ -12,9 +12,11 @@ one boundary crossing of every operator the workload sweeps, on that step's tens
             dequantisation.
 value = sum over the 9 compress+decompress pairs of the input bytes (4 x 128 x 32768) /
 device time of the step.  Each step is one CUDA graph of the 18 library launches (one
-graph per slot of a pool of 4 pre-drawn steps, so inputs differ from step to step); L2
-is flushed (256 MiB write) before every timed step and the flush is outside the timed
-interval.  `e2e` runs the same steps through the Python API without graphs, with the
+graph per slot of a pool of 4 pre-drawn steps, so inputs differ from step to step), with
+no event nodes inside; L2 is flushed (256 MiB write) before every timed step and the
+flush is outside the timed interval.  Per-launch times come from a second timed pass
+whose graphs record an event after every launch, and the dominant launch's duration
+(for `roofline`) from a third pass with one event pair around that launch only.  `e2e` runs the same steps through the Python API without graphs, with the
 step's inputs copied from pinned host memory and two outputs copied back inside the
 timed region.  `operators` times every operator of the path on its own workload.
 
@@ -272,24 +274,35 @@ class Step:
                 self.ops.append(("quant_decompress " + tag, algorithmic_bytes(R, L, bits=b, op="dequant")))
         self.input_bytes = 9 * 4 * R * L  # 9 compress+decompress pairs
 
-    def launch(self, slot: int, step: int, events=None, x=None, g=None):
-        """Enqueue the step's 18 launches; optionally record an event after each."""
+    def launch(self, slot: int, step: int, events=None, x=None, g=None, around=None):
+        """Enqueue the step's 18 launches.  events: one event recorded after each launch;
+        around: (i, ev0, ev1) records ev0 just before launch i and ev1 just after it."""
         m = self.mpc
         x = self.xs[slot] if x is None else x
         g = self.gs[slot] if g is None else g
         e = iter(events) if events is not None else None
+        n = [0]
+
+        def op(fn):
+            if around is not None and around[0] == n[0]:
+                around[1].record()
+            fn()
+            if around is not None and around[0] == n[0]:
+                around[2].record()
+            if e is not None:
+                next(e).record()
+            n[0] += 1
+
         for p in TOPK_PCTS:
-            m.mpc_ef_topk_compress(x, self.errs[p], self.ks[p], self.vals[p], self.idx[p])
-            if e: next(e).record()
-            m.mpc_topk_decompress(self.vals[p], self.idx[p], L, y=self.y)
-            if e: next(e).record()
+            op(lambda: m.mpc_ef_topk_compress(x, self.errs[p], self.ks[p], self.vals[p], self.idx[p]))
+            op(lambda: m.mpc_topk_decompress(self.vals[p], self.idx[p], L, y=self.y))
         for b in BITS:
             for sr in (False, True):
-                m.mpc_quant_compress(g, b, stochastic=sr, seed=(self.seed << 32) | step,
-                                     codes=self.codes[b], scale=self.scale[b], minv=self.minv[b])
-                if e: next(e).record()
-                m.mpc_quant_decompress(self.codes[b], self.scale[b], self.minv[b], L, b, y=self.gy)
-                if e: next(e).record()
+                op(lambda: m.mpc_quant_compress(g, b, stochastic=sr, seed=(self.seed << 32) | step,
+                                                codes=self.codes[b], scale=self.scale[b],
+                                                minv=self.minv[b]))
+                op(lambda: m.mpc_quant_decompress(self.codes[b], self.scale[b], self.minv[b], L, b,
+                                                  y=self.gy))
 
 
 def make_event(external: bool):
@@ -323,26 +336,29 @@ def run_ours(args, rank, local, world):
     stream.synchronize()
     assert mpc.mpc_get_status(stream) == 0, mpc.mpc_last_error()
 
-    # one graph per pool slot, with an event after every launch
-    probe = make_event(external=True)
-    per_op_events = probe is not None
-    graphs, evsets = [], []
-    for slot in range(POOL):
-        evs = [make_event(True) for _ in range(n_ops)] if per_op_events else None
+    # One graph per pool slot.  Event nodes inside a graph cost ~5 us each, so the
+    # headline steps replay event-free graphs; per-launch times come from a second
+    # timed pass with an event after every launch (shares of the step), and the
+    # dominant launch's duration from a third pass with one event pair around it.
+    if make_event(external=True) is None:
+        raise RuntimeError("torch.cuda.Event(external=True) is required")
+    keep = []  # events referenced by graph nodes must outlive the graphs
+
+    def capture(slot, **kw):
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=stream):
-            st.launch(slot, slot, events=evs)
-        graphs.append(g)
-        evsets.append(evs)
-    torch.cuda.synchronize()
-    for p in TOPK_PCTS:
-        st.errs[p].zero_()
+            st.launch(slot, slot, **kw)
+        return g
 
-    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    op_ms = [0.0] * n_ops
-    sampler = ClockSampler(local)
-    with sampler:
+    plain = [capture(slot) for slot in range(POOL)]
+    evsets = [[make_event(True) for _ in range(n_ops)] for _ in range(POOL)]
+    keep.append(evsets)
+    evented = [capture(slot, events=evsets[slot]) for slot in range(POOL)]
+    torch.cuda.synchronize()
+
+    def timed_pass(graphs, after_step=None):
+        starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+        ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
         with torch.cuda.stream(stream):
             for w in range(args.warmup):
                 flush.fill_(w & 0xff)
@@ -352,29 +368,48 @@ def run_ours(args, rank, local, world):
         torch.cuda.synchronize()
         t0 = time.perf_counter()
         with torch.cuda.stream(stream):
-            for s in range(args.steps):
-                flush.fill_(s & 0xff)
-                starts[s].record(stream)
-                graphs[s % POOL].replay()
-                ends[s].record(stream)
-                if per_op_events:
-                    # events inside the graph belong to its slot; read them before reuse
-                    if (s + 1) % POOL == 0 or s == args.steps - 1:
-                        stream.synchronize()
-                        base = s - (s % POOL)
-                        for j in range(base, s + 1):
-                            evs = evsets[j % POOL]
-                            prev = starts[j]
-                            for i, ev in enumerate(evs):
-                                op_ms[i] += prev.elapsed_time(ev)
-                                prev = ev
+            for i in range(args.steps):
+                flush.fill_(i & 0xff)
+                starts[i].record(stream)
+                graphs[i % POOL].replay()
+                ends[i].record(stream)
+                if after_step is not None and ((i + 1) % POOL == 0 or i == args.steps - 1):
+                    # events inside a graph belong to its slot: read them before reuse
+                    stream.synchronize()
+                    for j in range(i - (i % POOL), i + 1):
+                        after_step(j, starts[j], ends[j])
         stream.synchronize()
         torch.cuda.synchronize()
         barrier(world)
         wall = time.perf_counter() - t0
+        return sum(starts[i].elapsed_time(ends[i]) for i in range(args.steps)) / 1e3, wall
+
+    for p in TOPK_PCTS:
+        st.errs[p].zero_()
+    sampler = ClockSampler(local)
+    with sampler:
+        dev_s, wall = timed_pass(plain)
     clocks = sampler.summary()
-    step_ms = [starts[s].elapsed_time(ends[s]) for s in range(args.steps)]
-    dev_s = sum(step_ms) / 1e3
+
+    op_ms = [0.0] * n_ops
+
+    def read_ops(j, start, end):
+        prev = start
+        for i, ev in enumerate(evsets[j % POOL]):
+            op_ms[i] += prev.elapsed_time(ev)
+            prev = ev
+
+    timed_pass(evented, read_ops)
+    dom = max(range(n_ops), key=lambda j: op_ms[j])
+    pairs = [(make_event(True), make_event(True)) for _ in range(POOL)]
+    keep.append(pairs)
+    around = [capture(slot, around=(dom, pairs[slot][0], pairs[slot][1])) for slot in range(POOL)]
+    dom_ms = [0.0]
+
+    def read_dom(j, start, end):
+        dom_ms[0] += pairs[j % POOL][0].elapsed_time(pairs[j % POOL][1])
+
+    timed_pass(around, read_dom)
     status = mpc.mpc_get_status(stream)
     if status != 0:
         raise RuntimeError("device status %d: %s" % (status, mpc.mpc_last_error()))
@@ -384,27 +419,23 @@ def run_ours(args, rank, local, world):
 
     # roofline of the dominant kernel (largest share of the step)
     peak, peak_kind = hbm_peak()
-    roofline = None
-    if per_op_events and sum(op_ms) > 0:
-        i = max(range(n_ops), key=lambda j: op_ms[j])
-        name, nbytes = st.ops[i]
-        avg_ms = op_ms[i] / args.steps
-        achieved = nbytes / (avg_ms / 1e3) / 1e9
-        kern = "topk_cta_kernel" if "topk_compress" in name else (
-            "topk_decompress_kernel" if "decompress K" in name else (
-                "quant_cta_kernel" if "quant_compress" in name else "dequant_kernel"))
-        traffic = recorded_traffic(kern + ":" + name.replace(" ", "_"))
-        roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
-                    "frac": round(achieved / peak, 4), "traffic": traffic,
-                    "kernel": kern, "op": name, "algorithmic_bytes": nbytes,
-                    "avg_launch_us": round(avg_ms * 1e3, 2),
-                    "share_of_step": round(op_ms[i] / max(sum(op_ms), 1e-9), 4),
-                    "peak_source": peak_kind}
-        per_op = {st.ops[j][0]: {"avg_us": round(op_ms[j] / args.steps * 1e3, 2),
-                                 "GBps": round(st.ops[j][1] / (op_ms[j] / args.steps / 1e3) / 1e9, 1)}
-                  for j in range(n_ops)}
-    else:
-        per_op = None
+    name, nbytes = st.ops[dom]
+    avg_ms = dom_ms[0] / args.steps
+    achieved = nbytes / (avg_ms / 1e3) / 1e9
+    kern = "topk_cta_kernel" if "topk_compress" in name else (
+        "topk_decompress_rows_kernel" if "decompress K" in name else (
+            "quant_cta_kernel" if "quant_compress" in name else "dequant_kernel"))
+    traffic = recorded_traffic(kern + ":" + name.replace(" ", "_"))
+    roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                "frac": round(achieved / peak, 4), "traffic": traffic,
+                "kernel": kern, "op": name, "algorithmic_bytes": nbytes,
+                "avg_launch_us": round(avg_ms * 1e3, 2),
+                "share_of_step": round(op_ms[dom] / max(sum(op_ms), 1e-9), 4),
+                "peak_source": peak_kind,
+                "timing": "one event pair around this launch inside the step graph"}
+    per_op = {st.ops[j][0]: {"avg_us": round(op_ms[j] / args.steps * 1e3, 2),
+                             "GBps": round(st.ops[j][1] / (op_ms[j] / args.steps / 1e3) / 1e9, 1)}
+              for j in range(n_ops)}
 
     # end to end through the Python API: host inputs in, two outputs back, no graphs
     e2e = run_e2e(args, st, stream, world, device)
@@ -426,12 +457,15 @@ def run_ours(args, rank, local, world):
             "config": {"workload": WORKLOAD, "rows": R, "row_len": L,
                        "topk_percents": list(TOPK_PCTS), "bits": list(BITS),
                        "rounding": ["nearest", "stochastic"], "launches_per_step": n_ops,
-                       "step": "one CUDA graph per step", "l2": "256 MiB flush before each "
-                       "timed step, outside the timed interval", "parallelism":
+                       "step": "one CUDA graph per step (no event nodes inside)", "l2": "256 MiB flush "
+                       "before each timed step, outside the timed interval", "parallelism":
                        "replicas" if world > 1 else "single GPU"},
             "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
             "gpu_launches": n_ops * args.steps, "clocks": clocks,
-            "wall_s": round(wall, 3), "per_op": per_op, "operators": operators,
+            "wall_s": round(wall, 3), "per_op": per_op,
+            "per_op_timing": "an event after every launch inside the step graph (second pass; "
+                             "each interval includes the ~5 us of an event node)",
+            "operators": operators,
         }
         print(json.dumps(line), flush=True)
 

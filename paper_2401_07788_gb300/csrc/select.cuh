@@ -138,10 +138,11 @@ __device__ __forceinline__ Threshold warp_list_select(const int* keys, uint32_t 
 }
 
 // Rank test of one candidate key ki against the m keys: it is T when fewer than
-// kr keys are larger and at least kr are at least as large; then `need` is
-// kr minus the number larger.
+// kr keys are larger and at least kr are at least as large.  Then *t is the
+// threshold: {ki, kr - #larger}, or {ki - 1, 0} when every key equal to ki is
+// kept anyway (no tie has to be ranked by index).
 __device__ __forceinline__ bool rank_is_threshold(const int* keys, uint32_t m, uint32_t kr, int ki,
-                                                  uint32_t* need) {
+                                                  Threshold* t) {
   uint32_t gt = 0, ge = 0;
   uint32_t j = 0;
   for (; j + 4 <= m; j += 4) {
@@ -154,31 +155,29 @@ __device__ __forceinline__ bool rank_is_threshold(const int* keys, uint32_t m, u
     gt += a0 > ki;
     ge += a0 >= ki;
   }
-  *need = kr - gt;
-  return gt < kr && kr <= ge;
+  if (!(gt < kr && kr <= ge)) return false;
+  const uint32_t need = kr - gt;
+  *t = (need == ge - gt) ? Threshold{ki - 1, 0u} : Threshold{ki, need};
+  return true;
 }
 
 // One warp, m <= 64 keys in shared memory: each lane ranks its candidates
 // against all m keys (a loop of length m); the lane holding T reports it.
 __device__ __forceinline__ Threshold warp_rank_select(const int* keys, uint32_t m, uint32_t kr,
                                                       int lane) {
-  int T = -1;
-  uint32_t need = 0;
+  Threshold t = {-1, 0u};
   bool found = false;
   for (uint32_t i = lane; i < m; i += 32) {
-    uint32_t nd;
-    const int ki = keys[i];
-    if (rank_is_threshold(keys, m, kr, ki, &nd)) {
-      T = ki;
-      need = nd;
+    Threshold ti;
+    if (rank_is_threshold(keys, m, kr, keys[i], &ti)) {
+      t = ti;
       found = true;
     }
   }
   const unsigned who = __ballot_sync(kFull, found);
   const int src = who ? __ffs(who) - 1 : 0;
-  Threshold t;
-  t.T = __shfl_sync(kFull, T, src);
-  t.need = __shfl_sync(kFull, need, src);
+  t.T = __shfl_sync(kFull, t.T, src);
+  t.need = __shfl_sync(kFull, t.need, src);
   return t;
 }
 

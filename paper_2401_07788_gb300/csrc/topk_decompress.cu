@@ -89,34 +89,60 @@ __global__ void __launch_bounds__(kDecThreads)
   }
 }
 
-// Whole rows [r0, r0 + nrows) per CTA (rpc * row_len <= kRowsPerCta entries).
+// Rows of up to 65536 entries: a CTA owns either whole rows [r0, r0 + nrows)
+// (rpc rows, rpc * row_len <= kRowsPerCta) or the column range
+// [part * width, part * width + width) of one row (ppr parts per row).  It
+// zero-fills its region, then stores the kept values that fall in it; a part
+// reads its row's whole payload (from L2 after the first part) and keeps its own.
 constexpr int64_t kRowsPerCta = 16384;
+constexpr int64_t kPartWidth = 8192;
 
 __global__ void __launch_bounds__(kDecThreads)
     topk_decompress_rows_kernel(const float* __restrict__ vals, const int32_t* __restrict__ idx,
                                 int64_t rows, int64_t L, int64_t k, float* __restrict__ y,
-                                int64_t rpc, int aligned) {
+                                int64_t rpc, int64_t ppr, int aligned) {
   const int tid = threadIdx.x;
-  const int64_t r0 = static_cast<int64_t>(blockIdx.x) * rpc;
-  const int64_t nrows = min64(rpc, rows - r0);
-  const int64_t cells = nrows * L;
-  float* dst = y + r0 * L;
-  if (aligned) {
-    const int64_t n4 = cells / 4;
-    float4* d4 = reinterpret_cast<float4*>(dst);
-    for (int64_t i = tid; i < n4; i += kDecThreads) d4[i] = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int64_t i = n4 * 4 + tid; i < cells; i += kDecThreads) dst[i] = 0.0f;
+  int64_t r0, nrows, c0, ncols;
+  if (ppr == 1) {
+    r0 = static_cast<int64_t>(blockIdx.x) * rpc;
+    nrows = min64(rpc, rows - r0);
+    c0 = 0;
+    ncols = L;
   } else {
-    for (int64_t i = tid; i < cells; i += kDecThreads) dst[i] = 0.0f;
+    r0 = blockIdx.x / ppr;
+    nrows = 1;
+    c0 = (blockIdx.x % ppr) * kPartWidth;
+    ncols = min64(kPartWidth, L - c0);
+  }
+  float* dst = y + r0 * L + c0;
+  if (ppr == 1) {
+    const int64_t cells = nrows * L;
+    if (aligned) {
+      const int64_t n4 = cells / 4;
+      float4* d4 = reinterpret_cast<float4*>(dst);
+      for (int64_t i = tid; i < n4; i += kDecThreads) d4[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+      for (int64_t i = n4 * 4 + tid; i < cells; i += kDecThreads) dst[i] = 0.0f;
+    } else {
+      for (int64_t i = tid; i < cells; i += kDecThreads) dst[i] = 0.0f;
+    }
+  } else {
+    if (aligned) {
+      const int64_t n4 = ncols / 4;
+      float4* d4 = reinterpret_cast<float4*>(dst);
+      for (int64_t i = tid; i < n4; i += kDecThreads) d4[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+      for (int64_t i = n4 * 4 + tid; i < ncols; i += kDecThreads) dst[i] = 0.0f;
+    } else {
+      for (int64_t i = tid; i < ncols; i += kDecThreads) dst[i] = 0.0f;
+    }
   }
   __syncthreads();  // the zeros of this block precede its kept values
   const int64_t e_begin = r0 * k;
-  const uint32_t nk = static_cast<uint32_t>(nrows * k);  // <= rpc * L <= 65536
+  const uint32_t nk = static_cast<uint32_t>(nrows * k);  // <= 65536
   const uint32_t k32 = static_cast<uint32_t>(k);
   for (uint32_t e = tid; e < nk; e += kDecThreads) {
-    const uint32_t lr = e / k32;
-    const int64_t col = idx[e_begin + e];
-    if (col >= 0 && col < L) dst[static_cast<int64_t>(lr) * L + col] = vals[e_begin + e];
+    const uint32_t lr = (ppr == 1) ? e / k32 : 0u;
+    const int64_t col = static_cast<int64_t>(idx[e_begin + e]) - c0;
+    if (col >= 0 && col < ncols) dst[static_cast<int64_t>(lr) * L + col] = vals[e_begin + e];
   }
 }
 
@@ -149,11 +175,17 @@ cudaError_t launch_topk_decompress(const float* vals, const int32_t* idx, int64_
   (void)num_sms;
   if (rows <= 0) return cudaSuccess;
   if (L <= 65536) {
-    const int64_t rpc = max64(1, min64(rows, kRowsPerCta / L));
-    const int64_t blocks = (rows + rpc - 1) / rpc;
+    int64_t rpc = 1, ppr = 1, blocks;
+    if (L <= kRowsPerCta) {
+      rpc = max64(1, min64(rows, kRowsPerCta / L));
+      blocks = (rows + rpc - 1) / rpc;
+    } else {
+      ppr = (L + kPartWidth - 1) / kPartWidth;
+      blocks = rows * ppr;
+    }
     if (blocks > 0x7fffffffLL) return cudaErrorInvalidValue;
     topk_decompress_rows_kernel<<<static_cast<unsigned>(blocks), kDecThreads, 0, s>>>(
-        vals, idx, rows, L, k, y, rpc, aligned);
+        vals, idx, rows, L, k, y, rpc, ppr, aligned);
     return cudaGetLastError();
   }
   int64_t rpc = 1, tpr = 1, blocks;

@@ -141,7 +141,7 @@ struct CtaShared {
   int pub_lo, pub_hi;
   BinPick pick;
   Threshold thr;
-  uint64_t bar;
+  uint64_t bars[8];  // one per slice chunk (one float4 slot of every thread)
 };
 
 // The bin holding the kr-th element of an NBINS-bin histogram (bins ranked
@@ -276,18 +276,24 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
   }
   const float* xrow = a.x + row * L;
 
-  // ---- issue the loads: x by bulk copy, a sample of the row, err / state ----
-  bool failed = false;
+  // ---- issue the loads: x by bulk copies, a sample of the row, err / state --
+  // The slice of x arrives in chunks of one float4 slot per thread (4*NT
+  // entries), each completing on its own mbarrier, so the first pass starts on
+  // chunk 0 while the others are still in flight.
+  static_assert(QPT <= 8, "one mbarrier per chunk");
+  const int jmax = (n + 4 * NT - 1) / (4 * NT);  // float4 slots of each thread in use
   if (a.aligned) {
     if (tid == 0) {
-      mbar_init(&sh.bar, 1);
+      for (int j = 0; j < QPT; ++j) mbar_init(&sh.bars[j], 1);
       fence_mbar_init();
     }
     __syncthreads();
-    if (tid == 0 && n > 0) {
-      const uint32_t bytes = static_cast<uint32_t>(n) * 4u;
-      mbar_arrive_expect_tx(&sh.bar, bytes);
-      bulk_g2s(s4, xrow + c0, bytes, &sh.bar);
+    if (tid == 0) {
+      for (int j = 0; j < jmax; ++j) {
+        const uint32_t bytes = static_cast<uint32_t>(min(4 * NT, n - 4 * NT * j)) * 4u;
+        mbar_arrive_expect_tx(&sh.bars[j], bytes);
+        bulk_g2s(s4 + j * NT, xrow + c0 + 4 * NT * j, bytes, &sh.bars[j]);
+      }
     }
   }
   // The bin scale comes from a sample of the row, entries [p, p+4) spread over
@@ -322,29 +328,25 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
     smax = __reduce_max_sync(kFull, smax);
     if (lane == 0) sh.sample_max[warp] = smax;
   }
-
-  if (a.aligned) {
-    if (n > 0 && !mbar_wait_bounded(&sh.bar, 0, a.spin_limit, a.status)) {
-      mbar_wait_bounded(&sh.bar, 0, kDrainPolls, nullptr);
-      failed = true;
-    }
-    failed = __syncthreads_or(failed);
-  } else {
+  if (!a.aligned) {
     float* s = reinterpret_cast<float*>(s4);
     for (int e = tid; e < n; e += NT)
       s[e] = ranked_value<MODE>(xrow[c0 + e], (MODE != kPlain) ? arow[c0 + e] : 0.0f);
-    __syncthreads();
   }
-  const int nv = failed ? 0 : n;  // a failed slice takes part as an empty one
-  const int jmax = (nv + 4 * NT - 1) / (4 * NT);  // float4 slots of each thread in use
+  __syncthreads();
   const float scale = bucket_scale(max(sh.sample_max[0], sh.sample_max[1]), kNB);
   const bool binned = k < L && scale > 0.0f;
 
   // ---- ranked values into shared memory and the first histogram -------------
+  bool failed = false;
   uint32_t zc = 0;
 #pragma unroll
   for (int j = 0; j < QPT; ++j) {
     if (j < jmax) {
+      if (a.aligned && !mbar_wait_bounded(&sh.bars[j], 0, a.spin_limit, a.status)) {
+        mbar_wait_bounded(&sh.bars[j], 0, kDrainPolls, nullptr);
+        failed = true;
+      }
       const int q = j * NT + tid;
       float4 v = s4[q];
       if (MODE != kPlain && a.aligned) {
@@ -353,7 +355,7 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
       }
       if (binned) {
         int kk[4];
-        keys4<FULL>(v, 4 * q, nv, kk);
+        keys4<FULL>(v, 4 * q, n, kk);
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
           if (kk[i] == 0) ++zc;
@@ -366,7 +368,11 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
     zc = __reduce_add_sync(kFull, zc);
     if (lane == 0 && zc) atomicAdd(&sh.hist[0], zc);
   }
-  __syncthreads();
+  failed = __syncthreads_or(failed);
+  // A slice whose copy timed out takes part in the rest as an empty one (the
+  // status word reports the timeout; the row's outputs are then unspecified).
+  const int nv = failed ? 0 : n;
+  const int jv = failed ? 0 : jmax;
 
   // ---- select T and need -----------------------------------------------------
   int T = -1;
@@ -390,7 +396,7 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
 #pragma unroll 2
       for (int j = 0; j < QPT; ++j) {
         uint32_t ab = 0;
-        if (j < jmax) {
+        if (j < jv) {
           const int q = j * NT + tid;
           int kk[4];
           keys4<FULL>(s4[q], 4 * q, nv, kk);
@@ -451,9 +457,8 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
       // every thread ranks its candidates against the whole list; the
       // thread holding T reports it (all such threads report the same values)
       for (uint32_t i = tid; i < mt; i += NT) {
-        uint32_t nd;
-        const int ki = list[i];
-        if (rank_is_threshold(list, mt, kr, ki, &nd)) sh.thr = Threshold{ki, nd};
+        Threshold ti;
+        if (rank_is_threshold(list, mt, kr, list[i], &ti)) sh.thr = ti;
       }
       __syncthreads();
       T = sh.thr.T;
@@ -498,7 +503,7 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
       // ---- too many candidates for the list: integer rounds over the slice --
       int lo = 0x7fffffff, hi = -1;
 #pragma unroll 2
-      for (int j = 0; j < jmax; ++j) {
+      for (int j = 0; j < jv; ++j) {
         const int q = j * NT + tid;
         int kk[4];
         keys4<FULL>(s4[q], 4 * q, nv, kk);
@@ -533,7 +538,7 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
         for (int i = tid; i < kRoundBins; i += NT) sh.rhist[p][i] = 0;
         __syncthreads();
 #pragma unroll 2
-        for (int j = 0; j < jmax; ++j) {
+        for (int j = 0; j < jv; ++j) {
           const int q = j * NT + tid;
           int kk[4];
           keys4<FULL>(s4[q], 4 * q, nv, kk);
@@ -568,7 +573,7 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
 #pragma unroll 2
     for (int j = 0; j < QPT; ++j) {
       uint32_t g = 0, e = 0;
-      if (j < jmax) {
+      if (j < jv) {
         const int q = j * NT + tid;
         int kk[4];
         keys4<FULL>(s4[q], 4 * q, nv, kk);
@@ -613,7 +618,7 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
   int32_t* irow = a.idx + row * k;
   const unsigned lt = lanemask_lt();
 #pragma unroll 2
-  for (int j = 0; j < jmax; ++j) {
+  for (int j = 0; j < jv; ++j) {
     const int ch = j * NW + warp;
     const int q = j * NT + tid;
     const float4 v4 = s4[q];
