@@ -54,7 +54,7 @@ SAMPLE_ROWS = 16
 def parse_args():
     p = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     p.add_argument("--gpus", type=int, default=1)
-    p.add_argument("--steps", type=int, default=200)
+    p.add_argument("--steps", type=int, default=1000)
     p.add_argument("--warmup", type=int, default=10)
     p.add_argument("--impl", choices=("ours", "reference"), default="ours")
     p.add_argument("--no-operators", action="store_true", help="skip the per-operator table")
@@ -148,34 +148,90 @@ def recorded_traffic(kernel: str):
 
 
 class ClockSampler:
-    """nvidia-smi samples of SM clock and throttle reasons while the benchmark runs."""
+    """SM clock and clock-event reasons sampled every ~2 ms while the benchmark runs,
+    through NVML (read-only queries), else through nvidia-smi."""
 
-    FIELDS = ("clocks.sm,clocks.max.sm,clocks_event_reasons.hw_slowdown,"
-              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
-              "clocks_event_reasons.sw_power_cap")
+    # NVML clock-event reason bits
+    REASONS = ((0x4, "sw_power_cap"), (0x8, "hw_slowdown"), (0x20, "sw_thermal_slowdown"),
+               (0x40, "hw_thermal_slowdown"), (0x80, "hw_power_brake_slowdown"))
 
-    def __init__(self, device_index: int):
-        self.proc = None
+    def __init__(self, device_index: int, interval_s: float = 0.002):
+        self.interval = interval_s
+        self.samples = []  # (sm_mhz, reason bits)
+        self.max_mhz = None
+        self.source = None
+        self.bus = None
         try:
-            bus = torch.cuda.get_device_properties(device_index).pci_bus_id
+            p = torch.cuda.get_device_properties(device_index)
+            self.bus = "%08X:%02X:%02X.0" % (p.pci_domain_id, p.pci_bus_id, p.pci_device_id)
         except Exception:
-            bus = None
-        self.target = bus
-        self.out = os.path.join("/tmp", "mpc_clocks_%d.csv" % os.getpid())
+            pass
+        self.nvml = self._open_nvml()
+
+    def _open_nvml(self):
+        import ctypes
+
+        try:
+            lib = ctypes.CDLL("libnvidia-ml.so.1")
+            if lib.nvmlInit_v2() != 0 or self.bus is None:
+                return None
+            h = ctypes.c_void_p()
+            if lib.nvmlDeviceGetHandleByPciBusId_v2(self.bus.encode(), ctypes.byref(h)) != 0:
+                return None
+            reasons = getattr(lib, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+                lib.nvmlDeviceGetCurrentClocksThrottleReasons
+            mx = ctypes.c_uint()
+            if lib.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(mx)) == 0:
+                self.max_mhz = float(mx.value)
+            return (lib, h, reasons)
+        except (OSError, AttributeError):
+            return None
+
+    def _sample_nvml(self):
+        import ctypes
+
+        lib, h, reasons = self.nvml
+        mhz, bits = ctypes.c_uint(), ctypes.c_ulonglong()
+        if lib.nvmlDeviceGetClockInfo(h, 1, ctypes.byref(mhz)) == 0 and \
+                reasons(h, ctypes.byref(bits)) == 0:
+            self.samples.append((float(mhz.value), int(bits.value)))
 
     def __enter__(self):
-        cmd = ["nvidia-smi", "--query-gpu=" + self.FIELDS, "--format=csv,noheader,nounits",
-               "-lms", "100"]
-        if self.target:
-            cmd += ["-i", self.target]
-        try:
-            self.fh = open(self.out, "w")
-            self.proc = subprocess.Popen(cmd, stdout=self.fh, stderr=subprocess.DEVNULL)
-        except OSError:
-            self.proc = None
+        import threading
+
+        self.stop = threading.Event()
+        self.proc = None
+        if self.nvml is not None:
+            self.source = "nvml"
+            self._sample_nvml()
+
+            def loop():
+                while not self.stop.wait(self.interval):
+                    self._sample_nvml()
+
+            self.thread = threading.Thread(target=loop, daemon=True)
+            self.thread.start()
+        else:
+            self.thread = None
+            self.out = os.path.join("/tmp", "mpc_clocks_%d.csv" % os.getpid())
+            cmd = ["nvidia-smi", "--query-gpu=clocks.sm,clocks.max.sm,"
+                   "clocks_event_reasons.active", "--format=csv,noheader,nounits", "-lms", "20"]
+            if self.bus:
+                cmd += ["-i", self.bus]
+            try:
+                self.fh = open(self.out, "w")
+                self.proc = subprocess.Popen(cmd, stdout=self.fh, stderr=subprocess.DEVNULL)
+                self.source = "nvidia-smi"
+                time.sleep(0.5)  # let it start before the timed region
+            except OSError:
+                self.proc = None
         return self
 
     def __exit__(self, *exc):
+        self.stop.set()
+        if self.thread is not None:
+            self.thread.join()
+            self._sample_nvml()
         if self.proc is not None:
             self.proc.terminate()
             try:
@@ -183,35 +239,26 @@ class ClockSampler:
             except subprocess.TimeoutExpired:
                 self.proc.kill()
             self.fh.close()
+            try:
+                for row in open(self.out).read().splitlines():
+                    f = [c.strip() for c in row.split(",")]
+                    try:
+                        self.samples.append((float(f[0]), int(f[2], 16)))
+                        self.max_mhz = float(f[1])
+                    except (ValueError, IndexError):
+                        continue
+                os.remove(self.out)
+            except OSError:
+                pass
 
     def summary(self):
-        if self.proc is None:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
-        sm, mx, reasons = [], [], set()
-        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
-        try:
-            rows = open(self.out).read().splitlines()
-        except OSError:
-            rows = []
-        for row in rows:
-            f = [c.strip() for c in row.split(",")]
-            if len(f) < 6:
-                continue
-            try:
-                sm.append(float(f[0]))
-                mx.append(float(f[1]))
-            except ValueError:
-                continue
-            for n, v in zip(names, f[2:6]):
-                if v.lower().startswith("active"):
-                    reasons.add(n)
-        try:
-            os.remove(self.out)
-        except OSError:
-            pass
-        return {"sm_mhz": statistics.median(sm) if sm else None,
-                "sm_max_mhz": max(mx) if mx else None, "reasons": sorted(reasons),
-                "samples": len(sm)}
+        if not self.samples:
+            return {"sm_mhz": None, "sm_max_mhz": self.max_mhz, "reasons": [],
+                    "samples": 0, "source": self.source or "unavailable"}
+        reasons = sorted({name for _, b in self.samples for bit, name in self.REASONS if b & bit})
+        return {"sm_mhz": statistics.median(s for s, _ in self.samples),
+                "sm_max_mhz": self.max_mhz, "reasons": reasons,
+                "samples": len(self.samples), "source": self.source}
 
 
 # ---------------------------------------------------------------------------------------
@@ -356,7 +403,7 @@ def run_ours(args, rank, local, world):
     evented = [capture(slot, events=evsets[slot]) for slot in range(POOL)]
     torch.cuda.synchronize()
 
-    def timed_pass(graphs, after_step=None):
+    def timed_pass(graphs, after_step=None, sampler=None):
         starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
         ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
         with torch.cuda.stream(stream):
@@ -366,6 +413,8 @@ def run_ours(args, rank, local, world):
         stream.synchronize()
         barrier(world)
         torch.cuda.synchronize()
+        if sampler is not None:
+            sampler.__enter__()
         t0 = time.perf_counter()
         with torch.cuda.stream(stream):
             for i in range(args.steps):
@@ -380,15 +429,16 @@ def run_ours(args, rank, local, world):
                         after_step(j, starts[j], ends[j])
         stream.synchronize()
         torch.cuda.synchronize()
-        barrier(world)
         wall = time.perf_counter() - t0
+        if sampler is not None:
+            sampler.__exit__(None, None, None)
+        barrier(world)
         return sum(starts[i].elapsed_time(ends[i]) for i in range(args.steps)) / 1e3, wall
 
     for p in TOPK_PCTS:
         st.errs[p].zero_()
     sampler = ClockSampler(local)
-    with sampler:
-        dev_s, wall = timed_pass(plain)
+    dev_s, wall = timed_pass(plain, sampler=sampler)
     clocks = sampler.summary()
 
     op_ms = [0.0] * n_ops

@@ -224,9 +224,10 @@ mpc_status mpc_get_status(mpc_stream_t stream);
 const char* mpc_last_error(void);
 
 /* Test knobs (values persist for the process; not for production use):
- *   MPC_KNOB_SPIN_LIMIT   polls of a device-side wait before it gives up
- *                         (default 1<<20, about 0.1 s; 0 makes every first wait give up,
- *                         which tests the timeout report without a fault);
+ *   MPC_KNOB_SPIN_LIMIT   tries of a device-side wait before it gives up; the
+ *                         wait also stops after about 64 ns x this value
+ *                         (default 1<<20, about 0.07 s; 0 makes every first wait give
+ *                         up, which tests the timeout report without a fault);
  *   MPC_KNOB_TOPK_PATH    0 = automatic, 1 = force the on-chip row path when
  *                         it fits, 2 = force the multi-pass (workspace) path.
  * Returns MPC_ERR_INVALID_ARG for an unknown knob. */

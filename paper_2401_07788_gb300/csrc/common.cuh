@@ -69,11 +69,21 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t by
                : "memory");
 }
 
-// Non-blocking test of phase `parity` of `bar` (returns at once).
-__device__ __forceinline__ bool mbar_test_wait(uint64_t* bar, uint32_t parity) {
+// Nanoseconds of the global timer.
+__device__ __forceinline__ uint64_t global_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+// One wait of bounded length on phase `parity` of `bar`: the thread is
+// suspended until the phase completes or at most about 1 ms has passed (the
+// hint; the hardware may end the wait sooner), so a waiting warp takes no
+// issue slots.  Returns whether the phase completed.
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
-      "{\n .reg .pred p;\n mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, 1000000;\n"
       " selp.u32 %0, 1, 0, p;\n}\n"
       : "=r"(ok)
       : "r"(smem_addr(bar)), "r"(parity)
@@ -81,15 +91,18 @@ __device__ __forceinline__ bool mbar_test_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
-// Wait for phase `parity` of `bar` to complete, testing at most `limit`
-// times (a short sleep between tests after the first few, so every test
-// costs a bounded time).  Returns false, and records STATUS_TIMEOUT, if it
-// gave up.
+// Wait for phase `parity` of `bar` to complete: at most `limit` tries, and no
+// new try once about 64 ns x `limit` have passed since the first one (a try
+// itself ends within about 1 ms).
+// Returns false, and records STATUS_TIMEOUT, if it gave up.
 __device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity,
                                                   uint32_t limit, unsigned* status) {
+  uint64_t deadline = 0;
   for (uint32_t i = 0; i < limit; ++i) {
-    if (mbar_test_wait(bar, parity)) return true;
-    if (i >= 16) __nanosleep(64);
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t now = global_ns();
+    if (i == 0) deadline = now + 64ull * limit;
+    else if (now > deadline) break;
   }
   set_status(status, STATUS_TIMEOUT);
   return false;
@@ -106,7 +119,13 @@ __device__ __forceinline__ void bulk_g2s(void* dst_smem, const void* src_gmem, u
       : "memory");
 }
 
-// The number of polls a drain wait (after a timed-out wait, before the CTA
+// Bulk prefetch of `bytes` (multiple of 16, address 16-byte aligned) from
+// global memory into L2.
+__device__ __forceinline__ void bulk_prefetch_l2(const void* src_gmem, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src_gmem), "r"(bytes) : "memory");
+}
+
+// The number of tries a drain wait (after a timed-out wait, before the CTA
 // may exit with a copy still in flight) makes before giving up for good.
 constexpr uint32_t kDrainPolls = 1u << 22;
 
@@ -144,6 +163,14 @@ __device__ __forceinline__ int dsmem_ld_s32(uint32_t addr) {
 }
 __device__ __forceinline__ void dsmem_st_u32(uint32_t addr, uint32_t v) {
   asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
+}
+__device__ __forceinline__ void dsmem_st_u32x2(uint32_t addr, uint2 v) {
+  asm volatile("st.shared::cluster.v2.u32 [%0], {%1, %2};" ::"r"(addr), "r"(v.x), "r"(v.y) : "memory");
+}
+__device__ __forceinline__ void dsmem_st_u32x4(uint32_t addr, uint4 v) {
+  asm volatile("st.shared::cluster.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(v.x), "r"(v.y),
+               "r"(v.z), "r"(v.w)
+               : "memory");
 }
 __device__ __forceinline__ uint2 dsmem_ld_u32x2(uint32_t addr) {
   uint2 v;

@@ -37,8 +37,8 @@
 namespace mpc {
 namespace rows {
 
-constexpr int kNB = 2048;     // bins of the first histogram, CTA kernel
-constexpr int kLCAP = 256;    // candidate keys per row, CTA kernel (whole cluster)
+constexpr int kNB = 1024;   // bins of the first histogram, CTA kernel
+constexpr int kLCAP = 256;  // candidate keys per row, CTA kernel (whole cluster)
 constexpr int kLCAPW = 256;   // candidate keys per row, warp kernel
 constexpr int kMaxCluster = 8;
 constexpr int kSampleThreads = 64;  // threads that read the row sample (4 entries each)
@@ -71,6 +71,38 @@ __device__ __forceinline__ void keys4(const float4 v, int base, int n, int k[4])
     k[2] = (base + 2 < n) ? mag_key(v.z) : -1;
     k[3] = (base + 3 < n) ? mag_key(v.w) : -1;
   }
+}
+
+// Bin of a key (>= 0) in the first histogram of the CTA kernel: |x| * scale
+// rounded down and capped at kNB - 1 (scale = kNB / the largest magnitude of
+// a sample of the row), in FP32 operations only: the cap first, then the
+// floor as the low mantissa bits of p + 2^23 rounded toward zero.  Monotone
+// in the key.
+__device__ __forceinline__ int lin_bin(int key, float scale) {
+  const float p = fminf(fmul(__int_as_float(key), scale), static_cast<float>(kNB - 1));
+  return __float_as_int(__fadd_rz(p, 8388608.0f)) & 0x7fffff;
+}
+
+// The smallest key of bin b (1 <= b < kNB): the least c >= 0 with
+// |x(c)| * scale >= b.  `inv` = 1 / scale, rounded; the start point it gives
+// is a few units off at most and is corrected step by step, with bisection as
+// the bound-free fallback.
+__device__ __forceinline__ int bin_first_key(int b, float scale, float inv) {
+  const float fb = static_cast<float>(b);
+  auto reaches = [&](int c) { return fmul(__int_as_float(c), scale) >= fb; };
+  int c = min(__float_as_int(fmul(fb, inv)), 0x7f800000);
+  for (int i = 0; i < 8 && c > 0 && reaches(c - 1); ++i) --c;
+  for (int i = 0; i < 8 && !reaches(c); ++i) ++c;
+  if (!reaches(c) || (c > 0 && reaches(c - 1))) {
+    int lo = 0, hi = 0x7f800000;  // reaches(hi), !reaches(lo)
+    while (hi - lo > 1) {
+      const int mid = lo + (hi - lo) / 2;
+      if (reaches(mid)) hi = mid;
+      else lo = mid;
+    }
+    c = hi;
+  }
+  return c;
 }
 
 // ---------------------------------------------------------------------------
@@ -120,24 +152,28 @@ template <int NT, int SCAP>
 struct CtaShared {
   static constexpr int NW = NT / 32;
   static constexpr int NCH = SCAP / 128;  // chunks of 128 consecutive entries
-  uint32_t hist[kNB];
-  uint32_t rhist[2][kRoundBins];
-  int lkey[kLCAP];       // this CTA's candidate keys
-  uint16_t lch[kLCAP];   // and their chunks
-  int sel[kLCAP];        // the row's candidate keys (all CTAs), contiguous
-  uint32_t cgt[NCH];     // per chunk: entries kept for being above T
+  // The first histogram; dead once it has been packed and pushed, after which
+  // the same words hold the row's candidate keys, this CTA's candidate chunks
+  // and the histograms of the integer rounds.
+  union {
+    uint32_t hist[kNB];
+    struct {
+      int cand[kLCAP];        // the row's candidates, CTA by CTA (pushed)
+      uint16_t lch[kLCAP];    // chunk of each of this CTA's candidates
+    } c;
+    uint32_t rhist[2][kRoundBins];
+  } u;
+  uint32_t cgt[NCH];     // per chunk: entries kept for being above T (or bin B)
   uint32_t ceq[NCH];     // per chunk: entries equal to T
   uint32_t gbins[128];
-  uint32_t tot_gt[kMaxCluster];  // pushed by the lower ranks of the cluster
+  uint32_t wtot[kMaxCluster][NW];  // per CTA and warp: entries above bin B (pushed)
+  uint32_t tot_gt[kMaxCluster];    // pushed by the lower ranks of the cluster
   uint32_t tot_eq[kMaxCluster];
-  uint32_t gcnt[kMaxCluster];    // candidates of each CTA (pushed)
-  uint32_t gcab[kMaxCluster];    // entries above the chosen bin in each CTA (pushed)
   int red[NW];
   uint32_t ured[NW];
   int sample_max[2];
   uint32_t lcount;
   uint32_t pick_t, pick_excl;
-  uint32_t before_gt, before_eq;
   int pub_lo, pub_hi;
   BinPick pick;
   Threshold thr;
@@ -145,10 +181,10 @@ struct CtaShared {
 };
 
 // The bin holding the kr-th element of an NBINS-bin histogram (bins ranked
-// high to low) summed over the cluster's C CTAs.  Each thread owns a group of
-// G consecutive bins; group sums are pushed to every CTA (table `gsum`,
-// C x NT words), scanned locally, and only the chosen group's bins are pulled
-// from the other CTAs.
+// high to low) summed over the cluster's C CTAs (integer rounds).  Each thread
+// owns a group of G consecutive bins; group sums are pushed to every CTA
+// (table `gsum`, C x NT words), scanned locally, and only the chosen group's
+// bins are pulled from the other CTAs.
 template <int NT, int NBINS, class Sh>
 __device__ __forceinline__ BinPick cluster_pick(const uint32_t* hist, uint32_t* gsum, uint32_t C,
                                                 uint32_t crank, uint32_t kr, Sh& sh, int tid,
@@ -199,40 +235,38 @@ __device__ __forceinline__ BinPick cluster_pick(const uint32_t* hist, uint32_t* 
   return sh.pick;
 }
 
-// Warp 0: exclusive scan of the per-chunk counts in place; returns the totals
-// on lane 31.
+// Warp 0: exclusive scan in place of per-chunk counts; returns the total.
 template <int NCH>
-__device__ __forceinline__ void scan_chunks(uint32_t* cgt, uint32_t* ceq, int lane,
-                                            uint32_t* tot_g, uint32_t* tot_e) {
+__device__ __forceinline__ uint32_t scan_chunks1(uint32_t* c, int lane) {
   constexpr int PER = (NCH + 31) / 32;
-  uint32_t g[PER], e[PER], tg = 0, te = 0;
+  uint32_t g[PER], t = 0;
 #pragma unroll
   for (int j = 0; j < PER; ++j) {
     const int ch = lane * PER + j;
-    g[j] = ch < NCH ? cgt[ch] : 0u;
-    e[j] = ch < NCH ? ceq[ch] : 0u;
-    tg += g[j];
-    te += e[j];
+    g[j] = ch < NCH ? c[ch] : 0u;
+    t += g[j];
   }
-  uint32_t eg = warp_inclusive_scan(tg, lane) - tg;
-  uint32_t ee = warp_inclusive_scan(te, lane) - te;
+  uint32_t e = warp_inclusive_scan(t, lane) - t;
 #pragma unroll
   for (int j = 0; j < PER; ++j) {
     const int ch = lane * PER + j;
-    if (ch < NCH) {
-      cgt[ch] = eg;
-      ceq[ch] = ee;
-    }
-    eg += g[j];
-    ee += e[j];
+    if (ch < NCH) c[ch] = e;
+    e += g[j];
   }
-  *tot_g = eg;
-  *tot_e = ee;
+  return __shfl_sync(kFull, e, 31);
 }
 
-// Bytes of dynamic shared memory of the CTA kernel for cluster size C.
+// Bytes of dynamic shared memory of the CTA kernel for cluster size C: the
+// slice, and the packed histograms of the C CTAs (kNB / 2 words each; the
+// group-sum tables of the integer rounds, 2 x C x NT words, reuse them).
 constexpr int cta_smem_bytes(int NT, int SCAP, int C) {
-  return SCAP * 4 + C * NT * 4 + C * (kLCAP > NT ? kLCAP : NT) * 4;
+  return SCAP * 4 + C * (kNB / 2 > 2 * NT ? kNB / 2 : 2 * NT) * 4;
+}
+
+// Barrier over the row: the cluster, or the CTA when the row has one CTA.
+__device__ __forceinline__ void row_sync(uint32_t C) {
+  if (C > 1) cluster_sync();
+  else __syncthreads();
 }
 
 template <int MODE, int NT, int SCAP, bool FULL>
@@ -241,7 +275,10 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
   constexpr int NQ = SCAP / 4;     // float4 slots per slice
   constexpr int QPT = NQ / NT;     // float4 slots per thread
   constexpr int NCH = SCAP / 128;  // 128-entry chunks per slice
-  constexpr int GB = kLCAP > NT ? kLCAP : NT;
+  constexpr int G = kNB / NT;      // bins of a thread's group in the first histogram
+  constexpr int GW = G / 2;        // packed words of a group (two 16-bit counts each)
+  static_assert(G == 4 || G == 8, "bin groups of 4 or 8");
+  static_assert(SCAP < 65536, "per-CTA bin counts fit 16 bits");
   using Sh = CtaShared<NT, SCAP>;
   __shared__ Sh sh;
   extern __shared__ __align__(16) float4 dyn4[];
@@ -250,8 +287,7 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
   const uint32_t C = cluster_size();
   const uint32_t crank = cluster_rank();
   float4* s4 = dyn4;                                         // NQ float4: ranked values
-  uint32_t* gsumA = reinterpret_cast<uint32_t*>(dyn4 + NQ);  // C x NT group sums
-  uint32_t* gB = gsumA + C * NT;  // C x GB: pushed candidate lists, or group sums of a round
+  uint32_t* table = reinterpret_cast<uint32_t*>(dyn4 + NQ);  // C x NT x GW packed bins
   const int64_t row = blockIdx.x / C;
   const int64_t L = a.L;
   const int64_t k = a.k;
@@ -276,46 +312,52 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
   }
   const float* xrow = a.x + row * L;
 
-  // ---- issue the loads: x by bulk copies, a sample of the row, err / state --
-  // The slice of x arrives in chunks of one float4 slot per thread (4*NT
-  // entries), each completing on its own mbarrier, so the first pass starts on
-  // chunk 0 while the others are still in flight.
-  static_assert(QPT <= 8, "one mbarrier per chunk");
-  const int jmax = (n + 4 * NT - 1) / (4 * NT);  // float4 slots of each thread in use
-  if (a.aligned) {
-    if (tid == 0) {
-      for (int j = 0; j < QPT; ++j) mbar_init(&sh.bars[j], 1);
-      fence_mbar_init();
-    }
-    __syncthreads();
-    if (tid == 0) {
-      for (int j = 0; j < jmax; ++j) {
-        const uint32_t bytes = static_cast<uint32_t>(min(4 * NT, n - 4 * NT * j)) * 4u;
-        mbar_arrive_expect_tx(&sh.bars[j], bytes);
-        bulk_g2s(s4 + j * NT, xrow + c0 + 4 * NT * j, bytes, &sh.bars[j]);
-      }
-    }
-  }
-  // The bin scale comes from a sample of the row, entries [p, p+4) spread over
-  // it, read identically by every CTA of the cluster.
-  float smp[4] = {0.f, 0.f, 0.f, 0.f};
+  // ---- issue the loads: a sample of the row, x by bulk copies, err / state ----
+  // The bin placement comes from a sample of the row, entries [p, p+4) spread
+  // over it, read identically by every CTA of the cluster; it is requested
+  // first, so that it is not queued behind the slices.
+  float sx[4] = {0.f, 0.f, 0.f, 0.f}, sa[4] = {0.f, 0.f, 0.f, 0.f};
   const int64_t sp = (L / kSampleThreads) * tid / 4 * 4;
   if (tid < kSampleThreads) {
+    if (a.aligned && sp + 4 <= L) {
+      const float4 v = *reinterpret_cast<const float4*>(xrow + sp);
+      sx[0] = v.x, sx[1] = v.y, sx[2] = v.z, sx[3] = v.w;
+      if (MODE != kPlain) {
+        const float4 w = *reinterpret_cast<const float4*>(arow + sp);
+        sa[0] = w.x, sa[1] = w.y, sa[2] = w.z, sa[3] = w.w;
+      }
+    } else {
 #pragma unroll
-    for (int i = 0; i < 4; ++i)
-      if (sp + i < L)
-        smp[i] = ranked_value<MODE>(xrow[sp + i], (MODE != kPlain) ? arow[sp + i] : 0.0f);
-  }
-  float4 av[QPT];
-  if (a.aligned && MODE != kPlain) {
-#pragma unroll
-    for (int j = 0; j < QPT; ++j) {
-      const int q = j * NT + tid;
-      av[j] = (4 * q < n) ? *reinterpret_cast<const float4*>(arow + c0 + 4 * q)
-                          : make_float4(0.f, 0.f, 0.f, 0.f);
+      for (int i = 0; i < 4; ++i)
+        if (sp + i < L) {
+          sx[i] = xrow[sp + i];
+          if (MODE != kPlain) sa[i] = arow[sp + i];
+        }
     }
   }
-  for (int i = tid; i < kNB; i += NT) sh.hist[i] = 0;
+  // The slice of x arrives in chunks of one float4 slot per thread (4*NT
+  // entries), each completing on its own mbarrier and issued by its own lane,
+  // so the first pass starts on chunk 0 while the others are in flight.
+  static_assert(QPT <= 8, "one mbarrier per chunk");
+  const int jmax = (n + 4 * NT - 1) / (4 * NT);  // float4 slots of each thread in use
+  // The matching chunks of the error / state slice are prefetched into L2 by
+  // the same lanes and read from there chunk by chunk in the first pass.
+  if (a.aligned && warp == 0 && lane < jmax) {
+    const uint32_t bytes = static_cast<uint32_t>(min(4 * NT, n - 4 * NT * lane)) * 4u;
+    if (MODE != kPlain) bulk_prefetch_l2(arow + c0 + 4 * NT * lane, bytes);
+    mbar_init(&sh.bars[lane], 1);
+    fence_mbar_init();
+    mbar_arrive_expect_tx(&sh.bars[lane], bytes);
+    bulk_g2s(s4 + lane * NT, xrow + c0 + 4 * NT * lane, bytes, &sh.bars[lane]);
+  }
+  auto aux4 = [&](int j) {
+    const int q = j * NT + tid;
+    return (a.aligned && MODE != kPlain && j < QPT && 4 * q < n)
+               ? *reinterpret_cast<const float4*>(arow + c0 + 4 * q)
+               : make_float4(0.f, 0.f, 0.f, 0.f);
+  };
+  float4 anext = aux4(0);
+  for (int i = tid; i < kNB; i += NT) sh.u.hist[i] = 0;
   if (tid == 0) {
     sh.lcount = 0;
     sh.thr = Threshold{0x7fffffff, 0};
@@ -324,7 +366,7 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
     int smax = -1;
 #pragma unroll
     for (int i = 0; i < 4; ++i)
-      if (sp + i < L) smax = max(smax, mag_key(smp[i]));
+      if (sp + i < L) smax = max(smax, mag_key(ranked_value<MODE>(sx[i], sa[i])));
     smax = __reduce_max_sync(kFull, smax);
     if (lane == 0) sh.sample_max[warp] = smax;
   }
@@ -334,7 +376,8 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
       s[e] = ranked_value<MODE>(xrow[c0 + e], (MODE != kPlain) ? arow[c0 + e] : 0.0f);
   }
   __syncthreads();
-  const float scale = bucket_scale(max(sh.sample_max[0], sh.sample_max[1]), kNB);
+  const int smax = max(sh.sample_max[0], sh.sample_max[1]);
+  const float scale = bucket_scale(smax, kNB);
   const bool binned = k < L && scale > 0.0f;
 
   // ---- ranked values into shared memory and the first histogram -------------
@@ -343,6 +386,8 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
 #pragma unroll
   for (int j = 0; j < QPT; ++j) {
     if (j < jmax) {
+      const float4 acur = anext;
+      if (MODE != kPlain && j + 1 < QPT) anext = aux4(j + 1);
       if (a.aligned && !mbar_wait_bounded(&sh.bars[j], 0, a.spin_limit, a.status)) {
         mbar_wait_bounded(&sh.bars[j], 0, kDrainPolls, nullptr);
         failed = true;
@@ -350,7 +395,7 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
       const int q = j * NT + tid;
       float4 v = s4[q];
       if (MODE != kPlain && a.aligned) {
-        v = ranked4<MODE>(v, av[j]);
+        v = ranked4<MODE>(v, acur);
         s4[q] = v;
       }
       if (binned) {
@@ -359,14 +404,14 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
           if (kk[i] == 0) ++zc;
-          else if (kk[i] > 0) atomicAdd(&sh.hist[bucket_of(kk[i], scale, kNB)], 1u);
+          else if (kk[i] > 0) atomicAdd(&sh.u.hist[lin_bin(kk[i], scale)], 1u);
         }
       }
     }
   }
   if (binned) {
     zc = __reduce_add_sync(kFull, zc);
-    if (lane == 0 && zc) atomicAdd(&sh.hist[0], zc);
+    if (lane == 0 && zc) atomicAdd(&sh.u.hist[0], zc);
   }
   failed = __syncthreads_or(failed);
   // A slice whose copy timed out takes part in the rest as an empty one (the
@@ -377,22 +422,125 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
   // ---- select T and need -----------------------------------------------------
   int T = -1;
   uint32_t need = 0;
-  bool counted = false;  // per-chunk counts and the counts of earlier CTAs are in place
-  uint32_t gt_before = 0, eq_before = 0;
+  bool counted = false;  // per-chunk counts of kept entries are in place (fast path)
+  uint32_t own = 0, off = 0;  // this CTA's candidates and those of the CTAs before it
   if (k < L) {
     uint32_t kr = static_cast<uint32_t>(k);
     int B = 0;
     uint32_t m = static_cast<uint32_t>(L);  // with scale 0 every entry is a candidate
+    int kl = 0, kh = 0x7fffffff;            // the keys of bin B
     if (scale > 0.0f) {
-      const BinPick p = cluster_pick<NT, kNB>(sh.hist, gsumA, C, crank, kr, sh, tid, lane, warp);
-      B = p.bin;
-      kr -= p.above;
-      m = p.count;
+      // Every CTA pushes its histogram, packed two 16-bit counts to a word, to
+      // every CTA of the row; thread t owns group t of G bins (groups ranked
+      // high to low).
+      {
+        const int b0 = kNB - G * (tid + 1);
+        uint32_t w[GW];
+#pragma unroll
+        for (int i = 0; i < GW; ++i) w[i] = sh.u.hist[b0 + 2 * i] | (sh.u.hist[b0 + 2 * i + 1] << 16);
+        uint32_t* dst = table + (crank * NT + tid) * GW;
+        if (C > 1) {
+          for (uint32_t r = 0; r < C; ++r) {
+            if (GW == 2) dsmem_st_u32x2(dsmem_addr(dst, r), make_uint2(w[0], w[1]));
+            else dsmem_st_u32x4(dsmem_addr(dst, r), make_uint4(w[0], w[1], w[GW > 2 ? 2 : 0], w[GW > 3 ? 3 : 0]));
+          }
+        } else {
+#pragma unroll
+          for (int i = 0; i < GW; ++i) dst[i] = w[i];
+        }
+      }
+      row_sync(C);
+      // counts of group g's bins (ascending) summed over the row
+      auto group_bins = [&](int g, uint32_t (&cnt)[G]) {
+#pragma unroll
+        for (int b = 0; b < G; ++b) cnt[b] = 0;
+        for (uint32_t r = 0; r < C; ++r) {
+          const uint32_t* src = table + (r * NT + g) * GW;
+#pragma unroll
+          for (int i = 0; i < GW; ++i) {
+            const uint32_t wv = src[i];
+            cnt[2 * i] += wv & 0xffffu;
+            cnt[2 * i + 1] += wv >> 16;
+          }
+        }
+      };
+      uint32_t cnt[G];
+      group_bins(tid, cnt);
+      uint32_t total = 0;
+#pragma unroll
+      for (int b = 0; b < G; ++b) total += cnt[b];
+      const uint32_t incl = warp_inclusive_scan(total, lane);
+      if (lane == 31) sh.ured[warp] = incl;
+      __syncthreads();
+      // the warp whose groups hold the kr-th entry (every thread finds the same)
+      uint32_t wbase = 0;
+      int ws = NW - 1;
+#pragma unroll
+      for (int w = 0; w < NW; ++w) {
+        const uint32_t u = sh.ured[w];
+        if (ws == NW - 1 && w < NW - 1) {
+          if (wbase + u >= kr) ws = w;
+          else wbase += u;
+        }
+      }
+      // every warp ranks that warp's groups and bins itself
+      uint32_t c2[G];
+      if (warp == ws) {
+#pragma unroll
+        for (int b = 0; b < G; ++b) c2[b] = cnt[b];
+      } else {
+        group_bins(ws * 32 + lane, c2);
+      }
+      uint32_t t2 = 0;
+#pragma unroll
+      for (int b = 0; b < G; ++b) t2 += c2[b];
+      const uint32_t ex2 = wbase + warp_inclusive_scan(t2, lane) - t2;
+      const unsigned who = __ballot_sync(kFull, ex2 < kr && kr <= ex2 + t2);
+      const int src = who ? __ffs(who) - 1 : 31;
+      const int gb0 = kNB - G * (ws * 32 + lane + 1);
+      int pb = gb0;
+      uint32_t pab = ex2, pc = c2[0];
+      {
+        uint32_t run = ex2;
+        bool done = false;
+#pragma unroll
+        for (int b = G - 1; b >= 0; --b) {
+          if (!done && run + c2[b] >= kr) {
+            pb = gb0 + b;
+            pab = run;
+            pc = c2[b];
+            done = true;
+          }
+          if (!done) run += c2[b];
+        }
+      }
+      B = __shfl_sync(kFull, pb, src);
+      kr -= __shfl_sync(kFull, pab, src);
+      m = __shfl_sync(kFull, pc, src);
+      {
+        // this CTA's entries in bin B and those of the CTAs before it
+        const int gB = (kNB - 1 - B) / G;
+        const int ib = B - (kNB - G * (gB + 1));
+        for (uint32_t r = 0; r <= crank; ++r) {
+          const uint32_t wv = table[(r * NT + gB) * GW + ib / 2];
+          const uint32_t cr = (ib & 1) ? (wv >> 16) : (wv & 0xffffu);
+          if (r < crank) off += cr;
+          else own = cr;
+        }
+      }
+      // lanes 0 and 1 find the first keys of bins B and B + 1 side by side
+      const int bb = B + (lane & 1);
+      const float inv = fmul(__int_as_float(smax), 1.0f / kNB);
+      const int fk = (bb >= 1 && bb < kNB) ? bin_first_key(bb, scale, inv) : 0;
+      kl = (B == 0) ? 0 : __shfl_sync(kFull, fk, 0);
+      kh = (B == kNB - 1) ? 0x7fffffff : __shfl_sync(kFull, fk, 1) - 1;
     }
 
     if (scale > 0.0f && m <= static_cast<uint32_t>(kLCAP)) {
-      // ---- count and collect: entries above bin B are kept; the m entries
-      // in it are the candidates for T ---------------------------------------
+      // ---- count and collect: entries above bin B are kept; the m entries in
+      // it are the candidates for T, pushed to every CTA of the row at their
+      // place in the row's candidate table ------------------------------------
+      uint32_t wab = 0;
 #pragma unroll 2
       for (int j = 0; j < QPT; ++j) {
         uint32_t ab = 0;
@@ -402,105 +550,69 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
           keys4<FULL>(s4[q], 4 * q, nv, kk);
 #pragma unroll
           for (int i = 0; i < 4; ++i) {
-            if (FULL || kk[i] >= 0) {
-              const int b = bucket_of(kk[i], scale, kNB);
-              ab += b > B;
-              if (b == B) {
-                const uint32_t at = atomicAdd(&sh.lcount, 1u);
-                if (at < kLCAP) {
-                  sh.lkey[at] = kk[i];
-                  sh.lch[at] = static_cast<uint16_t>(j * NW + warp);
+            ab += kk[i] > kh;
+            if (kk[i] >= kl && kk[i] <= kh) {
+              const uint32_t at = atomicAdd(&sh.lcount, 1u);
+              if (at < own) {
+                sh.u.c.lch[at] = static_cast<uint16_t>(j * NW + warp);
+                int* slot = &sh.u.c.cand[off + at];
+                if (C > 1) {
+                  for (uint32_t r = 0; r < C; ++r)
+                    dsmem_st_u32(dsmem_addr(slot, r), static_cast<uint32_t>(kk[i]));
+                } else {
+                  *slot = kk[i];
                 }
               }
             }
           }
           ab = __reduce_add_sync(kFull, ab);
         }
-        if (lane == 0) {
-          sh.cgt[j * NW + warp] = ab;
-          sh.ceq[j * NW + warp] = 0;
+        if (lane == 0) sh.cgt[j * NW + warp] = ab;
+        wab += ab;
+      }
+      if (lane == 0) {
+        uint32_t* slot = &sh.wtot[crank][warp];
+        if (C > 1) {
+          for (uint32_t r = 0; r < C; ++r) dsmem_st_u32(dsmem_addr(slot, r), wab);
+        } else {
+          *slot = wab;
         }
       }
-      __syncthreads();
-      const uint32_t lc = min(sh.lcount, static_cast<uint32_t>(kLCAP));
-      const int* list = sh.lkey;
-      uint32_t mt = lc;
-      if (C > 1) {
-        // push this CTA's candidates and its above-bin count to every CTA
-        if (warp == 0) {
-          uint32_t cab = 0;
-          for (int ch = lane; ch < NCH; ch += 32) cab += sh.cgt[ch];
-          cab = __reduce_add_sync(kFull, cab);
-          if (lane == 0)
-            for (uint32_t r = 0; r < C; ++r) {
-              dsmem_st_u32(dsmem_addr(&sh.gcnt[crank], r), lc);
-              dsmem_st_u32(dsmem_addr(&sh.gcab[crank], r), cab);
-            }
+      row_sync(C);  // the last cluster barrier: nothing is read remotely after it
+      if (warp == 0) scan_chunks1<NCH>(sh.cgt, lane);
+      // P threads rank each candidate against the whole list (P a power of two,
+      // m x P <= NT); the group holding T reports it (all such groups report
+      // the same values)
+      {
+        uint32_t P = 1;
+        while (P < 32 && m * P * 2 <= static_cast<uint32_t>(NT)) P *= 2;
+        const uint32_t ci = static_cast<uint32_t>(tid) / P, part = static_cast<uint32_t>(tid) % P;
+        uint32_t gt = 0, ge = 0;
+        int ki = 0;
+        if (ci < m) {
+          ki = sh.u.c.cand[ci];
+          for (uint32_t j = part; j < m; j += P) {
+            const int aj = sh.u.c.cand[j];
+            gt += aj > ki;
+            ge += aj >= ki;
+          }
         }
-        for (uint32_t p = tid; p < lc; p += NT) {
-          const uint32_t key = static_cast<uint32_t>(sh.lkey[p]);
-          uint32_t* slot = gB + crank * GB + p;
-          for (uint32_t r = 0; r < C; ++r) dsmem_st_u32(dsmem_addr(slot, r), key);
+        for (uint32_t o = P >> 1; o > 0; o >>= 1) {
+          gt += __shfl_xor_sync(kFull, gt, o);
+          ge += __shfl_xor_sync(kFull, ge, o);
         }
-        cluster_sync();  // the last cluster barrier: nothing is read remotely after it
-        uint32_t off = 0;
-        for (uint32_t r = 0; r < C; ++r) {
-          const uint32_t cnt = sh.gcnt[r];
-          for (uint32_t p = tid; p < cnt && off + p < kLCAP; p += NT)
-            sh.sel[off + p] = static_cast<int>(gB[r * GB + p]);
-          off += cnt;
+        if (ci < m && part == 0 && gt < kr && kr <= ge) {
+          const uint32_t nd = kr - gt;
+          sh.thr = (nd == ge - gt) ? Threshold{ki - 1, 0u} : Threshold{ki, nd};
         }
-        __syncthreads();
-        list = sh.sel;
-        mt = min(off, static_cast<uint32_t>(kLCAP));
-      }
-      // every thread ranks its candidates against the whole list; the
-      // thread holding T reports it (all such threads report the same values)
-      for (uint32_t i = tid; i < mt; i += NT) {
-        Threshold ti;
-        if (rank_is_threshold(list, mt, kr, list[i], &ti)) sh.thr = ti;
       }
       __syncthreads();
       T = sh.thr.T;
       need = sh.thr.need;
-      // candidates above T, or equal to it, join their chunks' counts
-      for (uint32_t p = tid; p < lc; p += NT) {
-        const int key = sh.lkey[p];
-        if (key > T) atomicAdd(&sh.cgt[sh.lch[p]], 1u);
-        else if (key == T) atomicAdd(&sh.ceq[sh.lch[p]], 1u);
-      }
-      if (C > 1 && warp == 0) {
-        // kept entries of the earlier CTAs of the row
-        uint32_t gb = 0, eb = 0;
-        for (uint32_t r = 0; r < crank; ++r) {
-          if (lane == 0) gb += sh.gcab[r];
-          const uint32_t cnt = sh.gcnt[r];
-          for (uint32_t p = lane; p < cnt; p += 32) {
-            const int key = static_cast<int>(gB[r * GB + p]);
-            gb += key > T;
-            eb += key == T;
-          }
-        }
-        gb = __reduce_add_sync(kFull, gb);
-        eb = __reduce_add_sync(kFull, eb);
-        if (lane == 0) {
-          sh.before_gt = gb;
-          sh.before_eq = eb;
-        }
-      }
-      __syncthreads();
-      if (warp == 0) {
-        uint32_t tg, te;
-        scan_chunks<NCH>(sh.cgt, sh.ceq, lane, &tg, &te);
-      }
-      __syncthreads();
-      if (C > 1) {
-        gt_before = sh.before_gt;
-        eq_before = sh.before_eq;
-      }
+      own = min(own, sh.lcount);
       counted = true;
     } else {
-      // ---- too many candidates for the list: integer rounds over the slice --
+      // ---- too many candidates for the table: integer rounds over the slice --
       int lo = 0x7fffffff, hi = -1;
 #pragma unroll 2
       for (int j = 0; j < jv; ++j) {
@@ -509,7 +621,7 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
         keys4<FULL>(s4[q], 4 * q, nv, kk);
 #pragma unroll
         for (int i = 0; i < 4; ++i)
-          if (kk[i] >= 0 && (scale == 0.0f || bucket_of(kk[i], scale, kNB) == B)) {
+          if (kk[i] >= kl && kk[i] <= kh) {
             lo = min(lo, kk[i]);
             hi = max(hi, kk[i]);
           }
@@ -521,6 +633,8 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
           sh.pub_lo = lo;
           sh.pub_hi = hi;
         }
+        // also the point after which no CTA reads the packed histograms, whose
+        // words the round tables reuse
         cluster_sync();
         for (uint32_t r = 0; r < C; ++r) {
           lo = min(lo, dsmem_ld_s32(dsmem_addr(&sh.pub_lo, r)));
@@ -535,7 +649,7 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
           break;
         }
         const int sft = round_shift(lo, hi);
-        for (int i = tid; i < kRoundBins; i += NT) sh.rhist[p][i] = 0;
+        for (int i = tid; i < kRoundBins; i += NT) sh.u.rhist[p][i] = 0;
         __syncthreads();
 #pragma unroll 2
         for (int j = 0; j < jv; ++j) {
@@ -545,12 +659,12 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
 #pragma unroll
           for (int i = 0; i < 4; ++i)
             if (kk[i] >= lo && kk[i] <= hi)
-              atomicAdd(&sh.rhist[p][static_cast<uint32_t>(kk[i] - lo) >> sft], 1u);
+              atomicAdd(&sh.u.rhist[p][static_cast<uint32_t>(kk[i] - lo) >> sft], 1u);
         }
         __syncthreads();
         // the group-sum table alternates from round to round, so a push never
         // lands on sums another CTA may still be reading
-        const BinPick q = cluster_pick<NT, kRoundBins>(sh.rhist[p], p == 0 ? gB : gsumA, C,
+        const BinPick q = cluster_pick<NT, kRoundBins>(sh.u.rhist[p], table + p * C * NT, C,
                                                        crank, kr, sh, tid, lane, warp);
         kr -= q.above;
         const int nlo = lo + (q.bin << sft);
@@ -568,6 +682,7 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
     }
   }
 
+  uint32_t gt_before = 0, eq_before = 0;  // kept / tied entries of the earlier CTAs
   if (!counted) {
     // ---- count kept entries per 128-entry chunk ------------------------------
 #pragma unroll 2
@@ -592,8 +707,8 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
     }
     __syncthreads();
     if (warp == 0) {
-      uint32_t tg, te;
-      scan_chunks<NCH>(sh.cgt, sh.ceq, lane, &tg, &te);
+      const uint32_t tg = scan_chunks1<NCH>(sh.cgt, lane);
+      const uint32_t te = scan_chunks1<NCH>(sh.ceq, lane);
       if (C > 1 && lane == 31) {
         // push this slice's totals to every later CTA of the row
         for (uint32_t r = crank + 1; r < C; ++r) {
@@ -602,28 +717,65 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
         }
       }
     }
-    if (C > 1) {
-      cluster_sync();  // the last cluster barrier: nothing is read remotely after it
-      for (uint32_t r = 0; r < crank; ++r) {
-        gt_before += sh.tot_gt[r];
-        eq_before += sh.tot_eq[r];
-      }
-    } else {
-      __syncthreads();
+    row_sync(C);  // the last cluster barrier: nothing is read remotely after it
+    for (uint32_t r = 0; r < crank; ++r) {
+      gt_before += sh.tot_gt[r];
+      eq_before += sh.tot_eq[r];
     }
+  }
+
+  if (counted) {
+    // The chunk counts hold the entries above bin B before each chunk.  Each
+    // warp adds, for its own chunks ch_j = j * NW + warp, this CTA's
+    // candidates above T in earlier chunks, and sets the ties (== T) there.
+    uint32_t cg[QPT], ce[QPT];
+#pragma unroll
+    for (int j = 0; j < QPT; ++j) cg[j] = ce[j] = 0;
+    for (uint32_t p = lane; p < own; p += 32) {
+      const int key = sh.u.c.cand[off + p];
+      const int ch = sh.u.c.lch[p];
+      const uint32_t g = key > T, e = key == T;
+#pragma unroll
+      for (int j = 0; j < QPT; ++j) {
+        const bool before = ch < j * NW + warp;
+        cg[j] += before ? g : 0u;
+        ce[j] += before ? e : 0u;
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < QPT; ++j) {
+      const uint32_t g = __reduce_add_sync(kFull, cg[j]);
+      const uint32_t e = need ? __reduce_add_sync(kFull, ce[j]) : 0u;
+      if (lane == 0) {
+        sh.cgt[j * NW + warp] += g;
+        sh.ceq[j * NW + warp] = e;
+      }
+    }
+    // the earlier CTAs' kept entries and ties
+    uint32_t gb = 0, eb = 0;
+    for (uint32_t p = lane; p < off; p += 32) {
+      const int key = sh.u.c.cand[p];
+      gb += key > T;
+      eb += key == T;
+    }
+    for (uint32_t i = lane; i < crank * NW; i += 32) gb += sh.wtot[i / NW][i % NW];
+    gt_before = __reduce_add_sync(kFull, gb);
+    eq_before = need ? __reduce_add_sync(kFull, eb) : 0u;
+    __syncwarp();
   }
 
   // ---- write the payload (ascending column) and the buffers -----------------
   float* vrow = a.vals + row * k;
   int32_t* irow = a.idx + row * k;
+  const uint32_t kk32 = static_cast<uint32_t>(min64(k, 0x7fffffff));
   const unsigned lt = lanemask_lt();
 #pragma unroll 2
   for (int j = 0; j < jv; ++j) {
-    const int ch = j * NW + warp;
     const int q = j * NT + tid;
     const float4 v4 = s4[q];
     int kk[4];
     keys4<FULL>(v4, 4 * q, nv, kk);
+    const int ch = j * NW + warp;
     const uint32_t eqt = eq_before + sh.ceq[ch];
     uint32_t pos = gt_before + sh.cgt[ch] + min(need, eqt);
     bool kp[4];
@@ -647,19 +799,19 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
     if (!FULL && e0 >= nv) continue;
     const float val[4] = {v4.x, v4.y, v4.z, v4.w};
     const int col = static_cast<int>(c0) + e0;
-    for (uint32_t bits = (kp[0] ? 1u : 0u) | (kp[1] ? 2u : 0u) | (kp[2] ? 4u : 0u) |
-                         (kp[3] ? 8u : 0u);
-         bits; bits &= bits - 1u, ++pos) {
-      const int i = __ffs(bits) - 1;
-      const float vi = i == 0 ? val[0] : i == 1 ? val[1] : i == 2 ? val[2] : val[3];
-      if (pos < static_cast<uint64_t>(k)) {
-        vrow[pos] = vi;
-        irow[pos] = col + i;
-      }
-      if (MODE == kDelta) {
-        // state + d, against the same state value d was formed from
-        float* sp = arow + col + i;
-        *sp = fadd(*sp, vi);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      if (kp[i]) {
+        if (pos < kk32) {
+          vrow[pos] = val[i];
+          irow[pos] = col + i;
+        }
+        if (MODE == kDelta) {
+          // state + d, against the same state value d was formed from
+          float* sp = arow + col + i;
+          *sp = fadd(*sp, val[i]);
+        }
+        ++pos;
       }
     }
     if (MODE == kEF) {
