@@ -13,8 +13,9 @@ one boundary crossing of every operator the workload sweeps, on that step's tens
 value = sum over the 9 compress+decompress pairs of the input bytes (4 x 128 x 32768) /
 device time of the step.  Each step is one CUDA graph of the 18 library launches (one
 graph per slot of a pool of 4 pre-drawn steps, so inputs differ from step to step), with
-no event nodes inside; L2 is flushed (256 MiB write) before every timed step and the
-flush is outside the timed interval.  Per-launch times come from a second timed pass
+no event nodes inside; L2 is flushed before every timed step by writing and then
+reading a 256 MiB buffer (so the step's inputs are cold and the flush leaves no dirty
+lines for the first launch to write back), outside the timed interval.  Per-launch times come from a second timed pass
 whose graphs record an event after every launch, and the dominant launch's duration
 (for `roofline`) from a third pass with one event pair around that launch only.  `e2e` runs the same steps through the Python API without graphs, with the
 step's inputs copied from pinned host memory and two outputs copied back inside the
@@ -373,8 +374,16 @@ def run_ours(args, rank, local, world):
     st = Step(mpc, synth, device, seed)
     n_ops = len(st.ops)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=device)
+    flush_sink = torch.empty((), dtype=torch.int64, device=device)
     stream = torch.cuda.Stream(device)
     torch.cuda.synchronize()
+
+    def flush_l2(i):
+        # write then read a buffer twice the size of L2: the step's inputs leave
+        # L2, and the flush leaves no dirty lines whose write-back the first
+        # launch of the step would pay for
+        flush.fill_(i & 0xff)
+        torch.sum(flush, dim=0, dtype=torch.int64, out=flush_sink)
 
     # eager warm-up (sets kernel attributes) before capture
     with torch.cuda.stream(stream):
@@ -408,7 +417,7 @@ def run_ours(args, rank, local, world):
         ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
         with torch.cuda.stream(stream):
             for w in range(args.warmup):
-                flush.fill_(w & 0xff)
+                flush_l2(w)
                 graphs[w % POOL].replay()
         stream.synchronize()
         barrier(world)
@@ -418,7 +427,7 @@ def run_ours(args, rank, local, world):
         t0 = time.perf_counter()
         with torch.cuda.stream(stream):
             for i in range(args.steps):
-                flush.fill_(i & 0xff)
+                flush_l2(i)
                 starts[i].record(stream)
                 graphs[i % POOL].replay()
                 ends[i].record(stream)
@@ -507,8 +516,9 @@ def run_ours(args, rank, local, world):
             "config": {"workload": WORKLOAD, "rows": R, "row_len": L,
                        "topk_percents": list(TOPK_PCTS), "bits": list(BITS),
                        "rounding": ["nearest", "stochastic"], "launches_per_step": n_ops,
-                       "step": "one CUDA graph per step (no event nodes inside)", "l2": "256 MiB flush "
-                       "before each timed step, outside the timed interval", "parallelism":
+                       "step": "one CUDA graph per step (no event nodes inside)", "l2": "256 MiB buffer "
+                       "written then read before each timed step, outside the timed interval "
+                       "(inputs cold, no dirty lines left by the flush)", "parallelism":
                        "replicas" if world > 1 else "single GPU"},
             "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
             "gpu_launches": n_ops * args.steps, "clocks": clocks,
@@ -568,6 +578,7 @@ def time_op(fn, stream, flush, reps=5):
         fn()
         for r in range(reps):
             flush.fill_(r)
+            flush.sum(dtype=torch.int64)
             a = torch.cuda.Event(enable_timing=True)
             b = torch.cuda.Event(enable_timing=True)
             a.record(stream)

@@ -189,7 +189,7 @@ struct QuantShared {
   uint32_t redmax[kQNT / 32];
   uint32_t mm_min[8];  // per-CTA extrema of the row, pushed by every CTA of the cluster
   uint32_t mm_max[8];
-  uint64_t bar;
+  uint64_t bars[kQNV];  // one per slice chunk
 };
 
 template <int BITS>
@@ -206,42 +206,52 @@ __global__ void __launch_bounds__(kQNT) quant_cta_kernel(const QuantArgs a, int 
   const int n = static_cast<int>(max64(0, min64(a.slice, L - c0)));
   const float* xr = a.x + row * L;
 
+  // The slice arrives in chunks of one float4 per thread (4 x kQNT entries),
+  // each on its own mbarrier and issued by its own lane of warp 0; the
+  // extrema are taken chunk by chunk as the chunks land.
   bool failed = false;
-  if (a.aligned) {
-    if (tid == 0) {
-      mbar_init(&sh.bar, 1);
-      fence_mbar_init();
-    }
-    __syncthreads();
-    if (n > 0) {
-      if (tid == 0) {
-        mbar_arrive_expect_tx(&sh.bar, static_cast<uint32_t>(n) * 4u);
-        bulk_g2s(sx, xr + c0, static_cast<uint32_t>(n) * 4u, &sh.bar);
-      }
-      if (!mbar_wait_bounded(&sh.bar, 0, a.spin_limit, a.status)) {
-        mbar_wait_bounded(&sh.bar, 0, kDrainPolls, nullptr);
+  const int jmax = (n + 4 * kQNT - 1) / (4 * kQNT);
+  if (a.aligned && warp == 0 && lane < jmax) {
+    const uint32_t bytes = static_cast<uint32_t>(min(4 * kQNT, n - 4 * kQNT * lane)) * 4u;
+    mbar_init(&sh.bars[lane], 1);
+    fence_mbar_init();
+    mbar_arrive_expect_tx(&sh.bars[lane], bytes);
+    bulk_g2s(sx + 4 * kQNT * lane, xr + c0 + 4 * kQNT * lane, bytes, &sh.bars[lane]);
+  }
+  if (!a.aligned)
+    for (int e = tid; e < n; e += kQNT) sx[e] = xr[c0 + e];
+  __syncthreads();
+  uint32_t kmin = 0xffffffffu, kmax = 0u;
+#pragma unroll
+  for (int v = 0; v < kQNV; ++v) {
+    if (v < jmax) {
+      if (a.aligned && !mbar_wait_bounded(&sh.bars[v], 0, a.spin_limit, a.status)) {
+        mbar_wait_bounded(&sh.bars[v], 0, kDrainPolls, nullptr);
         failed = true;
       }
+      const int q = v * kQNT + tid;
+      const float4 f = reinterpret_cast<const float4*>(sx)[q];
+      const float xs[4] = {f.x, f.y, f.z, f.w};
+#pragma unroll
+      for (int t = 0; t < 4; ++t)
+        if (4 * q + t < n) {
+          const uint32_t ok = ord_key(xs[t]);
+          kmin = min(kmin, ok);
+          kmax = max(kmax, ok);
+        }
     }
-    failed = __syncthreads_or(failed);
-  } else {
-    for (int e = tid; e < n; e += kQNT) sx[e] = xr[c0 + e];
-    __syncthreads();
   }
+  failed = __syncthreads_or(failed);
   const int nv = failed ? 0 : n;
 
-  uint32_t kmin, kmax;
   if (from_ws) {
     const uint32_t* mm = static_cast<const uint32_t*>(a.ws) + 2 * row;
     kmin = mm[0];
     kmax = mm[1];
   } else {
-    kmin = 0xffffffffu;
-    kmax = 0u;
-    for (int e = tid; e < nv; e += kQNT) {
-      const uint32_t ok = ord_key(sx[e]);
-      kmin = min(kmin, ok);
-      kmax = max(kmax, ok);
+    if (failed) {
+      kmin = 0xffffffffu;
+      kmax = 0u;
     }
     kmin = __reduce_min_sync(kFull, kmin);
     kmax = __reduce_max_sync(kFull, kmax);
@@ -250,16 +260,15 @@ __global__ void __launch_bounds__(kQNT) quant_cta_kernel(const QuantArgs a, int 
       sh.redmax[warp] = kmax;
     }
     __syncthreads();
-    if (tid == 0) {
-      uint32_t a0 = 0xffffffffu, a1 = 0u;
-      for (int w = 0; w < kQNT / 32; ++w) {
-        a0 = min(a0, sh.redmin[w]);
-        a1 = max(a1, sh.redmax[w]);
-      }
+    if (warp == 0) {
+      uint32_t a0 = lane < kQNT / 32 ? sh.redmin[lane] : 0xffffffffu;
+      uint32_t a1 = lane < kQNT / 32 ? sh.redmax[lane] : 0u;
+      a0 = __reduce_min_sync(kFull, a0);
+      a1 = __reduce_max_sync(kFull, a1);
       // push this slice's extrema into every CTA of the cluster (itself included)
-      for (uint32_t r = 0; r < C; ++r) {
-        dsmem_st_u32(dsmem_addr(&sh.mm_min[sidx], r), a0);
-        dsmem_st_u32(dsmem_addr(&sh.mm_max[sidx], r), a1);
+      if (lane < static_cast<int>(C)) {
+        dsmem_st_u32(dsmem_addr(&sh.mm_min[sidx], lane), a0);
+        dsmem_st_u32(dsmem_addr(&sh.mm_max[sidx], lane), a1);
       }
     }
     if (C > 1) cluster_sync(); else __syncthreads();
@@ -374,11 +383,56 @@ __global__ void __launch_bounds__(256)
   }
 }
 
+// Rows with a 16-byte aligned output and L % 4 == 0: every thread writes whole
+// float4s, consecutive lanes consecutive float4s (512-byte warp stores), from
+// the one code word that holds their 4 codes; bpr blocks per row, kDqU float4
+// per thread.
+constexpr int kDqU = 4;
+
+template <int BITS>
+__global__ void __launch_bounds__(256)
+    dequant_rows_kernel(const uint32_t* __restrict__ codes, const float* __restrict__ scale,
+                        const float* __restrict__ minv, int64_t L, int64_t W, int bpr,
+                        float* __restrict__ y) {
+  const int64_t row = blockIdx.x / bpr;
+  const int64_t f0 = static_cast<int64_t>(blockIdx.x % bpr) * (256 * kDqU);
+  const int64_t n4 = L / 4;
+  const uint32_t* cr = codes + row * W;
+  float4* yr = reinterpret_cast<float4*>(y + row * L);
+  const float sc = scale[row], m = minv[row];
+  uint32_t w[kDqU];
+#pragma unroll
+  for (int u = 0; u < kDqU; ++u) {
+    const int64_t f = f0 + u * 256 + threadIdx.x;
+    w[u] = (f < n4) ? cr[(f * 4 * BITS) >> 5] : 0u;
+  }
+#pragma unroll
+  for (int u = 0; u < kDqU; ++u) {
+    const int64_t f = f0 + u * 256 + threadIdx.x;
+    if (f < n4) {
+      const uint32_t word = w[u] >> ((f * 4 * BITS) & 31);
+      float o[4];
+#pragma unroll
+      for (int t = 0; t < 4; ++t)
+        o[t] = fadd(m, fmul(static_cast<float>((word >> (BITS * t)) & ((1u << BITS) - 1u)), sc));
+      yr[f] = make_float4(o[0], o[1], o[2], o[3]);
+    }
+  }
+}
+
 // 32-bit word indexing whenever the code array allows it (cheaper division).
 template <int BITS>
 void launch_dequant(const uint32_t* codes, const float* scale, const float* minv, int64_t rows,
                     int64_t L, int64_t W, int64_t wpr, float* y, int aligned, unsigned grid,
                     cudaStream_t s) {
+  if (aligned && L % 4 == 0) {
+    const int64_t bpr = (L / 4 + 256 * kDqU - 1) / (256 * kDqU);
+    if (bpr > 0 && rows * bpr < 0x7fffffffLL) {
+      dequant_rows_kernel<BITS><<<static_cast<unsigned>(rows * bpr), 256, 0, s>>>(
+          codes, scale, minv, L, W, static_cast<int>(bpr), y);
+      return;
+    }
+  }
   if (rows * wpr < (int64_t{1} << 31))
     dequant_kernel<BITS, uint32_t><<<grid, 256, 0, s>>>(codes, scale, minv, static_cast<uint32_t>(rows),
                                                         L, W, static_cast<uint32_t>(wpr), y, aligned);

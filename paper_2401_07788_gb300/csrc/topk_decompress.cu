@@ -93,14 +93,15 @@ __global__ void __launch_bounds__(kDecThreads)
 // (rpc rows, rpc * row_len <= kRowsPerCta) or the column range
 // [part * width, part * width + width) of one row (ppr parts per row).  It
 // zero-fills its region, then stores the kept values that fall in it; a part
-// reads its row's whole payload (from L2 after the first part) and keeps its own.
+// reads its row's whole payload (from L2 after the first part) and keeps its
+// own, with 16-byte loads several deep so the payload costs few round trips.
 constexpr int64_t kRowsPerCta = 16384;
 constexpr int64_t kPartWidth = 8192;
 
 __global__ void __launch_bounds__(kDecThreads)
     topk_decompress_rows_kernel(const float* __restrict__ vals, const int32_t* __restrict__ idx,
                                 int64_t rows, int64_t L, int64_t k, float* __restrict__ y,
-                                int64_t rpc, int64_t ppr, int aligned) {
+                                int64_t rpc, int64_t ppr, int aligned, int vec) {
   const int tid = threadIdx.x;
   int64_t r0, nrows, c0, ncols;
   if (ppr == 1) {
@@ -139,10 +140,50 @@ __global__ void __launch_bounds__(kDecThreads)
   const int64_t e_begin = r0 * k;
   const uint32_t nk = static_cast<uint32_t>(nrows * k);  // <= 65536
   const uint32_t k32 = static_cast<uint32_t>(k);
-  for (uint32_t e = tid; e < nk; e += kDecThreads) {
-    const uint32_t lr = (ppr == 1) ? e / k32 : 0u;
-    const int64_t col = static_cast<int64_t>(idx[e_begin + e]) - c0;
-    if (col >= 0 && col < ncols) dst[static_cast<int64_t>(lr) * L + col] = vals[e_begin + e];
+  const float* vr = vals + e_begin;
+  const int32_t* ir = idx + e_begin;
+  if (vec) {
+    // 4 entries per 16-byte load, kU loads in flight per thread
+    constexpr int kU = 4;
+    const uint32_t n4 = nk / 4;
+    for (uint32_t b = tid; b < n4; b += kDecThreads * kU) {
+      int4 iv[kU];
+      float4 fv[kU];
+#pragma unroll
+      for (int u = 0; u < kU; ++u) {
+        const uint32_t q = b + u * kDecThreads;
+        if (q < n4) {
+          iv[u] = reinterpret_cast<const int4*>(ir)[q];
+          fv[u] = reinterpret_cast<const float4*>(vr)[q];
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < kU; ++u) {
+        const uint32_t q = b + u * kDecThreads;
+        if (q < n4) {
+          const int ci[4] = {iv[u].x, iv[u].y, iv[u].z, iv[u].w};
+          const float cv[4] = {fv[u].x, fv[u].y, fv[u].z, fv[u].w};
+#pragma unroll
+          for (int t = 0; t < 4; ++t) {
+            const uint32_t e = 4 * q + t;
+            const uint32_t lr = (ppr == 1) ? e / k32 : 0u;
+            const int64_t col = static_cast<int64_t>(ci[t]) - c0;
+            if (col >= 0 && col < ncols) dst[static_cast<int64_t>(lr) * L + col] = cv[t];
+          }
+        }
+      }
+    }
+    for (uint32_t e = 4 * n4 + tid; e < nk; e += kDecThreads) {
+      const uint32_t lr = (ppr == 1) ? e / k32 : 0u;
+      const int64_t col = static_cast<int64_t>(ir[e]) - c0;
+      if (col >= 0 && col < ncols) dst[static_cast<int64_t>(lr) * L + col] = vr[e];
+    }
+  } else {
+    for (uint32_t e = tid; e < nk; e += kDecThreads) {
+      const uint32_t lr = (ppr == 1) ? e / k32 : 0u;
+      const int64_t col = static_cast<int64_t>(ir[e]) - c0;
+      if (col >= 0 && col < ncols) dst[static_cast<int64_t>(lr) * L + col] = vr[e];
+    }
   }
 }
 
@@ -184,8 +225,11 @@ cudaError_t launch_topk_decompress(const float* vals, const int32_t* idx, int64_
       blocks = rows * ppr;
     }
     if (blocks > 0x7fffffffLL) return cudaErrorInvalidValue;
+    // 16-byte payload loads when every block's payload range is 16-byte aligned
+    const int vec = (k % 4 == 0) && (reinterpret_cast<uintptr_t>(vals) % 16 == 0) &&
+                    (reinterpret_cast<uintptr_t>(idx) % 16 == 0);
     topk_decompress_rows_kernel<<<static_cast<unsigned>(blocks), kDecThreads, 0, s>>>(
-        vals, idx, rows, L, k, y, rpc, ppr, aligned);
+        vals, idx, rows, L, k, y, rpc, ppr, aligned, vec);
     return cudaGetLastError();
   }
   int64_t rpc = 1, tpr = 1, blocks;

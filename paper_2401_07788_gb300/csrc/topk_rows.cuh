@@ -148,6 +148,16 @@ __device__ __forceinline__ uint32_t block_excl_scan(uint32_t v, uint32_t* red, i
 // ---------------------------------------------------------------------------
 // CTA / cluster kernel
 // ---------------------------------------------------------------------------
+// The first pick of the CTA kernel: bin B, the entries above it and in it
+// (whole row), its first and last keys, this CTA's entries in it and those of
+// the CTAs before it.
+struct PickOut {
+  int B;
+  uint32_t above, m;
+  int kl, kh;
+  uint32_t own, off;
+};
+
 template <int NT, int SCAP>
 struct CtaShared {
   static constexpr int NW = NT / 32;
@@ -175,7 +185,9 @@ struct CtaShared {
   uint32_t lcount;
   uint32_t pick_t, pick_excl;
   int pub_lo, pub_hi;
+  uint32_t before_gt, before_eq;
   BinPick pick;
+  PickOut pk;
   Threshold thr;
   uint64_t bars[8];  // one per slice chunk (one float4 slot of every thread)
 };
@@ -403,8 +415,10 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
         keys4<FULL>(v, 4 * q, n, kk);
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
-          if (kk[i] == 0) ++zc;
-          else if (kk[i] > 0) atomicAdd(&sh.u.hist[lin_bin(kk[i], scale)], 1u);
+          // zeros (common after ReLU) are counted per warp, not by atomics
+          zc += kk[i] == 0;
+          const int b = lin_bin(kk[i], scale);
+          if (kk[i] > 0) atomicAdd(&sh.u.hist[b], 1u);
         }
       }
     }
@@ -424,6 +438,7 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
   uint32_t need = 0;
   bool counted = false;  // per-chunk counts of kept entries are in place (fast path)
   uint32_t own = 0, off = 0;  // this CTA's candidates and those of the CTAs before it
+  uint32_t gt_before = 0, eq_before = 0;  // kept / tied entries of the earlier CTAs
   if (k < L) {
     uint32_t kr = static_cast<uint32_t>(k);
     int B = 0;
@@ -483,57 +498,57 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
           else wbase += u;
         }
       }
-      // every warp ranks that warp's groups and bins itself
-      uint32_t c2[G];
       if (warp == ws) {
+        // that warp finds the bin, this CTA's entries in it and those of the
+        // CTAs before it, and the bin's first and last keys
+        const uint32_t ex = wbase + incl - total;
+        const unsigned who = __ballot_sync(kFull, ex < kr && kr <= ex + total);
+        const int src = who ? __ffs(who) - 1 : 31;
+        const int gb0 = kNB - G * (tid + 1);
+        int pb = gb0;
+        uint32_t pab = ex, pc = cnt[0];
+        {
+          uint32_t run = ex;
+          bool done = false;
 #pragma unroll
-        for (int b = 0; b < G; ++b) c2[b] = cnt[b];
-      } else {
-        group_bins(ws * 32 + lane, c2);
-      }
-      uint32_t t2 = 0;
-#pragma unroll
-      for (int b = 0; b < G; ++b) t2 += c2[b];
-      const uint32_t ex2 = wbase + warp_inclusive_scan(t2, lane) - t2;
-      const unsigned who = __ballot_sync(kFull, ex2 < kr && kr <= ex2 + t2);
-      const int src = who ? __ffs(who) - 1 : 31;
-      const int gb0 = kNB - G * (ws * 32 + lane + 1);
-      int pb = gb0;
-      uint32_t pab = ex2, pc = c2[0];
-      {
-        uint32_t run = ex2;
-        bool done = false;
-#pragma unroll
-        for (int b = G - 1; b >= 0; --b) {
-          if (!done && run + c2[b] >= kr) {
-            pb = gb0 + b;
-            pab = run;
-            pc = c2[b];
-            done = true;
+          for (int b = G - 1; b >= 0; --b) {
+            if (!done && run + cnt[b] >= kr) {
+              pb = gb0 + b;
+              pab = run;
+              pc = cnt[b];
+              done = true;
+            }
+            if (!done) run += cnt[b];
           }
-          if (!done) run += c2[b];
         }
-      }
-      B = __shfl_sync(kFull, pb, src);
-      kr -= __shfl_sync(kFull, pab, src);
-      m = __shfl_sync(kFull, pc, src);
-      {
-        // this CTA's entries in bin B and those of the CTAs before it
-        const int gB = (kNB - 1 - B) / G;
-        const int ib = B - (kNB - G * (gB + 1));
-        for (uint32_t r = 0; r <= crank; ++r) {
-          const uint32_t wv = table[(r * NT + gB) * GW + ib / 2];
-          const uint32_t cr = (ib & 1) ? (wv >> 16) : (wv & 0xffffu);
-          if (r < crank) off += cr;
-          else own = cr;
+        const int Bw = __shfl_sync(kFull, pb, src);
+        const uint32_t above = __shfl_sync(kFull, pab, src);
+        const uint32_t mw = __shfl_sync(kFull, pc, src);
+        const int gB = (kNB - 1 - Bw) / G;
+        const int ib = Bw - (kNB - G * (gB + 1));
+        uint32_t cr = 0;
+        if (lane < static_cast<int>(C)) {
+          const uint32_t wv = table[(lane * NT + gB) * GW + ib / 2];
+          cr = (ib & 1) ? (wv >> 16) : (wv & 0xffffu);
         }
+        const uint32_t offw = __reduce_add_sync(kFull, lane < static_cast<int>(crank) ? cr : 0u);
+        const uint32_t ownw = __shfl_sync(kFull, cr, crank);
+        // lanes 0 and 1 find the first keys of bins B and B + 1 side by side
+        const int bb = Bw + (lane & 1);
+        const float inv = fmul(__int_as_float(smax), 1.0f / kNB);
+        const int fk = (bb >= 1 && bb < kNB) ? bin_first_key(bb, scale, inv) : 0;
+        const int klw = (Bw == 0) ? 0 : __shfl_sync(kFull, fk, 0);
+        const int khw = (Bw == kNB - 1) ? 0x7fffffff : __shfl_sync(kFull, fk, 1) - 1;
+        if (lane == 0) sh.pk = PickOut{Bw, above, mw, klw, khw, ownw, offw};
       }
-      // lanes 0 and 1 find the first keys of bins B and B + 1 side by side
-      const int bb = B + (lane & 1);
-      const float inv = fmul(__int_as_float(smax), 1.0f / kNB);
-      const int fk = (bb >= 1 && bb < kNB) ? bin_first_key(bb, scale, inv) : 0;
-      kl = (B == 0) ? 0 : __shfl_sync(kFull, fk, 0);
-      kh = (B == kNB - 1) ? 0x7fffffff : __shfl_sync(kFull, fk, 1) - 1;
+      __syncthreads();
+      B = sh.pk.B;
+      kr -= sh.pk.above;
+      m = sh.pk.m;
+      kl = sh.pk.kl;
+      kh = sh.pk.kh;
+      own = sh.pk.own;
+      off = sh.pk.off;
     }
 
     if (scale > 0.0f && m <= static_cast<uint32_t>(kLCAP)) {
@@ -548,26 +563,38 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
           const int q = j * NT + tid;
           int kk[4];
           keys4<FULL>(s4[q], 4 * q, nv, kk);
+          bool inb[4];
+          bool anyb = false;
 #pragma unroll
           for (int i = 0; i < 4; ++i) {
             ab += kk[i] > kh;
-            if (kk[i] >= kl && kk[i] <= kh) {
-              const uint32_t at = atomicAdd(&sh.lcount, 1u);
-              if (at < own) {
-                sh.u.c.lch[at] = static_cast<uint16_t>(j * NW + warp);
-                int* slot = &sh.u.c.cand[off + at];
-                if (C > 1) {
-                  for (uint32_t r = 0; r < C; ++r)
-                    dsmem_st_u32(dsmem_addr(slot, r), static_cast<uint32_t>(kk[i]));
-                } else {
-                  *slot = kk[i];
+            inb[i] = static_cast<uint32_t>(kk[i] - kl) <= static_cast<uint32_t>(kh - kl);
+            anyb |= inb[i];
+          }
+          if (__any_sync(kFull, anyb)) {
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              if (inb[i]) {
+                const uint32_t at = atomicAdd(&sh.lcount, 1u);
+                if (at < own) {
+                  sh.u.c.lch[at] = static_cast<uint16_t>(j * NW + warp);
+                  int* slot = &sh.u.c.cand[off + at];
+                  if (C > 1) {
+                    for (uint32_t r = 0; r < C; ++r)
+                      dsmem_st_u32(dsmem_addr(slot, r), static_cast<uint32_t>(kk[i]));
+                  } else {
+                    *slot = kk[i];
+                  }
                 }
               }
             }
           }
           ab = __reduce_add_sync(kFull, ab);
         }
-        if (lane == 0) sh.cgt[j * NW + warp] = ab;
+        if (lane == 0) {
+          sh.cgt[j * NW + warp] = ab;
+          sh.ceq[j * NW + warp] = 0;
+        }
         wab += ab;
       }
       if (lane == 0) {
@@ -579,7 +606,6 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
         }
       }
       row_sync(C);  // the last cluster barrier: nothing is read remotely after it
-      if (warp == 0) scan_chunks1<NCH>(sh.cgt, lane);
       // P threads rank each candidate against the whole list (P a power of two,
       // m x P <= NT); the group holding T reports it (all such groups report
       // the same values)
@@ -610,6 +636,36 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
       T = sh.thr.T;
       need = sh.thr.need;
       own = min(own, sh.lcount);
+      // this CTA's candidates above T, or equal to it, join their chunks' counts
+      for (uint32_t p = tid; p < own; p += NT) {
+        const int key = sh.u.c.cand[off + p];
+        const int ch = sh.u.c.lch[p];
+        if (key > T) atomicAdd(&sh.cgt[ch], 1u);
+        else if (key == T) atomicAdd(&sh.ceq[ch], 1u);
+      }
+      __syncthreads();
+      if (warp == 0) {
+        scan_chunks1<NCH>(sh.cgt, lane);
+        if (need) scan_chunks1<NCH>(sh.ceq, lane);
+        // the earlier CTAs' kept entries (above bin B, and candidates above T)
+        // and their ties
+        uint32_t gb = 0, eb = 0;
+        for (uint32_t p = lane; p < off; p += 32) {
+          const int key = sh.u.c.cand[p];
+          gb += key > T;
+          eb += key == T;
+        }
+        for (uint32_t i = lane; i < crank * NW; i += 32) gb += sh.wtot[i / NW][i % NW];
+        gb = __reduce_add_sync(kFull, gb);
+        eb = __reduce_add_sync(kFull, eb);
+        if (lane == 0) {
+          sh.before_gt = gb;
+          sh.before_eq = eb;
+        }
+      }
+      __syncthreads();
+      gt_before = sh.before_gt;
+      eq_before = sh.before_eq;
       counted = true;
     } else {
       // ---- too many candidates for the table: integer rounds over the slice --
@@ -682,7 +738,6 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
     }
   }
 
-  uint32_t gt_before = 0, eq_before = 0;  // kept / tied entries of the earlier CTAs
   if (!counted) {
     // ---- count kept entries per 128-entry chunk ------------------------------
 #pragma unroll 2
@@ -724,46 +779,6 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
     }
   }
 
-  if (counted) {
-    // The chunk counts hold the entries above bin B before each chunk.  Each
-    // warp adds, for its own chunks ch_j = j * NW + warp, this CTA's
-    // candidates above T in earlier chunks, and sets the ties (== T) there.
-    uint32_t cg[QPT], ce[QPT];
-#pragma unroll
-    for (int j = 0; j < QPT; ++j) cg[j] = ce[j] = 0;
-    for (uint32_t p = lane; p < own; p += 32) {
-      const int key = sh.u.c.cand[off + p];
-      const int ch = sh.u.c.lch[p];
-      const uint32_t g = key > T, e = key == T;
-#pragma unroll
-      for (int j = 0; j < QPT; ++j) {
-        const bool before = ch < j * NW + warp;
-        cg[j] += before ? g : 0u;
-        ce[j] += before ? e : 0u;
-      }
-    }
-#pragma unroll
-    for (int j = 0; j < QPT; ++j) {
-      const uint32_t g = __reduce_add_sync(kFull, cg[j]);
-      const uint32_t e = need ? __reduce_add_sync(kFull, ce[j]) : 0u;
-      if (lane == 0) {
-        sh.cgt[j * NW + warp] += g;
-        sh.ceq[j * NW + warp] = e;
-      }
-    }
-    // the earlier CTAs' kept entries and ties
-    uint32_t gb = 0, eb = 0;
-    for (uint32_t p = lane; p < off; p += 32) {
-      const int key = sh.u.c.cand[p];
-      gb += key > T;
-      eb += key == T;
-    }
-    for (uint32_t i = lane; i < crank * NW; i += 32) gb += sh.wtot[i / NW][i % NW];
-    gt_before = __reduce_add_sync(kFull, gb);
-    eq_before = need ? __reduce_add_sync(kFull, eb) : 0u;
-    __syncwarp();
-  }
-
   // ---- write the payload (ascending column) and the buffers -----------------
   float* vrow = a.vals + row * k;
   int32_t* irow = a.idx + row * k;
@@ -799,20 +814,23 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
     if (!FULL && e0 >= nv) continue;
     const float val[4] = {v4.x, v4.y, v4.z, v4.w};
     const int col = static_cast<int>(c0) + e0;
+    uint32_t pi[4];
+    pi[0] = pos;
+#pragma unroll
+    for (int i = 1; i < 4; ++i) pi[i] = pi[i - 1] + (kp[i - 1] ? 1u : 0u);
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-      if (kp[i]) {
-        if (pos < kk32) {
-          vrow[pos] = val[i];
-          irow[pos] = col + i;
-        }
-        if (MODE == kDelta) {
+      if (kp[i] && pi[i] < kk32) vrow[pi[i]] = val[i];
+      if (kp[i] && pi[i] < kk32) irow[pi[i]] = col + i;
+    }
+    if (MODE == kDelta) {
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+        if (kp[i]) {
           // state + d, against the same state value d was formed from
           float* sp = arow + col + i;
           *sp = fadd(*sp, val[i]);
         }
-        ++pos;
-      }
     }
     if (MODE == kEF) {
       const float ne[4] = {kp[0] ? 0.0f : val[0], kp[1] ? 0.0f : val[1], kp[2] ? 0.0f : val[2],
