@@ -278,6 +278,8 @@ def algorithmic_bytes(R_, L_, k=None, bits=None, op=""):
         return 8 * k * R_ + 4 * N
     if op == "delta_topk":  # EF21 / AQ-SGD: state written only where kept
         return 8 * N + 12 * k * R_
+    if op == "topk_gather":  # indices read, values gathered, payload written
+        return 12 * k * R_
     if op == "aqsgd_decompress":
         return 8 * k * R_ + 8 * k * R_
     if op in ("quant", "dequant"):
@@ -609,6 +611,15 @@ def measure_operators(mpc, synth, device, stream, peak):
         algorithmic_bytes(32, 16384, k=k, op="topk"))
     rec("topk_decompress 32x16384 K=10%", time_op(lambda: mpc.mpc_topk_decompress(v, i, 16384, y=y), stream, flush),
         algorithmic_bytes(32, 16384, k=k, op="topk_decompress"))
+    # index reuse at the CNN stage boundary: gradient values at the activation's Top10%
+    xg = synth.relu_normal((R, L), 3, device)
+    gg = synth.normal((R, L), 4, device, std=1e-3)
+    kg = synth.k_of(L, 10)
+    _, ig = mpc.mpc_topk_compress(xg, kg)
+    vg = mpc.mpc_topk_gather(gg, ig)
+    rec("topk_gather %dx%d K=10%%" % (R, L), time_op(lambda: mpc.mpc_topk_gather(gg, ig, vals=vg), stream, flush),
+        algorithmic_bytes(R, L, k=kg, op="topk_gather"))
+    del xg, gg
     # LM boundary: EF21 Top10% per token, 4-bit
     xl = synth.lm_hidden(0, device)
     gl = torch.zeros_like(xl)
@@ -648,6 +659,10 @@ def measure_operators(mpc, synth, device, stream, peak):
             rec("topk_compress 2^28 L=%d K=%d%%" % (Ls, pct), time_op(lambda: mpc.mpc_topk_compress(xv, ks, vs, is_), stream, flush, 3),
                 algorithmic_bytes(Rs, Ls, k=ks, op="topk"))
             if pct == 10:
+                gvs = mpc.mpc_topk_gather(xv, is_)
+                rec("topk_gather 2^28 L=%d K=10%%" % Ls, time_op(lambda: mpc.mpc_topk_gather(xv, is_, vals=gvs), stream, flush, 3),
+                    algorithmic_bytes(Rs, Ls, k=ks, op="topk_gather"))
+                del gvs
                 ys = torch.empty_like(xv)
                 rec("topk_decompress 2^28 L=%d K=10%%" % Ls, time_op(lambda: mpc.mpc_topk_decompress(vs, is_, Ls, y=ys), stream, flush, 3),
                     algorithmic_bytes(Rs, Ls, k=ks, op="topk_decompress"))

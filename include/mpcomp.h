@@ -97,6 +97,18 @@ mpc_status mpc_topk_decompress(const float* vals, const int32_t* idx, int64_t ro
                                int64_t row_len, int64_t k, float* y,
                                mpc_stream_t stream);
 
+/* TopK index reuse (§3.2, Table 5: the gradient at a boundary is compressed
+ * at the TopK indices of the activation, which fine-tuning needs to converge):
+ *   vals[r][i] = g[r][idx[r][i]]  (bit copy), for 0 <= i < k.
+ *   g     [rows][row_len] fp32, read only (device memory).
+ *   idx   [rows][k] int32, read only: the payload indices of a compress call
+ *         on the tensor g pairs with (any order is accepted).
+ *   vals  [rows][k] fp32, out; decompress with mpc_topk_decompress(vals, idx).
+ * An index outside [0, row_len) reads nothing: its value is +0 and
+ * mpc_get_status then reports MPC_ERR_DEVICE.  Requires 1 <= k <= row_len. */
+mpc_status mpc_topk_gather(const float* g, int64_t rows, int64_t row_len, const int32_t* idx,
+                           int64_t k, float* vals, mpc_stream_t stream);
+
 /* Error feedback of Seide et al. fused with TopK (§2.4: the message is
  * C(X + e) and the error kept is e = X - C(X), one global buffer per
  * operator carried across batches):

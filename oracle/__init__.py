@@ -64,6 +64,7 @@ def load(path: str | None = None) -> ctypes.CDLL:
         lib.orc_uniform.restype = ctypes.c_float
         lib.orc_topk_compress.argtypes = [_F32P, _i64, _i64, _i64, _F32P, _I32P]
         lib.orc_topk_decompress.argtypes = [_F32P, _I32P, _i64, _i64, _i64, _F32P]
+        lib.orc_topk_gather.argtypes = [_F32P, _i64, _i64, _I32P, _i64, _F32P]
         lib.orc_ef_topk_compress.argtypes = [_F32P, _F32P, _i64, _i64, _i64, _F32P, _I32P]
         lib.orc_ef21_topk_compress.argtypes = [_F32P, _F32P, _i64, _i64, _i64, _F32P, _I32P]
         lib.orc_aqsgd_compress.argtypes = [_F32P, _F32P, _i64, _I64P, _i64, _i64, _i64, _i64,
@@ -76,7 +77,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
                                            ctypes.c_uint64, _U32P, _F32P, _F32P]
         lib.orc_quant_decompress.argtypes = [_U32P, _F32P, _F32P, _i64, _i64, ctypes.c_int,
                                              _F32P]
-        for name in ("orc_topk_compress", "orc_topk_decompress", "orc_ef_topk_compress",
+        for name in ("orc_topk_compress", "orc_topk_decompress", "orc_topk_gather",
+                     "orc_ef_topk_compress",
                      "orc_ef21_topk_compress", "orc_aqsgd_compress", "orc_aqsgd_decompress",
                      "orc_quant_compress", "orc_quant_decompress"):
             getattr(lib, name).restype = None
@@ -124,6 +126,18 @@ def topk_decompress(vals, idx, row_len: int, lib=None):
     y = np.empty((R, row_len), np.float32)
     (lib or load()).orc_topk_decompress(vals, idx, R, row_len, k, y)
     return y
+
+
+def topk_gather(g, idx, lib=None):
+    """TopK index reuse (§3.2, Table 5): the values of g at the kept indices idx [R, k]."""
+    g = _f32(g)
+    idx = np.ascontiguousarray(idx, dtype=np.int32)
+    R, L = _rows_cols(g)
+    k = idx.shape[-1]
+    assert idx.size == R * k and (idx.size == 0 or (idx.min() >= 0 and idx.max() < L))
+    vals = np.empty((R, k), np.float32)
+    (lib or load()).orc_topk_gather(g, R, L, idx, k, vals)
+    return vals
 
 
 def ef_topk_compress(x, e, k: int, lib=None):

@@ -120,6 +120,17 @@ void orc_topk_decompress(const float* vals, const int32_t* idx, int64_t rows,
     }
 }
 
+/* TopK index reuse, §3.2 (Table 5): the gradient at a boundary is compressed
+ * at the indices kept for the activation in the forward pass, so the payload
+ * is the gradient's values at those indices, in the same order. */
+void orc_topk_gather(const float* g, int64_t rows, int64_t row_len, const int32_t* idx,
+                     int64_t k, float* vals)
+{
+    for (int64_t r = 0; r < rows; ++r)
+        for (int64_t i = 0; i < k; ++i)
+            vals[r * k + i] = g[r * row_len + idx[r * k + i]];
+}
+
 /* ------------------------------------------------------------------------- */
 /* Error feedback (Seide et al.), §2.4                                        */
 /* ------------------------------------------------------------------------- */

@@ -42,6 +42,10 @@ void orc_topk_compress(const float* x, int64_t rows, int64_t row_len, int64_t k,
 void orc_topk_decompress(const float* vals, const int32_t* idx, int64_t rows,
                          int64_t row_len, int64_t k, float* y);
 
+/* TopK index reuse, §3.2 (Table 5): vals[r][i] = g[r][idx[r][i]]. */
+void orc_topk_gather(const float* g, int64_t rows, int64_t row_len, const int32_t* idx,
+                     int64_t k, float* vals);
+
 /* Error feedback (Seide), §2.4: s = x + e, send C(s), e <- s - C(s). */
 void orc_ef_topk_compress(const float* x, float* e, int64_t rows, int64_t row_len,
                           int64_t k, float* vals, int32_t* idx);

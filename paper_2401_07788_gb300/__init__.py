@@ -21,6 +21,7 @@ from ._build import LIB_PATH
 
 __all__ = [
     "MpcError", "lib", "mpc_topk_workspace_bytes", "mpc_topk_compress", "mpc_topk_decompress",
+    "mpc_topk_gather",
     "mpc_ef_topk_compress", "mpc_ef21_topk_compress", "mpc_aqsgd_compress",
     "mpc_aqsgd_decompress", "mpc_quant_codes_words", "mpc_quant_workspace_bytes",
     "mpc_quant_compress", "mpc_quant_decompress", "mpc_get_status", "mpc_last_error",
@@ -44,6 +45,7 @@ _SIGNATURES = {
     "mpc_topk_workspace_bytes": ([_I64, _I64, _I64], _SZ),
     "mpc_topk_compress": ([_VP, _I64, _I64, _I64, _VP, _VP, _VP, _SZ, _VP], _INT),
     "mpc_topk_decompress": ([_VP, _VP, _I64, _I64, _I64, _VP, _VP], _INT),
+    "mpc_topk_gather": ([_VP, _I64, _I64, _VP, _I64, _VP, _VP], _INT),
     "mpc_ef_topk_compress": ([_VP, _VP, _I64, _I64, _I64, _VP, _VP, _VP, _SZ, _VP], _INT),
     "mpc_ef21_topk_compress": ([_VP, _VP, _I64, _I64, _I64, _VP, _VP, _VP, _SZ, _VP], _INT),
     "mpc_aqsgd_compress": ([_VP, _VP, _I64, _VP, _I64, _I64, _I64, _I64, _VP, _VP, _VP, _SZ,
@@ -198,6 +200,21 @@ def mpc_topk_decompress(vals, idx, row_len: int, y=None, stream=None):
     _check(lib().mpc_topk_decompress(_ptr(vals), _ptr(idx), R, row_len, k, _ptr(y),
                                      _stream(stream)))
     return y
+
+
+def mpc_topk_gather(g, idx, vals=None, stream=None):
+    """TopK index reuse (§3.2): the values of g [R, L] at the payload indices idx [R, k]."""
+    _cuda(g, torch.float32, "g")
+    _cuda(idx, torch.int32, "idx")
+    R, L = _rows_cols(g)
+    Ri, k = _rows_cols(idx)
+    if Ri != R:
+        raise MpcError(1, "idx must have one row per row of g")
+    if vals is None:
+        vals = torch.empty((R, k), dtype=torch.float32, device=g.device)
+    _cuda(vals, torch.float32, "vals")
+    _check(lib().mpc_topk_gather(_ptr(g), R, L, _ptr(idx), k, _ptr(vals), _stream(stream)))
+    return vals
 
 
 # ---------------------------------------------------------------------------------------

@@ -204,6 +204,21 @@ mpc_status mpc_topk_decompress(const float* vals, const int32_t* idx, int64_t ro
   return ok();
 }
 
+mpc_status mpc_topk_gather(const float* g, int64_t rows, int64_t row_len, const int32_t* idx,
+                           int64_t k, float* vals, mpc_stream_t stream) {
+  MPC_TRY(check_shape(rows, row_len, k));
+  if (rows == 0) return ok();
+  MPC_TRY(check_ptr(g, 4, "g"));
+  MPC_TRY(check_ptr(idx, 4, "idx"));
+  MPC_TRY(check_ptr(vals, 4, "vals"));
+  Device d;
+  MPC_TRY(current_device(&d));
+  cudaError_t e = mpc::launch_topk_gather(g, idx, rows, row_len, k, vals, d.status,
+                                          reinterpret_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_error(e, "topk_gather launch");
+  return ok();
+}
+
 mpc_status mpc_aqsgd_compress(const float* x, float* buf, int64_t num_samples,
                               const int64_t* sample_ids, int64_t n_ids, int64_t rows_per_sample,
                               int64_t row_len, int64_t k, float* vals, int32_t* idx, void* ws,

@@ -17,6 +17,7 @@ namespace mpc {
 enum : unsigned {
   STATUS_TIMEOUT = 1u,     // a bounded wait on an mbarrier gave up
   STATUS_BAD_SAMPLE = 2u,  // an AQ-SGD sample id was out of range
+  STATUS_BAD_INDEX = 4u,   // a payload index was out of range
 };
 // Kernels receive the address of the library's status word (one per device)
 // and OR their error bits into it.

@@ -58,6 +58,8 @@ cudaError_t launch_topk_grid(int mode, const TopkGridArgs& a, int num_sms, cudaS
 cudaError_t launch_topk_decompress(const float* vals, const int32_t* idx, int64_t rows,
                                    int64_t L, int64_t k, float* y, int aligned, int num_sms,
                                    cudaStream_t s);
+cudaError_t launch_topk_gather(const float* g, const int32_t* idx, int64_t rows, int64_t L,
+                              int64_t k, float* vals, unsigned* status, cudaStream_t s);
 cudaError_t launch_aqsgd_decompress(const float* vals, const int32_t* idx, float* buf,
                                     int64_t num_samples, const int64_t* ids, int64_t n_ids,
                                     int64_t rps, int64_t L, int64_t k, unsigned* status,

@@ -8,6 +8,9 @@
 // Longer rows: each output tile is built in shared memory (zero fill, scatter
 // of the tile's kept entries, found by a block-parallel search of the row's
 // ascending indices) and written once.
+//
+// Also here: the gather of TopK index reuse (§3.2), the payload of a second
+// tensor at the indices kept for the first.
 #include "common.cuh"
 #include "kernels.h"
 #include "launch_util.h"
@@ -187,6 +190,62 @@ __global__ void __launch_bounds__(kDecThreads)
   }
 }
 
+// TopK index reuse (§3.2, Table 5): vals[r][i] = g[r][idx[r][i]].  A block
+// covers kGU x 4 x 256 consecutive payload entries of one row (bpr blocks per
+// row): 16-byte index loads and value stores when every row's payload starts
+// 16-byte aligned, the gathered values fetched by independent 4-byte loads
+// (ascending within a row, so neighbouring lanes mostly share sectors).  An
+// index outside [0, L) reads nothing: its value is +0 and STATUS_BAD_INDEX is
+// recorded.
+constexpr int kGU = 4;
+
+__global__ void __launch_bounds__(kDecThreads)
+    topk_gather_kernel(const float* __restrict__ g, const int32_t* __restrict__ idx,
+                       int64_t L, int64_t k, int bpr, float* __restrict__ vals, int vec,
+                       unsigned* status) {
+  const int64_t row = blockIdx.x / bpr;
+  const int64_t q0 = static_cast<int64_t>(blockIdx.x % bpr) * (kDecThreads * kGU);
+  const float* gr = g + row * L;
+  const int32_t* ir = idx + row * k;
+  float* vr = vals + row * k;
+  bool bad = false;
+  if (vec) {
+    const int64_t n4 = k / 4;
+    int4 iv[kGU];
+#pragma unroll
+    for (int u = 0; u < kGU; ++u) {
+      const int64_t q = q0 + u * kDecThreads + threadIdx.x;
+      iv[u] = (q < n4) ? reinterpret_cast<const int4*>(ir)[q] : make_int4(0, 0, 0, 0);
+    }
+#pragma unroll
+    for (int u = 0; u < kGU; ++u) {
+      const int64_t q = q0 + u * kDecThreads + threadIdx.x;
+      if (q < n4) {
+        const int c[4] = {iv[u].x, iv[u].y, iv[u].z, iv[u].w};
+        float o[4];
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+          const bool ok = c[t] >= 0 && c[t] < L;
+          o[t] = ok ? gr[c[t]] : 0.0f;
+          bad |= !ok;
+        }
+        reinterpret_cast<float4*>(vr)[q] = make_float4(o[0], o[1], o[2], o[3]);
+      }
+    }
+  } else {
+    for (int u = 0; u < 4 * kGU; ++u) {
+      const int64_t i = 4 * q0 + u * kDecThreads + threadIdx.x;
+      if (i < k) {
+        const int c = ir[i];
+        const bool ok = c >= 0 && c < L;
+        vr[i] = ok ? gr[c] : 0.0f;
+        bad |= !ok;
+      }
+    }
+  }
+  if (bad) set_status(status, STATUS_BAD_INDEX);
+}
+
 // One CTA per logical payload row: buf_recv[s][r][idx] += vals.
 __global__ void __launch_bounds__(kDecThreads)
     aqsgd_decompress_kernel(const float* __restrict__ vals, const int32_t* __restrict__ idx,
@@ -247,6 +306,19 @@ cudaError_t launch_topk_decompress(const float* vals, const int32_t* idx, int64_
   if (err != cudaSuccess) return err;
   topk_decompress_kernel<<<static_cast<unsigned>(blocks), kDecThreads, smem, s>>>(
       vals, idx, rows, L, k, y, rpc, tpr, aligned);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_topk_gather(const float* g, const int32_t* idx, int64_t rows, int64_t L,
+                              int64_t k, float* vals, unsigned* status, cudaStream_t s) {
+  if (rows <= 0 || k <= 0) return cudaSuccess;
+  const int vec = (k % 4 == 0) && (reinterpret_cast<uintptr_t>(idx) % 16 == 0) &&
+                  (reinterpret_cast<uintptr_t>(vals) % 16 == 0);
+  const int64_t per_block = static_cast<int64_t>(kDecThreads) * kGU * 4;
+  const int64_t bpr = (k + per_block - 1) / per_block;
+  if (rows * bpr > 0x7fffffffLL) return cudaErrorInvalidValue;
+  topk_gather_kernel<<<static_cast<unsigned>(rows * bpr), kDecThreads, 0, s>>>(
+      g, idx, L, k, static_cast<int>(bpr), vals, vec, status);
   return cudaGetLastError();
 }
 

@@ -147,6 +147,24 @@ def pin_topk_decompress(lib, seed: int = 4):
         assert np.all(bits_of(y[r, ~kept]) == 0)  # +0 everywhere else
 
 
+def pin_topk_gather(lib, seed: int = 14):
+    """Index reuse (§3.2, Table 5): numpy's take_along_axis gives the values at the kept
+    indices; at a tensor's own TopK indices the gather is its TopK payload; gathering,
+    scattering back and gathering again changes nothing."""
+    rng = np.random.default_rng(seed)
+    a = rng.standard_normal((6, 257)).astype(np.float32)
+    g = rng.standard_normal((6, 257)).astype(np.float32)
+    g[1, 3] = -0.0
+    for k in (1, 25, 128, 257):
+        _, idx = oracle.topk_compress(a, k, lib)
+        v = oracle.topk_gather(g, idx, lib)
+        assert np.array_equal(bits_of(v), bits_of(np.take_along_axis(g, idx, axis=1)))
+        own_v, own_i = oracle.topk_compress(g, k, lib)
+        assert np.array_equal(bits_of(oracle.topk_gather(g, own_i, lib)), bits_of(own_v))
+        y = oracle.topk_decompress(v, idx, 257, lib)
+        assert np.array_equal(bits_of(oracle.topk_gather(y, idx, lib)), bits_of(v))
+
+
 # --------------------------------------------------------------------------------------
 # Error feedback, §2.4
 # --------------------------------------------------------------------------------------
