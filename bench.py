@@ -633,6 +633,14 @@ def measure_operators(mpc, synth, device, stream, peak):
         algorithmic_bytes(8192, 768, bits=4, op="quant"))
     rec("quant_decompress 8192x768 4-bit", time_op(lambda: mpc.mpc_quant_decompress(cq, sq, mq, 768, 4, y=yl), stream, flush),
         algorithmic_bytes(8192, 768, bits=4, op="dequant"))
+    # fw4-bw6: 6-bit codes of the transformer boundary's gradient (straddling words)
+    g6 = synth.normal((8192, 768), 5, device, std=1e-4)
+    c6, s6, m6 = mpc.mpc_quant_compress(g6, 6)
+    rec("quant_compress 8192x768 6-bit", time_op(lambda: mpc.mpc_quant_compress(g6, 6, codes=c6, scale=s6, minv=m6), stream, flush),
+        algorithmic_bytes(8192, 768, bits=6, op="quant"))
+    rec("quant_decompress 8192x768 6-bit", time_op(lambda: mpc.mpc_quant_decompress(c6, s6, m6, 768, 6, y=yl), stream, flush),
+        algorithmic_bytes(8192, 768, bits=6, op="dequant"))
+    del g6
     del xl, gl, yl
     # AQ-SGD boundary: 8 GiB buffer, 16 ids, Top30%
     S, rps, La = 4096, 512, 1024
@@ -671,10 +679,15 @@ def measure_operators(mpc, synth, device, stream, peak):
                     algorithmic_bytes(Rs, Ls, k=ks, op="ef_topk"))
                 del ys, es
             del vs, is_
-        for b in BITS:
+        for b in BITS + (6,):
             cq, sq, mq = mpc.mpc_quant_compress(xv, b)
             rec("quant_compress 2^28 L=%d %d-bit" % (Ls, b), time_op(lambda: mpc.mpc_quant_compress(xv, b, codes=cq, scale=sq, minv=mq), stream, flush, 3),
                 algorithmic_bytes(Rs, Ls, bits=b, op="quant"))
+            if b == 6:
+                ys = torch.empty_like(xv)
+                rec("quant_decompress 2^28 L=%d 6-bit" % Ls, time_op(lambda: mpc.mpc_quant_decompress(cq, sq, mq, Ls, 6, y=ys), stream, flush, 3),
+                    algorithmic_bytes(Rs, Ls, bits=6, op="dequant"))
+                del ys
             if b == 4:
                 rec("quant_compress 2^28 L=%d 4-bit stochastic" % Ls, time_op(lambda: mpc.mpc_quant_compress(xv, 4, True, 7, codes=cq, scale=sq, minv=mq), stream, flush, 3),
                     algorithmic_bytes(Rs, Ls, bits=4, op="quant"))

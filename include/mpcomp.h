@@ -164,8 +164,9 @@ mpc_status mpc_aqsgd_decompress(const float* vals, const int32_t* idx, float* bu
 /* ------------------------------------------------------------------------ */
 
 /* Total uint32 words of `codes` for this shape: rows * W with
- * W = roundup4(ceil(row_len * bits / 32)).  bits in {2, 4, 8, 32}; 0 for an
- * unsupported width. */
+ * W = roundup4(ceil(row_len * bits / 32)).  bits in 1..16 (§2.2 evaluates 2,
+ * 4, 6 and 8 bits; widths that do not divide 32, such as 6, have codes that
+ * straddle two words) or 32; 0 for an unsupported width. */
 size_t mpc_quant_codes_words(int64_t rows, int64_t row_len, int bits);
 
 /* Bytes of device workspace mpc_quant_compress needs (0 for rows that the

@@ -70,6 +70,9 @@ mpc_status current_device(Device* d) {
 
 bool aligned_to(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
+// Code widths: 1..16 bits (§2.2 evaluates 2, 4, 6 and 8), or 32 (raw fp32 passthrough).
+bool valid_bits(int bits) { return (bits >= 1 && bits <= 16) || bits == 32; }
+
 mpc_status check_ptr(const void* p, uintptr_t align, const char* name) {
   if (p == nullptr) return set_error(MPC_ERR_INVALID_ARG, "%s is NULL", name);
   if (!aligned_to(p, align))
@@ -292,7 +295,7 @@ mpc_status mpc_aqsgd_decompress(const float* vals, const int32_t* idx, float* bu
 
 size_t mpc_quant_codes_words(int64_t rows, int64_t row_len, int bits) {
   if (rows < 0 || row_len < 1) return 0;
-  if (bits != 2 && bits != 4 && bits != 8 && bits != 32) return 0;
+  if (!valid_bits(bits)) return 0;
   const int64_t words = (row_len * bits + 31) / 32;
   return static_cast<size_t>(rows) * static_cast<size_t>((words + 3) / 4 * 4);
 }
@@ -306,8 +309,8 @@ mpc_status mpc_quant_compress(const float* x, int64_t rows, int64_t row_len, int
                               mpc_rounding mode, uint64_t seed, uint32_t* codes, float* scale,
                               float* minv, void* ws, size_t ws_bytes, mpc_stream_t stream) {
   MPC_TRY(check_shape(rows, row_len, 1));
-  if (bits != 2 && bits != 4 && bits != 8 && bits != 32)
-    return set_error(MPC_ERR_INVALID_ARG, "bits=%d not in {2, 4, 8, 32}", bits);
+  if (!valid_bits(bits))
+    return set_error(MPC_ERR_INVALID_ARG, "bits=%d not in 1..16 or 32", bits);
   if (mode != MPC_ROUND_NEAREST && mode != MPC_ROUND_STOCHASTIC)
     return set_error(MPC_ERR_INVALID_ARG, "rounding mode %d", static_cast<int>(mode));
   if (row_len > 0x7fffffffLL / 32) return set_error(MPC_ERR_INVALID_ARG, "row_len too large");
@@ -346,8 +349,8 @@ mpc_status mpc_quant_compress_noalloc(const float* x, int64_t rows, int64_t row_
                                       mpc_rounding mode, uint64_t seed, uint32_t* codes,
                                       float* scale, float* minv, mpc_stream_t stream) {
   MPC_TRY(check_shape(rows, row_len, 1));
-  if (bits != 2 && bits != 4 && bits != 8 && bits != 32)
-    return set_error(MPC_ERR_INVALID_ARG, "bits=%d not in {2, 4, 8, 32}", bits);
+  if (!valid_bits(bits))
+    return set_error(MPC_ERR_INVALID_ARG, "bits=%d not in 1..16 or 32", bits);
   if (mode != MPC_ROUND_NEAREST && mode != MPC_ROUND_STOCHASTIC)
     return set_error(MPC_ERR_INVALID_ARG, "rounding mode %d", static_cast<int>(mode));
   if (row_len > 0x7fffffffLL / 32) return set_error(MPC_ERR_INVALID_ARG, "row_len too large");
@@ -387,8 +390,8 @@ mpc_status mpc_quant_decompress(const uint32_t* codes, const float* scale, const
                                 int64_t rows, int64_t row_len, int bits, float* y,
                                 mpc_stream_t stream) {
   MPC_TRY(check_shape(rows, row_len, 1));
-  if (bits != 2 && bits != 4 && bits != 8 && bits != 32)
-    return set_error(MPC_ERR_INVALID_ARG, "bits=%d not in {2, 4, 8, 32}", bits);
+  if (!valid_bits(bits))
+    return set_error(MPC_ERR_INVALID_ARG, "bits=%d not in 1..16 or 32", bits);
   if (row_len > 0x7fffffffLL / 32) return set_error(MPC_ERR_INVALID_ARG, "row_len too large");
   if (rows == 0) return ok();
   MPC_TRY(check_ptr(codes, 4, "codes"));

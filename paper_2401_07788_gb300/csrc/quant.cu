@@ -132,14 +132,56 @@ __device__ __forceinline__ bool assemble_word(uint32_t& piece, int lane) {
   return (lane & 3) == 0;
 }
 
+// Any width b in [1, 16] (BITS == 0 instantiations; b known at run time): the
+// codes of entries e0..e0+3 as one 4b-bit piece.
+__device__ __forceinline__ uint64_t codes4_any(const float xs[4], int64_t e0, int64_t n,
+                                               const RowParams& p, bool stochastic,
+                                               uint64_t seed, uint64_t flat0, int bits) {
+  uint64_t packed = 0;
+  if (p.degenerate) return 0;
+  float u[4] = {0.f, 0.f, 0.f, 0.f};
+  if (stochastic) uniform4(seed, flat0, u);
+#pragma unroll
+  for (int t = 0; t < 4; ++t)
+    if (e0 + t < n)
+      packed |= static_cast<uint64_t>(code_of(xs[t], p, stochastic, u[t])) << (bits * t);
+  return packed;
+}
+
+// One warp stores 128 consecutive codes of width b, its lanes' 4b-bit pieces in
+// lane order, as the 4b words that start at word `base` of the row (a code may
+// straddle two words).  The pieces meet by atomicOr in `buf`, 64 words of this
+// warp's shared memory; words at or past data_words are not written.
+__device__ __forceinline__ void store_codes_any(uint64_t piece, int bits, int lane, uint32_t* buf,
+                                                uint32_t* cr, int64_t base, int64_t data_words) {
+  const int nw = 4 * bits;
+  buf[lane] = 0u;
+  buf[lane + 32] = 0u;
+  __syncwarp();
+  const int o = nw * lane;  // bit offset of this lane's piece in the 128 codes
+  const int w = o >> 5, sh = o & 31;
+  const uint32_t v0 = static_cast<uint32_t>(piece << sh);
+  const uint32_t v1 = static_cast<uint32_t>((piece << sh) >> 32);
+  const uint32_t v2 = sh ? static_cast<uint32_t>(piece >> (64 - sh)) : 0u;
+  if (v0) atomicOr(&buf[w], v0);
+  if (v1) atomicOr(&buf[w + 1], v1);
+  if (v2) atomicOr(&buf[w + 2], v2);
+  __syncwarp();
+  for (int i = lane; i < nw; i += 32)
+    if (base + i < data_words) cr[base + i] = buf[i];
+  __syncwarp();
+}
+
 // ---------------------------------------------------------------------------
 // One warp per row
 // ---------------------------------------------------------------------------
 template <int BITS, int NVW>
 __global__ void __launch_bounds__(32 * kQWarps) quant_warp_kernel(const QuantArgs a) {
+  __shared__ uint32_t gbuf[BITS == 0 ? kQWarps * 64 : 1];  // width-b packing, per warp
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int64_t L = a.L;
-  const int64_t data_words = (L * BITS + 31) / 32;
+  const int bits = BITS == 0 ? a.bits : BITS;
+  const int64_t data_words = (L * bits + 31) / 32;
   for (int64_t row = static_cast<int64_t>(blockIdx.x) * kQWarps + warp; row < a.rows;
        row += static_cast<int64_t>(gridDim.x) * kQWarps) {
     const float* xr = a.x + row * L;
@@ -165,17 +207,23 @@ __global__ void __launch_bounds__(32 * kQWarps) quant_warp_kernel(const QuantArg
     }
     kmin = __reduce_min_sync(kFull, kmin);
     kmax = __reduce_max_sync(kFull, kmax);
-    const RowParams p = row_params(kmin, kmax, BITS, lane == 0 ? a.scale + row : nullptr,
+    const RowParams p = row_params(kmin, kmax, bits, lane == 0 ? a.scale + row : nullptr,
                                    lane == 0 ? a.minv + row : nullptr);
     uint32_t* cr = a.codes + row * a.W;
 #pragma unroll
     for (int v = 0; v < NVW; ++v) {
       const int64_t e0 = 4 * (v * 32 + lane);
-      uint32_t piece = codes4<BITS>(xs[v], e0, L, p, a.stochastic, a.seed,
-                                    static_cast<uint64_t>(row * L + e0));
-      const bool store = assemble_word<BITS>(piece, lane);
-      const int64_t w = e0 * BITS / 32;
-      if (store && w < data_words) cr[w] = piece;
+      if constexpr (BITS == 0) {
+        const uint64_t piece = codes4_any(xs[v], e0, L, p, a.stochastic, a.seed,
+                                          static_cast<uint64_t>(row * L + e0), bits);
+        store_codes_any(piece, bits, lane, gbuf + warp * 64, cr, 4 * bits * v, data_words);
+      } else {
+        uint32_t piece = codes4<BITS>(xs[v], e0, L, p, a.stochastic, a.seed,
+                                      static_cast<uint64_t>(row * L + e0));
+        const bool store = assemble_word<BITS>(piece, lane);
+        const int64_t w = e0 * BITS / 32;
+        if (store && w < data_words) cr[w] = piece;
+      }
     }
     if (lane < a.W - data_words) cr[data_words + lane] = 0u;  // row padding
   }
@@ -195,6 +243,8 @@ struct QuantShared {
 template <int BITS>
 __global__ void __launch_bounds__(kQNT) quant_cta_kernel(const QuantArgs a, int spr) {
   __shared__ QuantShared sh;
+  __shared__ uint32_t gbuf[BITS == 0 ? (kQNT / 32) * 64 : 1];  // width-b packing, per warp
+  const int bits = BITS == 0 ? a.bits : BITS;
   extern __shared__ __align__(16) float sx[];  // kQSCAP floats
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const bool from_ws = a.ws != nullptr;
@@ -280,11 +330,11 @@ __global__ void __launch_bounds__(kQNT) quant_cta_kernel(const QuantArgs a, int 
     }
   }
   const bool writer = sidx == 0 && tid == 0 && !failed;
-  const RowParams p = row_params(kmin, kmax, BITS, writer ? a.scale + row : nullptr,
+  const RowParams p = row_params(kmin, kmax, bits, writer ? a.scale + row : nullptr,
                                  writer ? a.minv + row : nullptr);
 
   uint32_t* cr = a.codes + row * a.W;
-  const int64_t data_words = (L * BITS + 31) / 32;
+  const int64_t data_words = (L * bits + 31) / 32;
   if (!failed) {
 #pragma unroll
     for (int v = 0; v < kQNV; ++v) {
@@ -292,11 +342,25 @@ __global__ void __launch_bounds__(kQNT) quant_cta_kernel(const QuantArgs a, int 
       const int64_t e0 = 4 * q;  // slice-relative
       const float4 f = reinterpret_cast<const float4*>(sx)[q];
       const float xs[4] = {f.x, f.y, f.z, f.w};
-      uint32_t piece = codes4<BITS>(xs, e0, nv, p, a.stochastic, a.seed,
-                                    static_cast<uint64_t>(row * L + c0 + e0));
-      const bool store = assemble_word<BITS>(piece, lane);
-      const int64_t w = (c0 + e0) * BITS / 32;
-      if (store && e0 < nv && w < data_words) cr[w] = piece;
+      if constexpr (BITS == 0) {
+        // the warp's 128 entries start at slice entry 128 (v * NW + warp); slices
+        // start on multiples of 128 entries, so the codes start on a word
+        // (this slice owns the words of its entries only: slices start on
+        // multiples of 128 entries, so no word is shared with the next one)
+        const int64_t chunk = 128 * (v * (kQNT / 32) + warp);
+        if (chunk < nv) {
+          const uint64_t piece = codes4_any(xs, e0, nv, p, a.stochastic, a.seed,
+                                            static_cast<uint64_t>(row * L + c0 + e0), bits);
+          const int64_t wend = min64(data_words, ((c0 + nv) * bits + 31) / 32);
+          store_codes_any(piece, bits, lane, gbuf + warp * 64, cr, (c0 + chunk) * bits / 32, wend);
+        }
+      } else {
+        uint32_t piece = codes4<BITS>(xs, e0, nv, p, a.stochastic, a.seed,
+                                      static_cast<uint64_t>(row * L + c0 + e0));
+        const bool store = assemble_word<BITS>(piece, lane);
+        const int64_t w = (c0 + e0) * BITS / 32;
+        if (store && e0 < nv && w < data_words) cr[w] = piece;
+      }
     }
     if (c0 + n >= L && tid < a.W - data_words) cr[data_words + tid] = 0u;  // row padding
   }
@@ -420,6 +484,59 @@ __global__ void __launch_bounds__(256)
   }
 }
 
+// Any width b in [1, 16], 16-byte aligned rows: as dequant_rows_kernel, the 4
+// codes of a float4 read from the one or two words that hold them.
+__global__ void __launch_bounds__(256)
+    dequant_rows_any_kernel(const uint32_t* __restrict__ codes, const float* __restrict__ scale,
+                            const float* __restrict__ minv, int64_t L, int64_t W, int bpr,
+                            int bits, float* __restrict__ y) {
+  const int64_t row = blockIdx.x / bpr;
+  const int64_t f0 = static_cast<int64_t>(blockIdx.x % bpr) * (256 * kDqU);
+  const int64_t n4 = L / 4;
+  const uint32_t* cr = codes + row * W;
+  float4* yr = reinterpret_cast<float4*>(y + row * L);
+  const float sc = scale[row], m = minv[row];
+  const uint32_t mask = (1u << bits) - 1u;
+#pragma unroll
+  for (int u = 0; u < kDqU; ++u) {
+    const int64_t f = f0 + u * 256 + threadIdx.x;
+    if (f < n4) {
+      const int64_t p = f * 4 * bits;  // bit offset of the 4 codes in the row
+      const int64_t w = p >> 5;
+      const int sh = static_cast<int>(p & 31);
+      uint64_t v = cr[w];
+      if (sh + 4 * bits > 32 && w + 1 < W) v |= static_cast<uint64_t>(cr[w + 1]) << 32;
+      if (sh + 4 * bits > 64 && w + 2 < W) v = (v >> sh) | (static_cast<uint64_t>(cr[w + 2]) << (64 - sh));
+      else v >>= sh;
+      float o[4];
+#pragma unroll
+      for (int t = 0; t < 4; ++t)
+        o[t] = fadd(m, fmul(static_cast<float>(static_cast<uint32_t>(v >> (bits * t)) & mask), sc));
+      yr[f] = make_float4(o[0], o[1], o[2], o[3]);
+    }
+  }
+}
+
+// Any width, any row: one entry per thread, grid-stride.
+__global__ void dequant_any_kernel(const uint32_t* __restrict__ codes, const float* __restrict__ scale,
+                                   const float* __restrict__ minv, int64_t rows, int64_t L,
+                                   int64_t W, int bits, float* __restrict__ y) {
+  const int64_t total = rows * L;
+  const uint32_t mask = (1u << bits) - 1u;
+  for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int64_t r = i / L, j = i - r * L;
+    const uint32_t* cr = codes + r * W;
+    const int64_t p = j * bits;
+    const int64_t w = p >> 5;
+    const int sh = static_cast<int>(p & 31);
+    uint64_t v = cr[w];
+    if (sh + bits > 32) v |= static_cast<uint64_t>(cr[w + 1]) << 32;
+    const uint32_t q = static_cast<uint32_t>(v >> sh) & mask;
+    y[i] = fadd(minv[r], fmul(static_cast<float>(q), scale[r]));
+  }
+}
+
 // 32-bit word indexing whenever the code array allows it (cheaper division).
 template <int BITS>
 void launch_dequant(const uint32_t* codes, const float* scale, const float* minv, int64_t rows,
@@ -530,7 +647,9 @@ cudaError_t launch_quant_compress(const QuantArgs& a, int num_sms, cudaStream_t 
       passthrough_kernel<<<grid_for(a.rows * a.W, num_sms), 256, 0, s>>>(a.x, a.rows, a.L, a.W,
                                                                           a.codes, a.scale, a.minv);
       return cudaGetLastError();
-    default: return cudaErrorInvalidValue;
+    default:
+      if (a.bits >= 1 && a.bits <= 16) return run_quant_bits<0>(a, num_sms, s);
+      return cudaErrorInvalidValue;
   }
 }
 
@@ -553,7 +672,16 @@ cudaError_t launch_quant_decompress(const uint32_t* codes, const float* scale,
     case 32:
       dequant_passthrough_kernel<<<grid_for(rows * L, num_sms), 256, 0, s>>>(codes, rows, L, W, y);
       break;
-    default: return cudaErrorInvalidValue;
+    default: {
+      if (bits < 1 || bits > 16) return cudaErrorInvalidValue;
+      const int64_t bpr = (L / 4 + 256 * kDqU - 1) / (256 * kDqU);
+      if (aligned && L % 4 == 0 && bpr > 0 && rows * bpr < 0x7fffffffLL)
+        dequant_rows_any_kernel<<<static_cast<unsigned>(rows * bpr), 256, 0, s>>>(
+            codes, scale, minv, L, W, static_cast<int>(bpr), bits, y);
+      else
+        dequant_any_kernel<<<grid_for(rows * L, num_sms), 256, 0, s>>>(codes, scale, minv, rows, L,
+                                                                      W, bits, y);
+    }
   }
   return cudaGetLastError();
 }

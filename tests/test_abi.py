@@ -52,7 +52,8 @@ def test_sizes(lib):
     assert lib.mpc_quant_codes_words(1, 31, 2) == 4
     assert lib.mpc_quant_codes_words(2, 16384, 8) == 2 * 4096
     assert lib.mpc_quant_codes_words(1, 5, 32) == 8
-    assert lib.mpc_quant_codes_words(1, 5, 6) == 0  # unsupported width
+    assert lib.mpc_quant_codes_words(1, 5, 6) == 4  # 6-bit codes straddle words
+    assert lib.mpc_quant_codes_words(1, 5, 17) == 0  # unsupported width
     assert lib.mpc_topk_workspace_bytes(128, 32768, 3276) == 0  # on-chip path
     assert lib.mpc_quant_workspace_bytes(128, 32768, 4) == 0
 
@@ -79,9 +80,16 @@ def test_zero_rows_is_a_noop(lib):
 
 def test_quant_validation(lib):
     p = ctypes.c_void_p(0x1000)
-    assert lib.mpc_quant_compress(p, 2, 16, 3, 0, 0, p, p, p, None, 0, None) == 1  # bits
+    for bad in (0, 17, 31, 33, -2):  # widths 1..16 and 32 only
+        assert lib.mpc_quant_compress(p, 2, 16, bad, 0, 0, p, p, p, None, 0, None) == 1
+        assert lib.mpc_quant_decompress(p, p, p, 2, 16, bad, p, None) == 1
+        assert lib.mpc_quant_codes_words(2, 16, bad) == 0
     assert lib.mpc_quant_compress(p, 2, 16, 4, 7, 0, p, p, p, None, 0, None) == 1  # mode
-    assert lib.mpc_quant_decompress(p, p, p, 2, 16, 5, p, None) == 1
+    # W = roundup4(ceil(L * bits / 32)) words per row, for every width
+    for bits in list(range(1, 17)) + [32]:
+        for L in (1, 31, 100, 4097):
+            w = -(-L * bits // 32)
+            assert lib.mpc_quant_codes_words(3, L, bits) == 3 * (-(-w // 4) * 4)
 
 
 def test_aqsgd_validation(lib):
