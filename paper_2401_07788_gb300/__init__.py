@@ -324,3 +324,9 @@ def mpc_last_error() -> str:
 
 def mpc_set_knob(knob: int, value: int) -> None:
     _check(lib().mpc_set_knob(knob, value))
+
+
+# The compression block between pipeline stages (§2.1) built on the calls above.
+from .boundary import CompressionBoundary, Quant, Reuse, TopK, with_boundaries  # noqa: E402
+
+__all__ += ["CompressionBoundary", "Quant", "TopK", "Reuse", "with_boundaries"]
