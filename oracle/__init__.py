@@ -67,6 +67,7 @@ def load(path: str | None = None) -> ctypes.CDLL:
         lib.orc_topk_gather.argtypes = [_F32P, _i64, _i64, _I32P, _i64, _F32P]
         lib.orc_ef_topk_compress.argtypes = [_F32P, _F32P, _i64, _i64, _i64, _F32P, _I32P]
         lib.orc_ef21_topk_compress.argtypes = [_F32P, _F32P, _i64, _i64, _i64, _F32P, _I32P]
+        lib.orc_efmix_topk_compress.argtypes = [_F32P, _F32P, _i64, _i64, _i64, _F32P, _I32P]
         lib.orc_aqsgd_compress.argtypes = [_F32P, _F32P, _i64, _I64P, _i64, _i64, _i64, _i64,
                                            _F32P, _I32P]
         lib.orc_aqsgd_decompress.argtypes = [_F32P, _I32P, _F32P, _i64, _I64P, _i64, _i64,
@@ -78,7 +79,7 @@ def load(path: str | None = None) -> ctypes.CDLL:
         lib.orc_quant_decompress.argtypes = [_U32P, _F32P, _F32P, _i64, _i64, ctypes.c_int,
                                              _F32P]
         for name in ("orc_topk_compress", "orc_topk_decompress", "orc_topk_gather",
-                     "orc_ef_topk_compress",
+                     "orc_ef_topk_compress", "orc_efmix_topk_compress",
                      "orc_ef21_topk_compress", "orc_aqsgd_compress", "orc_aqsgd_decompress",
                      "orc_quant_compress", "orc_quant_decompress"):
             getattr(lib, name).restype = None
@@ -148,6 +149,17 @@ def ef_topk_compress(x, e, k: int, lib=None):
     vals = np.empty((R, k), np.float32)
     idx = np.empty((R, k), np.int32)
     (lib or load()).orc_ef_topk_compress(x, e, R, L, k, vals, idx)
+    return vals, idx
+
+
+def efmix_topk_compress(x, e, k: int, lib=None):
+    """EF-mixed (§2.4). ``e`` (float32, C-contiguous) is updated in place."""
+    x = _f32(x)
+    assert e.dtype == np.float32 and e.flags.c_contiguous and e.shape == x.shape
+    R, L = _rows_cols(x)
+    vals = np.empty((R, k), np.float32)
+    idx = np.empty((R, k), np.int32)
+    (lib or load()).orc_efmix_topk_compress(x, e, R, L, k, vals, idx)
     return vals, idx
 
 

@@ -171,6 +171,57 @@ static void delta_row(const float* xr, float* gr, int64_t row_len, int64_t k,
     for (int64_t i = 0; i < k; ++i) gr[idx[i]] = gr[idx[i]] + vals[i];
 }
 
+/* EF-mixed, §2.4: the k largest magnitudes are split between the input and the
+ * error buffer, half each, and x + e is sent on the chosen entries.  Reading:
+ * the input's share is its ceil(k/2) largest |x|; the buffer's share, its
+ * floor(k/2) largest |e| among the entries the input's share did not take, so
+ * that exactly k entries are sent as the section states; the buffer keeps
+ * x + e everywhere else (e <- s - C(s) as in error feedback). */
+void orc_efmix_topk_compress(const float* x, float* e, int64_t rows, int64_t row_len,
+                             int64_t k, float* vals, int32_t* idx)
+{
+    const int64_t k1 = k - k / 2, k2 = k / 2;
+    orc_entry* work = (orc_entry*)malloc(sizeof(orc_entry) * (size_t)row_len);
+    char* taken = (char*)malloc((size_t)row_len);
+    for (int64_t r = 0; r < rows; ++r) {
+        const float* xr = x + r * row_len;
+        float* er = e + r * row_len;
+        memset(taken, 0, (size_t)row_len);
+        /* the input's share */
+        for (int64_t j = 0; j < row_len; ++j) {
+            work[j].mag = fabsf(xr[j]);
+            work[j].j = j;
+        }
+        qsort(work, (size_t)row_len, sizeof(orc_entry), by_magnitude_desc);
+        for (int64_t i = 0; i < k1; ++i) taken[work[i].j] = 1;
+        /* the buffer's share, among the entries left */
+        int64_t m = 0;
+        for (int64_t j = 0; j < row_len; ++j)
+            if (!taken[j]) {
+                work[m].mag = fabsf(er[j]);
+                work[m].j = j;
+                ++m;
+            }
+        qsort(work, (size_t)m, sizeof(orc_entry), by_magnitude_desc);
+        for (int64_t i = 0; i < k2; ++i) taken[work[i].j] = 1;
+        /* send s = x + e on the chosen entries, keep it elsewhere */
+        int64_t n = 0;
+        for (int64_t j = 0; j < row_len; ++j) {
+            float sj = xr[j] + er[j];
+            if (taken[j]) {
+                idx[r * k + n] = (int32_t)j;
+                vals[r * k + n] = sj;
+                ++n;
+                er[j] = 0.0f;
+            } else {
+                er[j] = sj;
+            }
+        }
+    }
+    free(taken);
+    free(work);
+}
+
 void orc_ef21_topk_compress(const float* x, float* g, int64_t rows, int64_t row_len,
                             int64_t k, float* vals, int32_t* idx)
 {

@@ -50,6 +50,11 @@ void orc_topk_gather(const float* g, int64_t rows, int64_t row_len, const int32_
 void orc_ef_topk_compress(const float* x, float* e, int64_t rows, int64_t row_len,
                           int64_t k, float* vals, int32_t* idx);
 
+/* EF-mixed, §2.4: ceil(k/2) largest |x|, then floor(k/2) largest |e| among the
+ * other entries; x + e sent there, e <- x + e elsewhere and +0 there. */
+void orc_efmix_topk_compress(const float* x, float* e, int64_t rows, int64_t row_len,
+                             int64_t k, float* vals, int32_t* idx);
+
 /* EF21, §2.4: send C(x - g), g <- g + C(x - g). */
 void orc_ef21_topk_compress(const float* x, float* g, int64_t rows, int64_t row_len,
                             int64_t k, float* vals, int32_t* idx);

@@ -210,6 +210,39 @@ def pin_ef_conservation(lib, seed: int = 6):
     assert np.linalg.norm(lhs - rhs) <= 1e-6 * np.linalg.norm(rhs)
 
 
+def pin_efmix_bruteforce(lib, n_rows: int = 3000, seed: int = 15):
+    """EF-mixed (§2.4) on tiny rows, every k: the input's ceil(k/2) by rank counting on
+    |x|, the buffer's floor(k/2) by rank counting on |e| over the rest; x + e sent there
+    in index order; the buffer keeps x + e elsewhere and +0 where sent; and the sent
+    message plus the new buffer is x + e exactly."""
+    rng = np.random.default_rng(seed)
+    for t in range(n_rows):
+        L = int(rng.integers(1, 24))
+        x = rng.standard_normal(L).astype(np.float32)
+        e = rng.standard_normal(L).astype(np.float32)
+        if t % 5 == 0:
+            x[rng.integers(0, L, L // 2)] = 0.5  # ties in |x|
+        if t % 7 == 0:
+            e[:] = 0.0  # the first step: an empty buffer
+        k = int(rng.integers(1, L + 1))
+        k1, k2 = k - k // 2, k // 2
+        s = x + e
+        first = set(brute_topk(x, k1).tolist())
+        rest = np.array(sorted(set(range(L)) - first), dtype=np.int64)
+        second = set(rest[brute_topk(e[rest], k2)].tolist()) if k2 else set()
+        want = np.array(sorted(first | second), dtype=np.int64)
+        e2 = e.copy()[None, :]
+        v, i = oracle.efmix_topk_compress(x[None, :], e2, k, lib)
+        assert np.array_equal(i[0], want), (t, i[0], want)
+        assert np.array_equal(bits_of(v[0]), bits_of(s[want]))
+        keep = np.ones(L, bool)
+        keep[want] = False
+        assert np.array_equal(bits_of(e2[0][keep]), bits_of(s[keep]))
+        assert np.all(bits_of(e2[0][~keep]) == 0)
+        y = oracle.topk_decompress(v, i, L, lib)
+        assert np.array_equal(bits_of(y[0] + e2[0]), bits_of(s + np.float32(0)))
+
+
 def pin_ef21_update(lib, seed: int = 7):
     rng = np.random.default_rng(seed)
     R, L, k = 10, 768, 76

@@ -40,6 +40,9 @@ MUTANTS = {
     "uniform_halves_swapped": ("(i & 1u) ? (uint32_t)(z >> 32) : (uint32_t)(z & 0xffffffffu)",
                                "(i & 1u) ? (uint32_t)(z & 0xffffffffu) : (uint32_t)(z >> 32)"),
     "signed_zero_min": ("return signbit(a) && !signbit(b);", "return 0;"),
+    "efmix_buffer_share_from_input": ("work[m].mag = fabsf(er[j]);", "work[m].mag = fabsf(xr[j]);"),
+    "efmix_shares_overlap": ("            if (!taken[j]) {\n                work[m].mag",
+                             "            if (1) {\n                work[m].mag"),
     "gather_row_offset_dropped": ("vals[r * k + i] = g[r * row_len + idx[r * k + i]];",
                                   "vals[r * k + i] = g[idx[r * k + i]];"),
 }
