@@ -278,6 +278,8 @@ def algorithmic_bytes(R_, L_, k=None, bits=None, op=""):
         return 8 * k * R_ + 4 * N
     if op == "delta_topk":  # EF21 / AQ-SGD: state written only where kept
         return 8 * N + 12 * k * R_
+    if op == "efmix_topk":  # x and err read, err written, payload written
+        return 12 * N + 8 * k * R_
     if op == "topk_gather":  # indices read, values gathered, payload written
         return 12 * k * R_
     if op == "aqsgd_decompress":
@@ -620,6 +622,15 @@ def measure_operators(mpc, synth, device, stream, peak):
     rec("topk_gather %dx%d K=10%%" % (R, L), time_op(lambda: mpc.mpc_topk_gather(gg, ig, vals=vg), stream, flush),
         algorithmic_bytes(R, L, k=kg, op="topk_gather"))
     del xg, gg
+    # EF-mixed at the CNN stage boundary, Top10% (two selections and four small steps)
+    xm = synth.relu_normal((R, L), 5, device)
+    em = torch.zeros_like(xm)
+    km = synth.k_of(L, 10)
+    vm, im = mpc.mpc_efmix_topk_compress(xm, em, km)
+    wsm = torch.empty(mpc.mpc_efmix_workspace_bytes(R, L, km), dtype=torch.uint8, device=device)
+    rec("efmix_topk_compress %dx%d K=10%%" % (R, L), time_op(lambda: mpc.mpc_efmix_topk_compress(xm, em, km, vm, im, ws=wsm), stream, flush),
+        algorithmic_bytes(R, L, k=km, op="efmix_topk"))
+    del xm, em, wsm
     # LM boundary: EF21 Top10% per token, 4-bit
     xl = synth.lm_hidden(0, device)
     gl = torch.zeros_like(xl)

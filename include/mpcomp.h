@@ -119,6 +119,23 @@ mpc_status mpc_ef_topk_compress(const float* x, float* err, int64_t rows, int64_
                                 int64_t k, float* vals, int32_t* idx, void* ws,
                                 size_t ws_bytes, mpc_stream_t stream);
 
+/* EF-mixed TopK (§2.4: "the largest K/2% values from the input vector X and
+ * K/2% of the current error buffer", then "the input vector and buffer are
+ * added and sent, resulting in the same K% non-zero values").  Reading: the
+ * input's share is its ceil(k/2) largest |x|; the buffer's share is its
+ * floor(k/2) largest |err| among the entries the input's share did not take
+ * (so exactly k entries are sent); ties go to the lower index.  Then
+ *   s = x + err;  (vals, idx) = s at those k entries, ascending idx;
+ *   err <- +0 there and s elsewhere.
+ * err [rows][row_len] is read and rewritten in place (start it at zero).
+ * ws: device workspace of ws_bytes >= mpc_efmix_workspace_bytes(rows,
+ * row_len, k), 256-byte aligned (never NULL: the input's share is kept there
+ * between the two selections); MPC_ERR_WORKSPACE if smaller. */
+size_t mpc_efmix_workspace_bytes(int64_t rows, int64_t row_len, int64_t k);
+mpc_status mpc_efmix_topk_compress(const float* x, float* err, int64_t rows, int64_t row_len,
+                                   int64_t k, float* vals, int32_t* idx, void* ws,
+                                   size_t ws_bytes, mpc_stream_t stream);
+
 /* EF21 fused with TopK (§2.4: message C(X_{i+1} - g_i), buffer
  * g_{i+1} = g_i + C(X_{i+1} - g_i)):
  *   d = x - g;  (vals, idx) = TopK(d, k);  g[kept] <- g[kept] + d[kept].

@@ -21,7 +21,7 @@ from ._build import LIB_PATH
 
 __all__ = [
     "MpcError", "lib", "mpc_topk_workspace_bytes", "mpc_topk_compress", "mpc_topk_decompress",
-    "mpc_topk_gather",
+    "mpc_topk_gather", "mpc_efmix_workspace_bytes", "mpc_efmix_topk_compress",
     "mpc_ef_topk_compress", "mpc_ef21_topk_compress", "mpc_aqsgd_compress",
     "mpc_aqsgd_decompress", "mpc_quant_codes_words", "mpc_quant_workspace_bytes",
     "mpc_quant_compress", "mpc_quant_decompress", "mpc_get_status", "mpc_last_error",
@@ -46,6 +46,8 @@ _SIGNATURES = {
     "mpc_topk_compress": ([_VP, _I64, _I64, _I64, _VP, _VP, _VP, _SZ, _VP], _INT),
     "mpc_topk_decompress": ([_VP, _VP, _I64, _I64, _I64, _VP, _VP], _INT),
     "mpc_topk_gather": ([_VP, _I64, _I64, _VP, _I64, _VP, _VP], _INT),
+    "mpc_efmix_workspace_bytes": ([_I64, _I64, _I64], _SZ),
+    "mpc_efmix_topk_compress": ([_VP, _VP, _I64, _I64, _I64, _VP, _VP, _VP, _SZ, _VP], _INT),
     "mpc_ef_topk_compress": ([_VP, _VP, _I64, _I64, _I64, _VP, _VP, _VP, _SZ, _VP], _INT),
     "mpc_ef21_topk_compress": ([_VP, _VP, _I64, _I64, _I64, _VP, _VP, _VP, _SZ, _VP], _INT),
     "mpc_aqsgd_compress": ([_VP, _VP, _I64, _VP, _I64, _I64, _I64, _I64, _VP, _VP, _VP, _SZ,
@@ -173,6 +175,23 @@ def mpc_ef_topk_compress(x, err, k: int, vals=None, idx=None, ws=None, stream=No
     ws, wsb = _workspace(mpc_topk_workspace_bytes(R, L, k) if R else 0, ws, x.device)
     _check(lib().mpc_ef_topk_compress(_ptr(x), _ptr(err), R, L, k, _ptr(vals), _ptr(idx),
                                       _ptr(ws), wsb, _stream(stream)))
+    return vals, idx
+
+
+def mpc_efmix_workspace_bytes(rows: int, row_len: int, k: int) -> int:
+    return int(lib().mpc_efmix_workspace_bytes(rows, row_len, k))
+
+
+def mpc_efmix_topk_compress(x, err, k: int, vals=None, idx=None, ws=None, stream=None):
+    """EF-mixed (§2.4); ``err`` is updated in place."""
+    _cuda(x, torch.float32, "x")
+    _cuda(err, torch.float32, "err")
+    if err.shape != x.shape:
+        raise MpcError(1, "err must have the shape of x")
+    R, L, vals, idx = _topk_outputs(x, k, vals, idx)
+    ws, wsb = _workspace(mpc_efmix_workspace_bytes(R, L, k) if R else 0, ws, x.device)
+    _check(lib().mpc_efmix_topk_compress(_ptr(x), _ptr(err), R, L, k, _ptr(vals), _ptr(idx),
+                                         _ptr(ws), wsb, _stream(stream)))
     return vals, idx
 
 

@@ -1,6 +1,7 @@
 // abi.cu -- the extern "C" entry points of libmpcomp (declared in
 // include/mpcomp.h): argument validation, path selection and the device
 // status word.  No entry point allocates device memory.
+#include <algorithm>
 #include <atomic>
 #include <cstdarg>
 #include <cstdio>
@@ -204,6 +205,56 @@ mpc_status mpc_topk_decompress(const float* vals, const int32_t* idx, int64_t ro
   cudaError_t e = mpc::launch_topk_decompress(vals, idx, rows, row_len, k, y, aligned, d.num_sms,
                                               reinterpret_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_error(e, "topk_decompress launch");
+  return ok();
+}
+
+size_t mpc_efmix_workspace_bytes(int64_t rows, int64_t row_len, int64_t k) {
+  if (rows <= 0 || row_len <= 0 || k < 1 || k > row_len || rows > INT64_MAX / row_len) return 0;
+  const int64_t k1 = k - k / 2;
+  const size_t share = (static_cast<size_t>(rows * k1) * 4u + 255u) / 256u * 256u;
+  size_t grid = 0;
+  if (!use_row_path(row_len))
+    grid = std::max(mpc::topk_grid_workspace_bytes(rows, row_len, k1),
+                    mpc::topk_grid_workspace_bytes(rows, row_len, k));
+  return 2 * share + grid;
+}
+
+mpc_status mpc_efmix_topk_compress(const float* x, float* err, int64_t rows, int64_t row_len,
+                                   int64_t k, float* vals, int32_t* idx, void* ws,
+                                   size_t ws_bytes, mpc_stream_t stream) {
+  MPC_TRY(check_shape(rows, row_len, k));
+  if (rows == 0) return ok();
+  MPC_TRY(check_ptr(x, 4, "x"));
+  MPC_TRY(check_ptr(err, 4, "err"));
+  MPC_TRY(check_ptr(vals, 4, "vals"));
+  MPC_TRY(check_ptr(idx, 4, "idx"));
+  const size_t need = mpc_efmix_workspace_bytes(rows, row_len, k);
+  if (ws == nullptr || ws_bytes < need)
+    return set_error(MPC_ERR_WORKSPACE, "workspace of %zu bytes needed, %zu given", need,
+                     ws == nullptr ? (size_t)0 : ws_bytes);
+  if (!aligned_to(ws, 256)) return set_error(MPC_ERR_INVALID_ARG, "ws is not 256-byte aligned");
+  Device d;
+  MPC_TRY(current_device(&d));
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const int64_t k1 = k - k / 2;
+  const size_t share = (static_cast<size_t>(rows * k1) * 4u + 255u) / 256u * 256u;
+  int32_t* idx1 = static_cast<int32_t*>(ws);
+  float* saved = reinterpret_cast<float*>(static_cast<char*>(ws) + share);
+  void* gws = static_cast<char*>(ws) + 2 * share;
+  const size_t gws_bytes = ws_bytes - 2 * share;
+  // the input's share (its values land in `saved`, which the marking then reuses)
+  MPC_TRY(topk_compress_common(mpc::kPlain, x, nullptr, rows, row_len, k1, saved, idx1,
+                               gws_bytes ? gws : nullptr, gws_bytes, s));
+  cudaError_t e = mpc::launch_efmix_mark(err, idx1, rows, row_len, k1, saved, 0, s);
+  if (e != cudaSuccess) return cuda_error(e, "efmix mark launch");
+  // the k largest |err| with the input's share at +inf: that share and the
+  // buffer's, in ascending index
+  MPC_TRY(topk_compress_common(mpc::kPlain, err, nullptr, rows, row_len, k, vals, idx,
+                               gws_bytes ? gws : nullptr, gws_bytes, s));
+  e = mpc::launch_efmix_mark(err, idx1, rows, row_len, k1, saved, 1, s);
+  if (e == cudaSuccess) e = mpc::launch_efmix_add(x, err, rows * row_len, d.num_sms, s);
+  if (e == cudaSuccess) e = mpc::launch_efmix_send(err, idx, rows, row_len, k, vals, s);
+  if (e != cudaSuccess) return cuda_error(e, "efmix launch");
   return ok();
 }
 

@@ -58,6 +58,12 @@ cudaError_t launch_topk_grid(int mode, const TopkGridArgs& a, int num_sms, cudaS
 cudaError_t launch_topk_decompress(const float* vals, const int32_t* idx, int64_t rows,
                                    int64_t L, int64_t k, float* y, int aligned, int num_sms,
                                    cudaStream_t s);
+// EF-mixed (§2.4): the steps between its two TopK calls (topk_efmix.cu).
+cudaError_t launch_efmix_mark(float* err, const int32_t* idx, int64_t rows, int64_t L, int64_t k,
+                              float* saved, int restore, cudaStream_t s);
+cudaError_t launch_efmix_add(const float* x, float* err, int64_t n, int num_sms, cudaStream_t s);
+cudaError_t launch_efmix_send(float* err, const int32_t* idx, int64_t rows, int64_t L, int64_t k,
+                              float* vals, cudaStream_t s);
 cudaError_t launch_topk_gather(const float* g, const int32_t* idx, int64_t rows, int64_t L,
                               int64_t k, float* vals, unsigned* status, cudaStream_t s);
 cudaError_t launch_aqsgd_decompress(const float* vals, const int32_t* idx, float* buf,

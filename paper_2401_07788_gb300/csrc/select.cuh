@@ -31,6 +31,11 @@ __device__ __forceinline__ float bucket_scale(int maxkey, int nb) {
   return (__float_as_uint(s) < 0x7f800000u) ? s : 0.0f;
 }
 
+// The key if it is that of a finite number, else -1: the bin scale comes from
+// the largest finite magnitude, and infinities (TopK marks entries with them)
+// or NaNs then fall in the top bin.
+__device__ __forceinline__ int finite_key(int key) { return key < 0x7f800000 ? key : -1; }
+
 // Bin of a key (>= 0) in the |x|-linear histogram.  Monotone in the key:
 // |x| * scale rounds monotonically and truncation is monotone.
 __device__ __forceinline__ int bucket_of(int key, float scale, int nb) {

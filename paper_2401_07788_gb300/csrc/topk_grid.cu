@@ -127,7 +127,7 @@ __global__ void __launch_bounds__(kGT) g_sample(const float* xr, const float* ar
   int mx = -1;
   for (int s = threadIdx.x; s < kSamples; s += kGT) {
     const int64_t e = (L / kSamples) * s;
-    if (e < L) mx = max(mx, mag_key(ranked<MODE>(xr[e], MODE != kPlain ? ar[e] : 0.0f)));
+    if (e < L) mx = max(mx, finite_key(mag_key(ranked<MODE>(xr[e], MODE != kPlain ? ar[e] : 0.0f))));
   }
   mx = __reduce_max_sync(kFull, mx);
   if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = static_cast<uint32_t>(mx);

@@ -378,7 +378,7 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
     int smax = -1;
 #pragma unroll
     for (int i = 0; i < 4; ++i)
-      if (sp + i < L) smax = max(smax, mag_key(ranked_value<MODE>(sx[i], sa[i])));
+      if (sp + i < L) smax = max(smax, finite_key(mag_key(ranked_value<MODE>(sx[i], sa[i]))));
     smax = __reduce_max_sync(kFull, smax);
     if (lane == 0) sh.sample_max[warp] = smax;
   }
@@ -954,8 +954,8 @@ __global__ void __launch_bounds__(32 * WPC) topk_warp_kernel(const TopkRowArgs a
     float4* x4 = reinterpret_cast<float4*>(xs);
     const float4* a4 = reinterpret_cast<const float4*>(as);
 
-    // ---- ranked values (in place) and the row maximum ----------------------
-    int kmax = -1;
+    // ---- ranked values (in place), the largest finite magnitude, any NaN -------
+    int kmax = -1, kall = -1;
 #pragma unroll
     for (int v = 0; v < NVW; ++v) {
       const int q = v * 32 + lane;
@@ -966,9 +966,13 @@ __global__ void __launch_bounds__(32 * WPC) topk_warp_kernel(const TopkRowArgs a
       }
       int kk[4];
       keys4<FULL>(val, 4 * q, n, kk);
-      kmax = max(kmax, max(max(kk[0], kk[1]), max(kk[2], kk[3])));
+      kmax = max(kmax, max(max(finite_key(kk[0]), finite_key(kk[1])),
+                           max(finite_key(kk[2]), finite_key(kk[3]))));
+      kall = max(kall, max(max(kk[0], kk[1]), max(kk[2], kk[3])));
     }
     kmax = __reduce_max_sync(kFull, kmax);
+    // a NaN row (outside the finite-input contract) takes the integer rounds
+    if (__reduce_max_sync(kFull, kall) > 0x7f800000) kmax = 0;
 
     // ---- select ---------------------------------------------------------------
     Threshold t;
