@@ -166,7 +166,7 @@ struct CtaShared {
   // the same words hold the row's candidate keys, this CTA's candidate chunks
   // and the histograms of the integer rounds.
   union {
-    uint32_t hist[kNB];
+    uint32_t hist[kNB + 64];  // + 32 zero spill counters, + 32 past-the-end ones
     struct {
       int cand[kLCAP];        // the row's candidates, CTA by CTA (pushed)
       uint16_t lch[kLCAP];    // chunk of each of this CTA's candidates
@@ -369,7 +369,7 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
                : make_float4(0.f, 0.f, 0.f, 0.f);
   };
   float4 anext = aux4(0);
-  for (int i = tid; i < kNB; i += NT) sh.u.hist[i] = 0;
+  for (int i = tid; i < kNB + 64; i += NT) sh.u.hist[i] = 0;
   if (tid == 0) {
     sh.lcount = 0;
     sh.thr = Threshold{0x7fffffff, 0};
@@ -394,7 +394,6 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
 
   // ---- ranked values into shared memory and the first histogram -------------
   bool failed = false;
-  uint32_t zc = 0;
 #pragma unroll
   for (int j = 0; j < QPT; ++j) {
     if (j < jmax) {
@@ -415,17 +414,16 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
         keys4<FULL>(v, 4 * q, n, kk);
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
-          // zeros (common after ReLU) are counted per warp, not by atomics
-          zc += kk[i] == 0;
+          // one atomic per entry and no branch: zeros (common after ReLU) go to
+          // this lane's own spill counter rather than all to bin 0 (folded into
+          // bin 0 when the histogram is packed), slots past the slice end to a
+          // second spill counter that is never read
           const int b = lin_bin(kk[i], scale);
-          if (kk[i] > 0) atomicAdd(&sh.u.hist[b], 1u);
+          const int slot = kk[i] > 0 ? b : ((FULL || kk[i] == 0) ? kNB + lane : kNB + 32 + lane);
+          atomicAdd(&sh.u.hist[slot], 1u);
         }
       }
     }
-  }
-  if (binned) {
-    zc = __reduce_add_sync(kFull, zc);
-    if (lane == 0 && zc) atomicAdd(&sh.u.hist[0], zc);
   }
   failed = __syncthreads_or(failed);
   // A slice whose copy timed out takes part in the rest as an empty one (the
@@ -453,6 +451,12 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
         uint32_t w[GW];
 #pragma unroll
         for (int i = 0; i < GW; ++i) w[i] = sh.u.hist[b0 + 2 * i] | (sh.u.hist[b0 + 2 * i + 1] << 16);
+        if (b0 == 0) {
+          // the zeros, from the spill counters, into bin 0
+          uint32_t z = 0;
+          for (int l = 0; l < 32; ++l) z += sh.u.hist[kNB + l];
+          w[0] += z;
+        }
         uint32_t* dst = table + (crank * NT + tid) * GW;
         if (C > 1) {
           for (uint32_t r = 0; r < C; ++r) {
@@ -850,7 +854,7 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
 // Warp-per-row kernel (rows of at most 128 * NVW entries, WPC warps per CTA)
 // ---------------------------------------------------------------------------
 struct WarpShared {
-  uint32_t hist[kRoundBins];
+  uint32_t hist[kRoundBins + 64];  // + 32 zero spill counters, + 32 past-the-end ones
   int lkey[kLCAPW];
   uint32_t lcount;
   uint64_t bar[2];
@@ -987,9 +991,10 @@ __global__ void __launch_bounds__(32 * WPC) topk_warp_kernel(const TopkRowArgs a
       if (scale > 0.0f) {
 #pragma unroll
         for (int j = 0; j < 8; ++j) sh.hist[lane * 8 + j] = 0;
+        sh.hist[kRoundBins + lane] = 0;
+        sh.hist[kRoundBins + 32 + lane] = 0;
         if (lane == 0) sh.lcount = 0;
         __syncwarp();
-        uint32_t zc = 0;
 #pragma unroll
         for (int v = 0; v < NVW; ++v) {
           const int q = v * 32 + lane;
@@ -997,12 +1002,18 @@ __global__ void __launch_bounds__(32 * WPC) topk_warp_kernel(const TopkRowArgs a
           keys4<FULL>(x4[q], 4 * q, n, kk);
 #pragma unroll
           for (int i = 0; i < 4; ++i) {
-            if (kk[i] == 0) ++zc;
-            else if (kk[i] > 0) atomicAdd(&sh.hist[bucket_of(kk[i], scale, kRoundBins)], 1u);
+            // one atomic per entry and no branch: zeros to this lane's spill
+            // counter (folded into bin 0 below), past-the-end slots to another
+            const int b = bucket_of(kk[i], scale, kRoundBins);
+            const int slot = kk[i] > 0 ? b
+                                       : ((FULL || kk[i] == 0) ? kRoundBins + lane
+                                                               : kRoundBins + 32 + lane);
+            atomicAdd(&sh.hist[slot], 1u);
           }
         }
-        zc = __reduce_add_sync(kFull, zc);
-        if (lane == 0 && zc) atomicAdd(&sh.hist[0], zc);
+        __syncwarp();
+        const uint32_t zc = __reduce_add_sync(kFull, sh.hist[kRoundBins + lane]);
+        if (lane == 0) sh.hist[0] += zc;
         __syncwarp();
         const BinPick p = warp_pick_bin(sh.hist, kr, lane);
         __syncwarp();
