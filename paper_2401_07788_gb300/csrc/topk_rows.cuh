@@ -186,6 +186,7 @@ struct CtaShared {
   uint32_t pick_t, pick_excl;
   int pub_lo, pub_hi;
   uint32_t before_gt, before_eq;
+  uint8_t woff[NW][128];  // per warp: column offsets of a chunk's staged kept entries
   BinPick pick;
   PickOut pk;
   Threshold thr;
@@ -812,20 +813,44 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
 #pragma unroll
       for (int i = 0; i < 4; ++i) kp[i] = kk[i] > T;
     }
-#pragma unroll
-    for (int i = 0; i < 4; ++i) pos += __popc(__ballot_sync(kFull, kp[i]) & lt);
-    const int e0 = 4 * q;
-    if (!FULL && e0 >= nv) continue;
-    const float val[4] = {v4.x, v4.y, v4.z, v4.w};
-    const int col = static_cast<int>(c0) + e0;
-    uint32_t pi[4];
-    pi[0] = pos;
-#pragma unroll
-    for (int i = 1; i < 4; ++i) pi[i] = pi[i - 1] + (kp[i - 1] ? 1u : 0u);
+    // this lane's first position among the chunk's kept entries, and their count
+    uint32_t pre = 0, tot = 0;
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-      if (kp[i] && pi[i] < kk32) vrow[pi[i]] = val[i];
-      if (kp[i] && pi[i] < kk32) irow[pi[i]] = col + i;
+      const unsigned b = __ballot_sync(kFull, kp[i]);
+      pre += __popc(b & lt);
+      tot += __popc(b);
+    }
+    const int e0 = 4 * q;
+    const float val[4] = {v4.x, v4.y, v4.z, v4.w};
+    const int col = static_cast<int>(c0) + e0;
+    // The kept entries are staged in the chunk's own float4 slots (every lane
+    // has read its slot) with their column offsets, then written out with
+    // coalesced stores.
+    float* sval = reinterpret_cast<float*>(s4 + j * NT + warp * 32);
+    uint8_t* soff = sh.woff[warp];
+    __syncwarp();
+    {
+      uint32_t r = pre;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        if (kp[i]) {
+          sval[r] = val[i];
+          soff[r] = static_cast<uint8_t>(4 * lane + i);
+        }
+        r += kp[i] ? 1u : 0u;
+      }
+    }
+    __syncwarp();
+    {
+      const int colbase = static_cast<int>(c0) + 4 * (j * NT + warp * 32);
+      for (uint32_t t = lane; t < tot; t += 32) {
+        const uint32_t p = pos + t;
+        if (p < kk32) {
+          vrow[p] = sval[t];
+          irow[p] = colbase + soff[t];
+        }
+      }
     }
     if (MODE == kDelta) {
 #pragma unroll
