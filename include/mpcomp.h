@@ -259,9 +259,14 @@ const char* mpc_last_error(void);
  *                         (default 1<<20, about 0.07 s; 0 makes every first wait give
  *                         up, which tests the timeout report without a fault);
  *   MPC_KNOB_TOPK_PATH    0 = automatic, 1 = force the on-chip row path when
- *                         it fits, 2 = force the multi-pass (workspace) path.
- * Returns MPC_ERR_INVALID_ARG for an unknown knob. */
-typedef enum { MPC_KNOB_SPIN_LIMIT = 1, MPC_KNOB_TOPK_PATH = 2 } mpc_knob;
+ *                         it fits, 2 = force the multi-pass (workspace) path;
+ *   MPC_KNOB_PDL          1 (default) = launch the hot kernels with
+ *                         programmatic dependent launch, so that a launch
+ *                         overlaps the end of the previous one in the stream
+ *                         (every kernel first waits for the grids it depends
+ *                         on); 0 = plain stream order.
+ * Returns MPC_ERR_INVALID_ARG for an unknown knob or value. */
+typedef enum { MPC_KNOB_SPIN_LIMIT = 1, MPC_KNOB_TOPK_PATH = 2, MPC_KNOB_PDL = 3 } mpc_knob;
 mpc_status mpc_set_knob(mpc_knob knob, int64_t value);
 
 #ifdef __cplusplus

@@ -25,7 +25,7 @@ __all__ = [
     "mpc_ef_topk_compress", "mpc_ef21_topk_compress", "mpc_aqsgd_compress",
     "mpc_aqsgd_decompress", "mpc_quant_codes_words", "mpc_quant_workspace_bytes",
     "mpc_quant_compress", "mpc_quant_decompress", "mpc_get_status", "mpc_last_error",
-    "mpc_set_knob", "MPC_KNOB_SPIN_LIMIT", "MPC_KNOB_TOPK_PATH", "STATUS_NAMES",
+    "mpc_set_knob", "MPC_KNOB_SPIN_LIMIT", "MPC_KNOB_TOPK_PATH", "MPC_KNOB_PDL", "STATUS_NAMES",
 ]
 
 STATUS_NAMES = {0: "MPC_OK", 1: "MPC_ERR_INVALID_ARG", 2: "MPC_ERR_UNSUPPORTED",
@@ -33,6 +33,7 @@ STATUS_NAMES = {0: "MPC_OK", 1: "MPC_ERR_INVALID_ARG", 2: "MPC_ERR_UNSUPPORTED",
                 6: "MPC_ERR_DEVICE"}
 MPC_KNOB_SPIN_LIMIT = 1
 MPC_KNOB_TOPK_PATH = 2
+MPC_KNOB_PDL = 3
 
 _VP = ctypes.c_void_p
 _I64 = ctypes.c_int64

@@ -18,6 +18,7 @@ __device__ unsigned g_status_word = 0;
 
 thread_local char g_last_error[512];
 std::atomic<uint32_t> g_spin_limit{1u << 20};
+std::atomic<int> g_pdl{1};
 std::atomic<int> g_topk_path{0};
 
 constexpr int kMaxDevices = 64;
@@ -160,6 +161,10 @@ mpc_status topk_compress_common(int mode, const float* x, float* aux, int64_t ro
 }
 
 }  // namespace
+
+namespace mpc {
+bool pdl_enabled() { return g_pdl.load(std::memory_order_relaxed) != 0; }
+}  // namespace mpc
 
 extern "C" {
 
@@ -483,6 +488,10 @@ const char* mpc_last_error(void) { return g_last_error; }
 
 mpc_status mpc_set_knob(mpc_knob knob, int64_t value) {
   switch (knob) {
+    case MPC_KNOB_PDL:
+      if (value != 0 && value != 1) return set_error(MPC_ERR_INVALID_ARG, "pdl knob is 0 or 1");
+      g_pdl.store(static_cast<int>(value));
+      return ok();
     case MPC_KNOB_SPIN_LIMIT:
       if (value < 0 || value > 0xffffffffLL) return set_error(MPC_ERR_INVALID_ARG, "spin limit");
       g_spin_limit.store(static_cast<uint32_t>(value));

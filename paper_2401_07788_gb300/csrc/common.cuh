@@ -26,6 +26,20 @@ __device__ __forceinline__ void set_status(unsigned* status, unsigned bits) {
 }
 
 // ---------------------------------------------------------------------------
+// Programmatic dependent launch.  Every kernel calls pdl_begin() before it
+// touches global memory: it waits until the grids it depends on have completed
+// and their writes are visible (at once when it was launched without the
+// programmatic-serialisation attribute).  The hot kernels call pdl_end() when
+// their last phase has started, which lets the next grid in the stream be
+// scheduled then, so that its launch overlaps this grid's tail (a grid that
+// does not call it lets the next one start as its CTAs exit).
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void pdl_begin() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_end() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+// ---------------------------------------------------------------------------
 // Exact fp32 arithmetic: every call is one IEEE round-to-nearest-even
 // operation and is never contracted into a fused multiply-add.
 // ---------------------------------------------------------------------------

@@ -91,26 +91,32 @@ __device__ __forceinline__ RowParams row_params(uint32_t kmin, uint32_t kmax, in
   return p;
 }
 
-// Code of one entry.
-__device__ __forceinline__ uint32_t code_of(float x, const RowParams& p, bool stochastic, float u) {
+// Code of one entry.  q is a whole number in [0, 2^16 - 1], so q + 2^23 is
+// exact and its low mantissa bits are q: the float-to-integer step stays on
+// the FP32 pipe.
+template <bool SR>
+__device__ __forceinline__ uint32_t code_of(float x, const RowParams& p, float u) {
   const float t = fmul(fsub(x, p.mn), p.inv);
-  float q = stochastic ? floorf(fadd(t, u)) : rintf(t);
+  float q = SR ? floorf(fadd(t, u)) : rintf(t);
   q = fminf(fmaxf(q, 0.0f), p.levels);
-  return static_cast<uint32_t>(q);
+  return __float_as_uint(fadd(q, 8388608.0f)) & 0x7fffffu;
 }
 
 // Codes of the 4 entries e0..e0+3 of a row (entries at or past n give 0).
-template <int BITS>
+// u: the stochastic rounding offsets of the 4 entries (unused for nearest).
+template <int BITS, bool SR>
 __device__ __forceinline__ uint32_t codes4(const float xs[4], int64_t e0, int64_t n,
-                                           const RowParams& p, bool stochastic, uint64_t seed,
-                                           uint64_t flat0) {
+                                           const RowParams& p, const float u[4]) {
   uint32_t packed = 0;
   if (p.degenerate) return 0;
-  float u[4] = {0.f, 0.f, 0.f, 0.f};
-  if (stochastic) uniform4(seed, flat0, u);
+  if (e0 + 4 <= n) {
 #pragma unroll
-  for (int t = 0; t < 4; ++t)
-    if (e0 + t < n) packed |= code_of(xs[t], p, stochastic, u[t]) << (BITS * t);
+    for (int t = 0; t < 4; ++t) packed |= code_of<SR>(xs[t], p, u[t]) << (BITS * t);
+  } else {
+#pragma unroll
+    for (int t = 0; t < 4; ++t)
+      if (e0 + t < n) packed |= code_of<SR>(xs[t], p, u[t]) << (BITS * t);
+  }
   return packed;
 }
 
@@ -134,17 +140,14 @@ __device__ __forceinline__ bool assemble_word(uint32_t& piece, int lane) {
 
 // Any width b in [1, 16] (BITS == 0 instantiations; b known at run time): the
 // codes of entries e0..e0+3 as one 4b-bit piece.
+template <bool SR>
 __device__ __forceinline__ uint64_t codes4_any(const float xs[4], int64_t e0, int64_t n,
-                                               const RowParams& p, bool stochastic,
-                                               uint64_t seed, uint64_t flat0, int bits) {
+                                               const RowParams& p, const float u[4], int bits) {
   uint64_t packed = 0;
   if (p.degenerate) return 0;
-  float u[4] = {0.f, 0.f, 0.f, 0.f};
-  if (stochastic) uniform4(seed, flat0, u);
 #pragma unroll
   for (int t = 0; t < 4; ++t)
-    if (e0 + t < n)
-      packed |= static_cast<uint64_t>(code_of(xs[t], p, stochastic, u[t])) << (bits * t);
+    if (e0 + t < n) packed |= static_cast<uint64_t>(code_of<SR>(xs[t], p, u[t])) << (bits * t);
   return packed;
 }
 
@@ -175,8 +178,9 @@ __device__ __forceinline__ void store_codes_any(uint64_t piece, int bits, int la
 // ---------------------------------------------------------------------------
 // One warp per row
 // ---------------------------------------------------------------------------
-template <int BITS, int NVW>
+template <int BITS, int NVW, bool SR>
 __global__ void __launch_bounds__(32 * kQWarps) quant_warp_kernel(const QuantArgs a) {
+  pdl_begin();
   __shared__ uint32_t gbuf[BITS == 0 ? kQWarps * 64 : 1];  // width-b packing, per warp
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int64_t L = a.L;
@@ -214,12 +218,14 @@ __global__ void __launch_bounds__(32 * kQWarps) quant_warp_kernel(const QuantArg
     for (int v = 0; v < NVW; ++v) {
       const int64_t e0 = 4 * (v * 32 + lane);
       if constexpr (BITS == 0) {
-        const uint64_t piece = codes4_any(xs[v], e0, L, p, a.stochastic, a.seed,
-                                          static_cast<uint64_t>(row * L + e0), bits);
+        float u[4] = {0.f, 0.f, 0.f, 0.f};
+        if (SR) uniform4(a.seed, static_cast<uint64_t>(row * L + e0), u);
+        const uint64_t piece = codes4_any<SR>(xs[v], e0, L, p, u, bits);
         store_codes_any(piece, bits, lane, gbuf + warp * 64, cr, 4 * bits * v, data_words);
       } else {
-        uint32_t piece = codes4<BITS>(xs[v], e0, L, p, a.stochastic, a.seed,
-                                      static_cast<uint64_t>(row * L + e0));
+        float u[4] = {0.f, 0.f, 0.f, 0.f};
+        if (SR) uniform4(a.seed, static_cast<uint64_t>(row * L + e0), u);
+        uint32_t piece = codes4<BITS, SR>(xs[v], e0, L, p, u);
         const bool store = assemble_word<BITS>(piece, lane);
         const int64_t w = e0 * BITS / 32;
         if (store && w < data_words) cr[w] = piece;
@@ -240,8 +246,9 @@ struct QuantShared {
   uint64_t bars[kQNV];  // one per slice chunk
 };
 
-template <int BITS>
+template <int BITS, bool SR>
 __global__ void __launch_bounds__(kQNT) quant_cta_kernel(const QuantArgs a, int spr) {
+  pdl_begin();
   __shared__ QuantShared sh;
   __shared__ uint32_t gbuf[BITS == 0 ? (kQNT / 32) * 64 : 1];  // width-b packing, per warp
   const int bits = BITS == 0 ? a.bits : BITS;
@@ -335,6 +342,7 @@ __global__ void __launch_bounds__(kQNT) quant_cta_kernel(const QuantArgs a, int 
 
   uint32_t* cr = a.codes + row * a.W;
   const int64_t data_words = (L * bits + 31) / 32;
+  pdl_end();
   if (!failed) {
 #pragma unroll
     for (int v = 0; v < kQNV; ++v) {
@@ -349,14 +357,16 @@ __global__ void __launch_bounds__(kQNT) quant_cta_kernel(const QuantArgs a, int 
         // multiples of 128 entries, so no word is shared with the next one)
         const int64_t chunk = 128 * (v * (kQNT / 32) + warp);
         if (chunk < nv) {
-          const uint64_t piece = codes4_any(xs, e0, nv, p, a.stochastic, a.seed,
-                                            static_cast<uint64_t>(row * L + c0 + e0), bits);
+          float u[4] = {0.f, 0.f, 0.f, 0.f};
+          if (SR) uniform4(a.seed, static_cast<uint64_t>(row * L + c0 + e0), u);
+          const uint64_t piece = codes4_any<SR>(xs, e0, nv, p, u, bits);
           const int64_t wend = min64(data_words, ((c0 + nv) * bits + 31) / 32);
           store_codes_any(piece, bits, lane, gbuf + warp * 64, cr, (c0 + chunk) * bits / 32, wend);
         }
       } else {
-        uint32_t piece = codes4<BITS>(xs, e0, nv, p, a.stochastic, a.seed,
-                                      static_cast<uint64_t>(row * L + c0 + e0));
+        float u[4] = {0.f, 0.f, 0.f, 0.f};
+        if (SR) uniform4(a.seed, static_cast<uint64_t>(row * L + c0 + e0), u);
+        uint32_t piece = codes4<BITS, SR>(xs, e0, nv, p, u);
         const bool store = assemble_word<BITS>(piece, lane);
         const int64_t w = (c0 + e0) * BITS / 32;
         if (store && e0 < nv && w < data_words) cr[w] = piece;
@@ -370,6 +380,7 @@ __global__ void __launch_bounds__(kQNT) quant_cta_kernel(const QuantArgs a, int 
 // launcher initialises to {0xffffffff, 0}).
 __global__ void __launch_bounds__(kQNT) quant_minmax_kernel(const float* x, int64_t L, int spr,
                                                             int64_t slice, uint32_t* mm) {
+  pdl_begin();
   const int64_t row = blockIdx.x / spr;
   const int64_t c0 = (blockIdx.x % spr) * slice;
   const int64_t n = max64(0, min64(slice, L - c0));
@@ -389,6 +400,7 @@ __global__ void __launch_bounds__(kQNT) quant_minmax_kernel(const float* x, int6
 }
 
 __global__ void minmax_init_kernel(uint32_t* mm, int64_t rows) {
+  pdl_begin();
   for (int64_t r = blockIdx.x * blockDim.x + threadIdx.x; r < rows;
        r += static_cast<int64_t>(gridDim.x) * blockDim.x) {
     mm[2 * r] = 0xffffffffu;
@@ -400,6 +412,7 @@ __global__ void minmax_init_kernel(uint32_t* mm, int64_t rows) {
 __global__ void passthrough_kernel(const float* __restrict__ x, int64_t rows, int64_t L,
                                    int64_t W, uint32_t* __restrict__ codes, float* scale,
                                    float* minv) {
+  pdl_begin();
   const int64_t total = rows * W;
   for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
        i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
@@ -420,6 +433,7 @@ __global__ void __launch_bounds__(256)
     dequant_kernel(const uint32_t* __restrict__ codes, const float* __restrict__ scale,
                    const float* __restrict__ minv, Index rows, int64_t L, int64_t W, Index wpr,
                    float* __restrict__ y, int aligned) {
+  pdl_begin();
   constexpr int PER = 32 / BITS;  // codes per word
   const Index total = rows * wpr;
   for (Index g = static_cast<Index>(blockIdx.x) * blockDim.x + threadIdx.x; g < total;
@@ -458,6 +472,7 @@ __global__ void __launch_bounds__(256)
     dequant_rows_kernel(const uint32_t* __restrict__ codes, const float* __restrict__ scale,
                         const float* __restrict__ minv, int64_t L, int64_t W, int bpr,
                         float* __restrict__ y) {
+  pdl_begin();
   const int64_t row = blockIdx.x / bpr;
   const int64_t f0 = static_cast<int64_t>(blockIdx.x % bpr) * (256 * kDqU);
   const int64_t n4 = L / 4;
@@ -490,6 +505,7 @@ __global__ void __launch_bounds__(256)
     dequant_rows_any_kernel(const uint32_t* __restrict__ codes, const float* __restrict__ scale,
                             const float* __restrict__ minv, int64_t L, int64_t W, int bpr,
                             int bits, float* __restrict__ y) {
+  pdl_begin();
   const int64_t row = blockIdx.x / bpr;
   const int64_t f0 = static_cast<int64_t>(blockIdx.x % bpr) * (256 * kDqU);
   const int64_t n4 = L / 4;
@@ -521,6 +537,7 @@ __global__ void __launch_bounds__(256)
 __global__ void dequant_any_kernel(const uint32_t* __restrict__ codes, const float* __restrict__ scale,
                                    const float* __restrict__ minv, int64_t rows, int64_t L,
                                    int64_t W, int bits, float* __restrict__ y) {
+  pdl_begin();
   const int64_t total = rows * L;
   const uint32_t mask = (1u << bits) - 1u;
   for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
@@ -545,8 +562,8 @@ void launch_dequant(const uint32_t* codes, const float* scale, const float* minv
   if (aligned && L % 4 == 0) {
     const int64_t bpr = (L / 4 + 256 * kDqU - 1) / (256 * kDqU);
     if (bpr > 0 && rows * bpr < 0x7fffffffLL) {
-      dequant_rows_kernel<BITS><<<static_cast<unsigned>(rows * bpr), 256, 0, s>>>(
-          codes, scale, minv, L, W, static_cast<int>(bpr), y);
+      launch_kernel(dequant_rows_kernel<BITS>, dim3(static_cast<unsigned>(rows * bpr)), dim3(256), 0,
+                    s, 0u, codes, scale, minv, L, W, static_cast<int>(bpr), y);
       return;
     }
   }
@@ -559,6 +576,7 @@ void launch_dequant(const uint32_t* codes, const float* scale, const float* minv
 
 __global__ void dequant_passthrough_kernel(const uint32_t* __restrict__ codes, int64_t rows,
                                            int64_t L, int64_t W, float* __restrict__ y) {
+  pdl_begin();
   const int64_t total = rows * L;
   for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
        i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
@@ -567,28 +585,28 @@ __global__ void dequant_passthrough_kernel(const uint32_t* __restrict__ codes, i
   }
 }
 
-template <int BITS, int NVW>
+template <int BITS, int NVW, bool SR>
 cudaError_t run_quant_warp(const QuantArgs& a, int num_sms, cudaStream_t s) {
-  auto kernel = quant_warp_kernel<BITS, NVW>;
+  auto kernel = quant_warp_kernel<BITS, NVW, SR>;
   const int occ = resident_blocks(kernel, 32 * kQWarps, 0);
   const int64_t want = (a.rows + kQWarps - 1) / kQWarps;
   const int64_t cap = static_cast<int64_t>(num_sms) * occ;
-  kernel<<<static_cast<unsigned>(want < cap ? want : cap), 32 * kQWarps, 0, s>>>(a);
-  return cudaGetLastError();
+  return launch_kernel(kernel, dim3(static_cast<unsigned>(want < cap ? want : cap)),
+                       dim3(32 * kQWarps), 0, s, 0u, a);
 }
 
-template <int BITS>
+template <int BITS, bool SR>
 cudaError_t run_quant_bits(const QuantArgs& a0, int num_sms, cudaStream_t s) {
   QuantArgs a = a0;
   const int64_t L = a.L;
   if (a.ws == nullptr && L <= 2048) {
-    if (L <= 256) return run_quant_warp<BITS, 2>(a, num_sms, s);
-    if (L <= 512) return run_quant_warp<BITS, 4>(a, num_sms, s);
-    if (L <= 768) return run_quant_warp<BITS, 6>(a, num_sms, s);
-    if (L <= 1024) return run_quant_warp<BITS, 8>(a, num_sms, s);
-    return run_quant_warp<BITS, 16>(a, num_sms, s);
+    if (L <= 256) return run_quant_warp<BITS, 2, SR>(a, num_sms, s);
+    if (L <= 512) return run_quant_warp<BITS, 4, SR>(a, num_sms, s);
+    if (L <= 768) return run_quant_warp<BITS, 6, SR>(a, num_sms, s);
+    if (L <= 1024) return run_quant_warp<BITS, 8, SR>(a, num_sms, s);
+    return run_quant_warp<BITS, 16, SR>(a, num_sms, s);
   }
-  auto kernel = quant_cta_kernel<BITS>;
+  auto kernel = quant_cta_kernel<BITS, SR>;
   const int smem = kQSCAP * 4;
   cudaError_t err = ensure_dynamic_smem(kernel, smem);
   if (err != cudaSuccess) return err;
@@ -609,19 +627,9 @@ cudaError_t run_quant_bits(const QuantArgs& a0, int num_sms, cudaStream_t s) {
   }
   const int64_t blocks = a.rows * spr;
   if (blocks > 0x7fffffffLL) return cudaErrorInvalidValue;
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(static_cast<unsigned>(blocks), 1, 1);
-  cfg.blockDim = dim3(kQNT, 1, 1);
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = s;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = (a.ws == nullptr) ? static_cast<unsigned>(spr) : 1u;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, kernel, a, static_cast<int>(spr));
+  return launch_kernel(kernel, dim3(static_cast<unsigned>(blocks)), dim3(kQNT), smem, s,
+                       (a.ws == nullptr) ? static_cast<unsigned>(spr) : 1u, a,
+                       static_cast<int>(spr));
 }
 
 unsigned grid_for(int64_t work, int num_sms) {
@@ -640,15 +648,20 @@ size_t quant_workspace_bytes(int64_t rows, int64_t L, int bits) {
 cudaError_t launch_quant_compress(const QuantArgs& a, int num_sms, cudaStream_t s) {
   if (a.rows <= 0) return cudaSuccess;
   switch (a.bits) {
-    case 2: return run_quant_bits<2>(a, num_sms, s);
-    case 4: return run_quant_bits<4>(a, num_sms, s);
-    case 8: return run_quant_bits<8>(a, num_sms, s);
+    case 2: return a.stochastic ? run_quant_bits<2, true>(a, num_sms, s)
+                                : run_quant_bits<2, false>(a, num_sms, s);
+    case 4: return a.stochastic ? run_quant_bits<4, true>(a, num_sms, s)
+                                : run_quant_bits<4, false>(a, num_sms, s);
+    case 8: return a.stochastic ? run_quant_bits<8, true>(a, num_sms, s)
+                                : run_quant_bits<8, false>(a, num_sms, s);
     case 32:
       passthrough_kernel<<<grid_for(a.rows * a.W, num_sms), 256, 0, s>>>(a.x, a.rows, a.L, a.W,
                                                                           a.codes, a.scale, a.minv);
       return cudaGetLastError();
     default:
-      if (a.bits >= 1 && a.bits <= 16) return run_quant_bits<0>(a, num_sms, s);
+      if (a.bits >= 1 && a.bits <= 16)
+        return a.stochastic ? run_quant_bits<0, true>(a, num_sms, s)
+                            : run_quant_bits<0, false>(a, num_sms, s);
       return cudaErrorInvalidValue;
   }
 }
@@ -676,8 +689,8 @@ cudaError_t launch_quant_decompress(const uint32_t* codes, const float* scale,
       if (bits < 1 || bits > 16) return cudaErrorInvalidValue;
       const int64_t bpr = (L / 4 + 256 * kDqU - 1) / (256 * kDqU);
       if (aligned && L % 4 == 0 && bpr > 0 && rows * bpr < 0x7fffffffLL)
-        dequant_rows_any_kernel<<<static_cast<unsigned>(rows * bpr), 256, 0, s>>>(
-            codes, scale, minv, L, W, static_cast<int>(bpr), bits, y);
+        launch_kernel(dequant_rows_any_kernel, dim3(static_cast<unsigned>(rows * bpr)), dim3(256),
+                      0, s, 0u, codes, scale, minv, L, W, static_cast<int>(bpr), bits, y);
       else
         dequant_any_kernel<<<grid_for(rows * L, num_sms), 256, 0, s>>>(codes, scale, minv, rows, L,
                                                                       W, bits, y);

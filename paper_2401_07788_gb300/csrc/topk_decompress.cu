@@ -47,6 +47,7 @@ __global__ void __launch_bounds__(kDecThreads)
     topk_decompress_kernel(const float* __restrict__ vals, const int32_t* __restrict__ idx,
                            int64_t rows, int64_t L, int64_t k, float* __restrict__ y,
                            int64_t rpc, int64_t tpr, int aligned) {
+  pdl_begin();
   extern __shared__ __align__(16) float tile[];  // kTile floats
   const int tid = threadIdx.x;
   const int64_t g = blockIdx.x;
@@ -105,6 +106,7 @@ __global__ void __launch_bounds__(kDecThreads)
     topk_decompress_rows_kernel(const float* __restrict__ vals, const int32_t* __restrict__ idx,
                                 int64_t rows, int64_t L, int64_t k, float* __restrict__ y,
                                 int64_t rpc, int64_t ppr, int aligned, int vec) {
+  pdl_begin();
   const int tid = threadIdx.x;
   int64_t r0, nrows, c0, ncols;
   if (ppr == 1) {
@@ -203,6 +205,7 @@ __global__ void __launch_bounds__(kDecThreads)
     topk_gather_kernel(const float* __restrict__ g, const int32_t* __restrict__ idx,
                        int64_t L, int64_t k, int bpr, float* __restrict__ vals, int vec,
                        unsigned* status) {
+  pdl_begin();
   const int64_t row = blockIdx.x / bpr;
   const int64_t q0 = static_cast<int64_t>(blockIdx.x % bpr) * (kDecThreads * kGU);
   const float* gr = g + row * L;
@@ -252,6 +255,7 @@ __global__ void __launch_bounds__(kDecThreads)
                             float* __restrict__ buf, int64_t num_samples,
                             const int64_t* __restrict__ ids, int64_t rps, int64_t L, int64_t k,
                             unsigned* status) {
+  pdl_begin();
   const int64_t lr = blockIdx.x;
   const int64_t sid = ids[lr / rps];
   if (sid < 0 || sid >= num_samples) {
@@ -287,9 +291,9 @@ cudaError_t launch_topk_decompress(const float* vals, const int32_t* idx, int64_
     // 16-byte payload loads when every block's payload range is 16-byte aligned
     const int vec = (k % 4 == 0) && (reinterpret_cast<uintptr_t>(vals) % 16 == 0) &&
                     (reinterpret_cast<uintptr_t>(idx) % 16 == 0);
-    topk_decompress_rows_kernel<<<static_cast<unsigned>(blocks), kDecThreads, 0, s>>>(
-        vals, idx, rows, L, k, y, rpc, ppr, aligned, vec);
-    return cudaGetLastError();
+    return launch_kernel(topk_decompress_rows_kernel, dim3(static_cast<unsigned>(blocks)),
+                         dim3(kDecThreads), 0, s, 0u, vals, idx, rows, L, k, y, rpc, ppr, aligned,
+                         vec);
   }
   int64_t rpc = 1, tpr = 1, blocks;
   if (L <= kTile) {
@@ -317,9 +321,9 @@ cudaError_t launch_topk_gather(const float* g, const int32_t* idx, int64_t rows,
   const int64_t per_block = static_cast<int64_t>(kDecThreads) * kGU * 4;
   const int64_t bpr = (k + per_block - 1) / per_block;
   if (rows * bpr > 0x7fffffffLL) return cudaErrorInvalidValue;
-  topk_gather_kernel<<<static_cast<unsigned>(rows * bpr), kDecThreads, 0, s>>>(
-      g, idx, L, k, static_cast<int>(bpr), vals, vec, status);
-  return cudaGetLastError();
+  return launch_kernel(topk_gather_kernel, dim3(static_cast<unsigned>(rows * bpr)),
+                       dim3(kDecThreads), 0, s, 0u, g, idx, L, k, static_cast<int>(bpr), vals, vec,
+                       status);
 }
 
 cudaError_t launch_aqsgd_decompress(const float* vals, const int32_t* idx, float* buf,

@@ -32,6 +32,7 @@ __device__ __forceinline__ void payload_block(int bpr, int64_t k, int64_t* row, 
 __global__ void __launch_bounds__(kT)
     efmix_mark_kernel(float* __restrict__ err, const int32_t* __restrict__ idx, int64_t L,
                       int64_t k, int bpr, float* __restrict__ saved, int restore) {
+  pdl_begin();
   int64_t row, i0;
   payload_block(bpr, k, &row, &i0);
   float* er = err + row * L;
@@ -54,6 +55,7 @@ __global__ void __launch_bounds__(kT)
 // when both are aligned and the count is a multiple of 4.
 __global__ void __launch_bounds__(kT)
     efmix_add_kernel(const float* __restrict__ x, float* __restrict__ err, int64_t n, int vec) {
+  pdl_begin();
   const int64_t stride = static_cast<int64_t>(gridDim.x) * kT;
   if (vec) {
     const int64_t n4 = n / 4;
@@ -76,6 +78,7 @@ __global__ void __launch_bounds__(kT)
 __global__ void __launch_bounds__(kT)
     efmix_send_kernel(float* __restrict__ err, const int32_t* __restrict__ idx, int64_t L,
                       int64_t k, int bpr, float* __restrict__ vals) {
+  pdl_begin();
   int64_t row, i0;
   payload_block(bpr, k, &row, &i0);
   float* er = err + row * L;

@@ -110,6 +110,7 @@ __device__ __forceinline__ uint32_t block_sum(uint32_t v, uint32_t* red) {
 }
 
 __global__ void g_init(GridMeta* meta, uint32_t* hist, int64_t nchunks) {
+  pdl_begin();
   for (int i = threadIdx.x; i < kGNB; i += blockDim.x) hist[i] = 0;
   if (threadIdx.x == 0) {
     GridMeta m = {};
@@ -123,6 +124,7 @@ __global__ void g_init(GridMeta* meta, uint32_t* hist, int64_t nchunks) {
 template <int MODE>
 __global__ void __launch_bounds__(kGT) g_sample(const float* xr, const float* ar, int64_t L,
                                                 int64_t k, GridMeta* meta) {
+  pdl_begin();
   __shared__ uint32_t red[kGT / 32];
   int mx = -1;
   for (int s = threadIdx.x; s < kSamples; s += kGT) {
@@ -156,6 +158,7 @@ __global__ void __launch_bounds__(kGT) g_sample(const float* xr, const float* ar
 template <int MODE>
 __global__ void __launch_bounds__(kGT) g_hist(const float* xr, float* ar, int64_t L,
                                               GridMeta* meta, uint32_t* hist, int first) {
+  pdl_begin();
   __shared__ uint32_t sh[kGNB];
   const GridMeta m = *meta;
   const bool bins = !m.resolved && m.m > kCandCap;
@@ -201,6 +204,7 @@ __device__ int first_key_of_bin(int b, float scale) {
 
 // Pick the bin holding the kr-th entry and narrow [lo, hi] to it.
 __global__ void __launch_bounds__(kGT) g_pick(GridMeta* meta, uint32_t* hist) {
+  pdl_begin();
   __shared__ uint32_t red[kGT / 32];
   __shared__ uint32_t pick_t, pick_excl;
   GridMeta m = *meta;
@@ -274,6 +278,7 @@ template <int MODE>
 __global__ void __launch_bounds__(kGT) g_count(const float* xr, const float* ar, int64_t L,
                                                GridMeta* meta, uint32_t* cgt, uint32_t* ceq,
                                                int* ckey, int64_t* cidx) {
+  pdl_begin();
   __shared__ uint32_t red[kGT / 32];
   const GridMeta m = *meta;
   const int64_t c0 = static_cast<int64_t>(blockIdx.x) * kCH;
@@ -307,6 +312,7 @@ __global__ void __launch_bounds__(kGT) g_count(const float* xr, const float* ar,
 // T and need from the candidate list (one CTA), then the candidates' chunks.
 __global__ void __launch_bounds__(1024) g_select(GridMeta* meta, uint32_t* cgt, uint32_t* ceq,
                                                  const int* ckey, const int64_t* cidx) {
+  pdl_begin();
   __shared__ uint32_t hist[kRoundBins];
   __shared__ int s_lo, s_hi, s_T;
   __shared__ uint32_t s_kr, s_need, s_done;
@@ -396,6 +402,7 @@ __device__ __forceinline__ uint32_t excl_scan_1024(uint32_t v, uint32_t* red, ui
 // written in place of the chunk's counts.
 __global__ void __launch_bounds__(1024) g_scan(const GridMeta* meta, uint32_t* cgt, uint32_t* ceq,
                                                int64_t nchunks) {
+  pdl_begin();
   __shared__ uint32_t red[32];
   const uint32_t need = meta->need;
   uint32_t carry_g = 0, carry_e = 0;  // identical in every thread
@@ -421,6 +428,7 @@ template <int MODE>
 __global__ void __launch_bounds__(kGT) g_write(const float* xr, float* ar, int64_t L, int64_t k,
                                                const GridMeta* meta, const uint32_t* cgt,
                                                const uint32_t* ceq, float* vals, int32_t* idx) {
+  pdl_begin();
   constexpr int NW = kGT / 32;
   __shared__ uint32_t ug[kGPT * NW], ue[kGPT * NW];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;

@@ -284,6 +284,7 @@ __device__ __forceinline__ void row_sync(uint32_t C) {
 
 template <int MODE, int NT, int SCAP, bool FULL>
 __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const TopkRowArgs a) {
+  pdl_begin();
   constexpr int NW = NT / 32;
   constexpr int NQ = SCAP / 4;     // float4 slots per slice
   constexpr int QPT = NQ / NT;     // float4 slots per thread
@@ -785,6 +786,7 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
   }
 
   // ---- write the payload (ascending column) and the buffers -----------------
+  pdl_end();
   float* vrow = a.vals + row * k;
   int32_t* irow = a.idx + row * k;
   const uint32_t kk32 = static_cast<uint32_t>(min64(k, 0x7fffffff));
@@ -905,6 +907,7 @@ __device__ __forceinline__ float* state_row(const TopkRowArgs& a, int64_t row, b
 
 template <int MODE, int NVW, int WPC, bool FULL>
 __global__ void __launch_bounds__(32 * WPC) topk_warp_kernel(const TopkRowArgs a) {
+  pdl_begin();
   constexpr int RCAP = 128 * NVW;
   constexpr int NBUF = (MODE == kPlain) ? 1 : 2;  // x (+ err / state) per row
   __shared__ WarpShared wsh[WPC];
@@ -1210,8 +1213,7 @@ cudaError_t run_warp(const TopkRowArgs& a, int num_sms, cudaStream_t s) {
   const int64_t want = (a.rows + WPC - 1) / WPC;
   const int64_t cap = static_cast<int64_t>(num_sms) * occ;
   const int blocks = static_cast<int>(want < cap ? want : cap);
-  kernel<<<blocks, 32 * WPC, smem, s>>>(a);
-  return cudaGetLastError();
+  return launch_kernel(kernel, dim3(blocks), dim3(32 * WPC), smem, s, 0u, a);
 }
 
 template <int MODE, int NVW>
@@ -1226,19 +1228,8 @@ cudaError_t run_cta(const TopkRowArgs& a, int C, cudaStream_t s) {
   const int smem = cta_smem_bytes(NT, SCAP, C);
   cudaError_t err = ensure_dynamic_smem(kernel, cta_smem_bytes(NT, SCAP, kMaxCluster));
   if (err != cudaSuccess) return err;
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(static_cast<unsigned>(a.rows * C), 1, 1);
-  cfg.blockDim = dim3(NT, 1, 1);
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = s;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = C;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, kernel, a);
+  return launch_kernel(kernel, dim3(static_cast<unsigned>(a.rows * C)), dim3(NT), smem, s,
+                       static_cast<unsigned>(C), a);
 }
 
 // FULL when every CTA's slice is a whole number of NT x 4-entry slots.
