@@ -78,6 +78,13 @@ def load(path: str | None = None) -> ctypes.CDLL:
                                            ctypes.c_uint64, _U32P, _F32P, _F32P]
         lib.orc_quant_decompress.argtypes = [_U32P, _F32P, _F32P, _i64, _i64, ctypes.c_int,
                                              _F32P]
+        lib.orc_aqsgd_quant_compress.argtypes = [_F32P, _F32P, _i64, _I64P, _i64, _i64, _i64,
+                                                 ctypes.c_int, ctypes.c_int, ctypes.c_uint64,
+                                                 _U32P, _F32P, _F32P]
+        lib.orc_aqsgd_quant_decompress.argtypes = [_U32P, _F32P, _F32P, _F32P, _i64, _I64P, _i64,
+                                                   _i64, _i64, ctypes.c_int]
+        for name in ("orc_aqsgd_quant_compress", "orc_aqsgd_quant_decompress"):
+            getattr(lib, name).restype = None
         for name in ("orc_topk_compress", "orc_topk_decompress", "orc_topk_gather",
                      "orc_ef_topk_compress", "orc_efmix_topk_compress",
                      "orc_ef21_topk_compress", "orc_aqsgd_compress", "orc_aqsgd_decompress",
@@ -223,3 +230,34 @@ def quant_decompress(codes, scale, minv, row_len: int, bits: int, lib=None):
     y = np.empty((R, row_len), np.float32)
     (lib or load()).orc_quant_decompress(codes, scale, minv, R, row_len, bits, y)
     return y
+
+
+def aqsgd_quant_compress(x, buf, sample_ids, bits: int, stochastic: bool = False, seed: int = 0,
+                         lib=None):
+    """AQ-SGD with quantisation (§2.5). x [n_ids, rps, L]; buf [S, rps, L] updated in place.
+    Returns (codes, scale, minv) of the gathered rows."""
+    x = _f32(x)
+    assert buf.dtype == np.float32 and buf.flags.c_contiguous
+    ids = np.ascontiguousarray(sample_ids, dtype=np.int64)
+    n_ids = ids.shape[0]
+    S, rps, L = buf.shape
+    assert x.shape == (n_ids, rps, L)
+    lib = lib or load()
+    R = n_ids * rps
+    W = quant_row_words(L, bits, lib)
+    codes = np.zeros((R, W), np.uint32)
+    scale = np.empty(R, np.float32)
+    minv = np.empty(R, np.float32)
+    lib.orc_aqsgd_quant_compress(x, buf, S, ids, n_ids, rps, L, bits, 1 if stochastic else 0,
+                                 seed, codes, scale, minv)
+    return codes, scale, minv
+
+
+def aqsgd_quant_decompress(codes, scale, minv, buf_recv, sample_ids, bits: int, lib=None):
+    ids = np.ascontiguousarray(sample_ids, dtype=np.int64)
+    S, rps, L = buf_recv.shape
+    assert buf_recv.dtype == np.float32 and buf_recv.flags.c_contiguous
+    (lib or load()).orc_aqsgd_quant_decompress(
+        np.ascontiguousarray(codes, dtype=np.uint32), _f32(scale), _f32(minv), buf_recv, S, ids,
+        ids.shape[0], rps, L, bits)
+    return buf_recv

@@ -385,3 +385,56 @@ void orc_quant_decompress(const uint32_t* codes, const float* scale, const float
         }
     }
 }
+
+/* AQ-SGD with quantisation, §2.5 (the cited work compresses the change of the
+ * activations by quantisation; the section applies the same scheme with
+ * TopK): for each listed sample id and row, d = x - buf[id, r], the message is
+ * Quant(d) (§2.2, the quantiser above on the gathered rows, logical row i * rps
+ * + r), and buf[id, r] <- buf[id, r] + Dequant(Quant(d)). */
+void orc_aqsgd_quant_compress(const float* x, float* buf, int64_t num_samples,
+                              const int64_t* sample_ids, int64_t n_ids,
+                              int64_t rows_per_sample, int64_t row_len, int bits, int mode,
+                              uint64_t seed, uint32_t* codes, float* scale, float* minv)
+{
+    (void)num_samples;
+    const int64_t rows = n_ids * rows_per_sample;
+    float* d = (float*)malloc(sizeof(float) * (size_t)(rows * row_len));
+    float* dh = (float*)malloc(sizeof(float) * (size_t)(rows * row_len));
+    for (int64_t i = 0; i < n_ids; ++i)
+        for (int64_t r = 0; r < rows_per_sample; ++r) {
+            const int64_t logical = i * rows_per_sample + r;
+            const float* br = buf + (sample_ids[i] * rows_per_sample + r) * row_len;
+            for (int64_t j = 0; j < row_len; ++j)
+                d[logical * row_len + j] = x[logical * row_len + j] - br[j];
+        }
+    orc_quant_compress(d, rows, row_len, bits, mode, seed, codes, scale, minv);
+    orc_quant_decompress(codes, scale, minv, rows, row_len, bits, dh);
+    for (int64_t i = 0; i < n_ids; ++i)
+        for (int64_t r = 0; r < rows_per_sample; ++r) {
+            const int64_t logical = i * rows_per_sample + r;
+            float* br = buf + (sample_ids[i] * rows_per_sample + r) * row_len;
+            for (int64_t j = 0; j < row_len; ++j) br[j] = br[j] + dh[logical * row_len + j];
+        }
+    free(dh);
+    free(d);
+}
+
+/* The receiver's side: buf_recv[id, r] <- buf_recv[id, r] + Dequant(codes of the
+ * logical row), which it then uses as the activation. */
+void orc_aqsgd_quant_decompress(const uint32_t* codes, const float* scale, const float* minv,
+                                float* buf_recv, int64_t num_samples,
+                                const int64_t* sample_ids, int64_t n_ids,
+                                int64_t rows_per_sample, int64_t row_len, int bits)
+{
+    (void)num_samples;
+    const int64_t rows = n_ids * rows_per_sample;
+    float* dh = (float*)malloc(sizeof(float) * (size_t)(rows * row_len));
+    orc_quant_decompress(codes, scale, minv, rows, row_len, bits, dh);
+    for (int64_t i = 0; i < n_ids; ++i)
+        for (int64_t r = 0; r < rows_per_sample; ++r) {
+            const int64_t logical = i * rows_per_sample + r;
+            float* br = buf_recv + (sample_ids[i] * rows_per_sample + r) * row_len;
+            for (int64_t j = 0; j < row_len; ++j) br[j] = br[j] + dh[logical * row_len + j];
+        }
+    free(dh);
+}

@@ -78,6 +78,18 @@ void orc_quant_compress(const float* x, int64_t rows, int64_t row_len, int bits,
 void orc_quant_decompress(const uint32_t* codes, const float* scale, const float* minv,
                           int64_t rows, int64_t row_len, int bits, float* y);
 
+/* AQ-SGD with quantisation, §2.5: d = x - buf[id, r]; message Quant(d);
+ * buf[id, r] <- buf[id, r] + Dequant(Quant(d)).  Codes as orc_quant_compress
+ * on the gathered rows (logical row i * rows_per_sample + r). */
+void orc_aqsgd_quant_compress(const float* x, float* buf, int64_t num_samples,
+                              const int64_t* sample_ids, int64_t n_ids,
+                              int64_t rows_per_sample, int64_t row_len, int bits, int mode,
+                              uint64_t seed, uint32_t* codes, float* scale, float* minv);
+void orc_aqsgd_quant_decompress(const uint32_t* codes, const float* scale, const float* minv,
+                                float* buf_recv, int64_t num_samples,
+                                const int64_t* sample_ids, int64_t n_ids,
+                                int64_t rows_per_sample, int64_t row_len, int bits);
+
 #ifdef __cplusplus
 }
 #endif

@@ -425,4 +425,37 @@ def pin_quant_stochastic(lib, seed: int = 13, n_seeds: int = 10000):
     assert np.array_equal(a, b) and not np.array_equal(a, d)
 
 
+def pin_aqsgd_quant(lib, seed: int = 16):
+    """AQ-SGD with quantisation (§2.5): the stored rows take exactly the dequantised
+    message (the same fp32 add), untouched samples stay bit-identical, the receiver's
+    copy follows bit for bit; with an empty buffer the message is the plain quantisation
+    of x; and the codes are those of the quantiser applied to x - buf, read back with
+    numpy from the bitstream."""
+    rng = np.random.default_rng(seed)
+    S, rps, L = 9, 2, 100
+    buf = rng.standard_normal((S, rps, L)).astype(np.float32)
+    before = buf.copy()
+    recv = buf.copy()
+    ids = np.array([4, 0, 7], np.int64)
+    x = rng.standard_normal((3, rps, L)).astype(np.float32)
+    for bits, sr in ((4, False), (6, True), (2, True)):
+        b0 = buf.copy()
+        c, s, m = oracle.aqsgd_quant_compress(x, buf, ids, bits, sr, 11, lib)
+        d = (x - b0[ids]).reshape(3 * rps, L)
+        c2, s2, m2 = oracle.quant_compress(d, bits, sr, 11, lib)
+        assert np.array_equal(c, c2) and np.array_equal(bits_of(s), bits_of(s2))
+        dh = oracle.quant_decompress(c, s, m, L, bits, lib).reshape(3, rps, L)
+        assert np.array_equal(bits_of(buf[ids]), bits_of(b0[ids] + dh))
+        untouched = np.setdiff1d(np.arange(S), ids)
+        assert np.array_equal(bits_of(buf[untouched]), bits_of(before[untouched]))
+        oracle.aqsgd_quant_decompress(c, s, m, recv, ids, bits, lib)
+        assert np.array_equal(bits_of(recv), bits_of(buf))
+    zero = np.zeros((S, rps, L), np.float32)
+    c, s, m = oracle.aqsgd_quant_compress(x, zero, ids, 8, False, 0, lib)
+    c2, s2, m2 = oracle.quant_compress(x.reshape(3 * rps, L), 8, False, 0, lib)
+    assert np.array_equal(c, c2) and np.array_equal(bits_of(m), bits_of(m2))
+    q = stream_codes(c[0], 8, L)
+    assert q.min() >= 0 and q.max() == 255
+
+
 ALL_PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_")]

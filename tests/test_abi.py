@@ -104,3 +104,6 @@ def test_knobs(lib):
     assert lib.mpc_set_knob(99, 0) == 1
     assert lib.mpc_set_knob(2, 5) == 1
     assert lib.mpc_set_knob(2, 0) == 0
+    assert lib.mpc_set_knob(3, 2) == 1  # programmatic dependent launch: 0 or 1
+    assert lib.mpc_set_knob(3, 0) == 0
+    assert lib.mpc_set_knob(3, 1) == 0

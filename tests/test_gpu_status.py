@@ -50,3 +50,36 @@ def test_timeout_is_reported_and_context_survives(mpc, op, L):
     assert mpc.mpc_get_status() == 0
     assert_bits_equal(i.cpu().numpy(), oi, "idx after timeout")
     assert_bits_equal(v.cpu().numpy(), ov, "vals after timeout")
+
+
+def test_results_do_not_depend_on_dependent_launch(mpc):
+    """The same sequence of dependent calls (error feedback carried across steps, then
+    decompression and quantisation of the result) gives the same bits with programmatic
+    dependent launch on and off."""
+    import numpy as np
+
+    def run():
+        torch.manual_seed(0)
+        x = torch.randn(64, 32768, device="cuda")
+        e = torch.zeros_like(x)
+        outs = []
+        for _ in range(3):
+            v, i = mpc.mpc_ef_topk_compress(x, e, 3276)
+            y = mpc.mpc_topk_decompress(v, i, 32768)
+            c, s, m = mpc.mpc_quant_compress(y, 4, stochastic=True, seed=5)
+            outs += [v, i, e.clone(), mpc.mpc_quant_decompress(c, s, m, 32768, 4)]
+            x = x + 0.1
+        torch.cuda.synchronize()
+        return [o.cpu().numpy() for o in outs]
+
+    try:
+        mpc.mpc_set_knob(mpc.MPC_KNOB_PDL, 1)
+        a = run()
+        mpc.mpc_set_knob(mpc.MPC_KNOB_PDL, 0)
+        b = run()
+    finally:
+        mpc.mpc_set_knob(mpc.MPC_KNOB_PDL, 1)
+    for p, q in zip(a, b):
+        assert np.array_equal(p.view(np.uint32) if p.dtype.itemsize == 4 else p,
+                              q.view(np.uint32) if q.dtype.itemsize == 4 else q)
+    assert mpc.mpc_get_status() == 0

@@ -43,6 +43,10 @@ MUTANTS = {
     "efmix_buffer_share_from_input": ("work[m].mag = fabsf(er[j]);", "work[m].mag = fabsf(xr[j]);"),
     "efmix_shares_overlap": ("            if (!taken[j]) {\n                work[m].mag",
                              "            if (1) {\n                work[m].mag"),
+    "aqsgd_quant_delta_transposed": ("d[logical * row_len + j] = x[logical * row_len + j] - br[j];",
+                                     "d[logical * row_len + j] = br[j] - x[logical * row_len + j];"),
+    "aqsgd_quant_update_dropped": ("for (int64_t j = 0; j < row_len; ++j) br[j] = br[j] + dh[logical * row_len + j];\n        }\n    free(dh);\n    free(d);",
+                                   "for (int64_t j = 0; j < row_len; ++j) br[j] = dh[logical * row_len + j];\n        }\n    free(dh);\n    free(d);"),
     "gather_row_offset_dropped": ("vals[r * k + i] = g[r * row_len + idx[r * k + i]];",
                                   "vals[r * k + i] = g[idx[r * k + i]];"),
 }
