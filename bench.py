@@ -284,6 +284,10 @@ def algorithmic_bytes(R_, L_, k=None, bits=None, op=""):
         return 12 * k * R_
     if op == "aqsgd_decompress":
         return 8 * k * R_ + 8 * k * R_
+    if op == "aqsgd_quant":  # x and buffer rows read, buffer rows and codes written
+        return 12 * N + (N * bits + 7) // 8 + 8 * R_
+    if op == "aqsgd_dequant_add":  # codes and buffer rows read, buffer rows written
+        return 8 * N + (N * bits + 7) // 8 + 8 * R_
     if op in ("quant", "dequant"):
         return 4 * N + (N * bits + 7) // 8 + 8 * R_
     raise ValueError(op)
@@ -664,7 +668,15 @@ def measure_operators(mpc, synth, device, stream, peak):
         algorithmic_bytes(16 * rps, La, k=ka, op="delta_topk"))
     rec("aqsgd_decompress 16x512x1024 K=30%", time_op(lambda: mpc.mpc_aqsgd_decompress(va, ia, buf, ids), stream, flush),
         algorithmic_bytes(16 * rps, La, k=ka, op="aqsgd_decompress"))
-    del buf, xa
+    # the same boundary with 4-bit quantisation of the change (§2.5 with §2.2's quantiser)
+    wsq = torch.empty(mpc.mpc_aqsgd_quant_workspace_bytes(16, rps, La, 4), dtype=torch.uint8,
+                      device=device)
+    cqa, sqa, mqa = mpc.mpc_aqsgd_quant_compress(xa, buf, ids, 4, ws=wsq)
+    rec("aqsgd_quant_compress 16x512x1024 4-bit", time_op(lambda: mpc.mpc_aqsgd_quant_compress(xa, buf, ids, 4, codes=cqa, scale=sqa, minv=mqa, ws=wsq), stream, flush),
+        algorithmic_bytes(16 * rps, La, bits=4, op="aqsgd_quant"))
+    rec("aqsgd_quant_decompress 16x512x1024 4-bit", time_op(lambda: mpc.mpc_aqsgd_quant_decompress(cqa, sqa, mqa, buf, ids, 4), stream, flush),
+        algorithmic_bytes(16 * rps, La, bits=4, op="aqsgd_dequant_add"))
+    del buf, xa, wsq
     torch.cuda.empty_cache()
     # bandwidth sweep point: one 1 GiB tensor
     N = 1 << 28

@@ -218,6 +218,43 @@ mpc_status mpc_quant_decompress(const uint32_t* codes, const float* scale,
                                 const float* minv, int64_t rows, int64_t row_len, int bits,
                                 float* y, mpc_stream_t stream);
 
+/* AQ-SGD with quantisation (§2.5: the change of each training sample's
+ * activation against a buffer kept per sample is what travels; the cited work
+ * compresses that change with the quantiser of §2.2):
+ *   for i < n_ids, r < rows_per_sample, with s = sample_ids[i] and logical row
+ *   l = i*rows_per_sample + r:
+ *     d = x[i][r] - buf[s][r];  codes/scale/minv row l = Quant(d) exactly as
+ *     mpc_quant_compress on the [n_ids*rows_per_sample][row_len] rows of d
+ *     (the same seed gives the same stochastic draws);
+ *     buf[s][r] <- buf[s][r] + Dequant(row l)   (fp32 round to nearest).
+ *   x          [n_ids][rows_per_sample][row_len] fp32.
+ *   buf        [num_samples][rows_per_sample][row_len] fp32, in place.
+ *   sample_ids device int64[n_ids], each in [0, num_samples), no duplicates
+ *              (duplicates race; an id out of range sets MPC_ERR_DEVICE, its
+ *              d rows are taken as zero and its buffer rows are left alone).
+ *   bits, mode as mpc_quant_compress; codes, scale, minv out as there.
+ *   ws         device workspace of mpc_aqsgd_quant_workspace_bytes() bytes,
+ *              8-byte aligned (always needed: it holds d).
+ * Three launches (d, the quantiser, the buffer update), stream-ordered. */
+size_t mpc_aqsgd_quant_workspace_bytes(int64_t n_ids, int64_t rows_per_sample,
+                                       int64_t row_len, int bits);
+mpc_status mpc_aqsgd_quant_compress(const float* x, float* buf, int64_t num_samples,
+                                    const int64_t* sample_ids, int64_t n_ids,
+                                    int64_t rows_per_sample, int64_t row_len, int bits,
+                                    mpc_rounding mode, uint64_t seed, uint32_t* codes,
+                                    float* scale, float* minv, void* ws, size_t ws_bytes,
+                                    mpc_stream_t stream);
+
+/* AQ-SGD with quantisation, the receiver: its copy of the buffer takes the
+ * same update, buf_recv[s][r] <- buf_recv[s][r] + Dequant(row l), with the
+ * sender's fp32 operations, so the two copies stay bit-identical.  Shapes and
+ * id rules as mpc_aqsgd_quant_compress. */
+mpc_status mpc_aqsgd_quant_decompress(const uint32_t* codes, const float* scale,
+                                      const float* minv, float* buf_recv, int64_t num_samples,
+                                      const int64_t* sample_ids, int64_t n_ids,
+                                      int64_t rows_per_sample, int64_t row_len, int bits,
+                                      mpc_stream_t stream);
+
 /* Quantise without allocating (the paper has no counterpart; this is a
  * deployment convenience).  Same operation, arguments and results as
  * mpc_quant_compress, bit for bit, but with no workspace argument: for callers

@@ -24,7 +24,8 @@ __all__ = [
     "mpc_topk_gather", "mpc_efmix_workspace_bytes", "mpc_efmix_topk_compress",
     "mpc_ef_topk_compress", "mpc_ef21_topk_compress", "mpc_aqsgd_compress",
     "mpc_aqsgd_decompress", "mpc_quant_codes_words", "mpc_quant_workspace_bytes",
-    "mpc_quant_compress", "mpc_quant_decompress", "mpc_get_status", "mpc_last_error",
+    "mpc_quant_compress", "mpc_quant_decompress", "mpc_aqsgd_quant_workspace_bytes",
+    "mpc_aqsgd_quant_compress", "mpc_aqsgd_quant_decompress", "mpc_get_status", "mpc_last_error",
     "mpc_set_knob", "MPC_KNOB_SPIN_LIMIT", "MPC_KNOB_TOPK_PATH", "MPC_KNOB_PDL", "STATUS_NAMES",
 ]
 
@@ -59,6 +60,11 @@ _SIGNATURES = {
     "mpc_quant_compress": ([_VP, _I64, _I64, _INT, _INT, _U64, _VP, _VP, _VP, _VP, _SZ, _VP],
                            _INT),
     "mpc_quant_decompress": ([_VP, _VP, _VP, _I64, _I64, _INT, _VP, _VP], _INT),
+    "mpc_aqsgd_quant_workspace_bytes": ([_I64, _I64, _I64, _INT], _SZ),
+    "mpc_aqsgd_quant_compress": ([_VP, _VP, _I64, _VP, _I64, _I64, _I64, _INT, _INT, _U64, _VP,
+                                  _VP, _VP, _VP, _SZ, _VP], _INT),
+    "mpc_aqsgd_quant_decompress": ([_VP, _VP, _VP, _VP, _I64, _VP, _I64, _I64, _I64, _INT, _VP],
+                                   _INT),
     "mpc_quant_compress_noalloc": ([_VP, _I64, _I64, _INT, _INT, _U64, _VP, _VP, _VP, _VP],
                                    _INT),
     "mpc_get_status": ([_VP], _INT),
@@ -327,6 +333,69 @@ def mpc_quant_decompress(codes, scale, minv, row_len: int, bits: int, y=None, st
     _check(lib().mpc_quant_decompress(_ptr(codes), _ptr(scale), _ptr(minv), R, row_len, bits,
                                       _ptr(y), _stream(stream)))
     return y
+
+
+def mpc_aqsgd_quant_workspace_bytes(n_ids: int, rows_per_sample: int, row_len: int,
+                                    bits: int) -> int:
+    return int(lib().mpc_aqsgd_quant_workspace_bytes(n_ids, rows_per_sample, row_len, bits))
+
+
+def _aqsgd_shapes(x_shape, buf, sample_ids):
+    if buf.dim() != 3:
+        raise MpcError(1, "buf must be [num_samples, rps, L]")
+    S, rps, L = buf.shape
+    n_ids = sample_ids.numel()
+    if x_shape is not None and tuple(x_shape) != (n_ids, rps, L):
+        raise MpcError(1, "x must be [n_ids, rps, L] with buf [num_samples, rps, L]")
+    return S, rps, L, n_ids
+
+
+def mpc_aqsgd_quant_compress(x, buf, sample_ids, bits: int, stochastic: bool = False,
+                             seed: int = 0, codes=None, scale=None, minv=None, ws=None,
+                             stream=None):
+    """AQ-SGD with quantisation (§2.5). x [n_ids, rps, L]; buf [num_samples, rps, L]
+    updated in place; returns (codes [R, W] int32 of uint32 words, scale [R], minv [R])
+    with R = n_ids * rps."""
+    _cuda(x, torch.float32, "x")
+    _cuda(buf, torch.float32, "buf")
+    _cuda(sample_ids, torch.int64, "sample_ids")
+    S, rps, L, n_ids = _aqsgd_shapes(x.shape, buf, sample_ids)
+    R = n_ids * rps
+    words = mpc_quant_codes_words(R, L, bits)
+    if words == 0 and R > 0:
+        raise MpcError(1, "bits=%d is not supported" % bits)
+    W = words // R if R else 0
+    if codes is None:
+        codes = torch.empty((R, W), dtype=torch.int32, device=x.device)
+    if scale is None:
+        scale = torch.empty(R, dtype=torch.float32, device=x.device)
+    if minv is None:
+        minv = torch.empty(R, dtype=torch.float32, device=x.device)
+    _cuda(codes, torch.int32, "codes")
+    _cuda(scale, torch.float32, "scale")
+    _cuda(minv, torch.float32, "minv")
+    need = mpc_aqsgd_quant_workspace_bytes(n_ids, rps, L, bits) if R else 0
+    ws, wsb = _workspace(need, ws, x.device)
+    _check(lib().mpc_aqsgd_quant_compress(_ptr(x), _ptr(buf), S, _ptr(sample_ids), n_ids, rps,
+                                          L, bits, 1 if stochastic else 0,
+                                          seed & 0xFFFFFFFFFFFFFFFF, _ptr(codes), _ptr(scale),
+                                          _ptr(minv), _ptr(ws), wsb, _stream(stream)))
+    return codes, scale, minv
+
+
+def mpc_aqsgd_quant_decompress(codes, scale, minv, buf_recv, sample_ids, bits: int,
+                               stream=None):
+    """Receiver: buf_recv[ids] += Dequant(codes) (in place)."""
+    _cuda(codes, torch.int32, "codes")
+    _cuda(scale, torch.float32, "scale")
+    _cuda(minv, torch.float32, "minv")
+    _cuda(buf_recv, torch.float32, "buf_recv")
+    _cuda(sample_ids, torch.int64, "sample_ids")
+    S, rps, L, n_ids = _aqsgd_shapes(None, buf_recv, sample_ids)
+    _check(lib().mpc_aqsgd_quant_decompress(_ptr(codes), _ptr(scale), _ptr(minv),
+                                            _ptr(buf_recv), S, _ptr(sample_ids), n_ids, rps,
+                                            L, bits, _stream(stream)))
+    return buf_recv
 
 
 # ---------------------------------------------------------------------------------------

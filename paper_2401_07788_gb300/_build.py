@@ -17,7 +17,8 @@ OUT_DIR = os.path.join(PKG, "_build")
 LIB_PATH = os.path.join(OUT_DIR, "libmpcomp.so")
 
 SOURCES = ["abi.cu", "topk_rows.cu", "topk_rows_plain.cu", "topk_rows_ef.cu", "topk_rows_delta.cu",
-           "topk_grid.cu", "topk_decompress.cu", "topk_efmix.cu", "quant.cu"]
+           "topk_grid.cu", "topk_decompress.cu", "topk_efmix.cu", "quant.cu",
+           "aqsgd_quant.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 # -fmad=false: no multiply-add contraction anywhere; the order-critical lines
 # also use the explicit round-to-nearest intrinsics.

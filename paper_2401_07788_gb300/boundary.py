@@ -7,12 +7,15 @@ exchange compressed messages.
 output is the decompressed activation (what the next stage receives); its backward
 returns the decompressed gradient (what the previous stage receives).  Every compression
 step runs in the library's kernels through the ``mpc_*`` calls; this module only reshapes
-tensors into rows, keeps the feedback state between steps and routes the calls.
+tensors into rows, keeps the feedback state between steps, routes the calls and reads the
+reconstruction out of the feedback buffer.
 
 Compressors (the operators of §2.2 - §2.5):
 
-* ``Quant(bits, stochastic)``  min-max quantisation to 2^bits levels (§2.2), bits 1..16
-  (the paper uses 2, 4, 6, 8), round to nearest or stochastic.
+* ``Quant(bits, stochastic, feedback)``  min-max quantisation to 2^bits levels (§2.2),
+  bits 1..16 (the paper uses 2, 4, 6, 8), round to nearest or stochastic; ``feedback``
+  ``"aqsgd"`` quantises the change against a buffer kept per training sample, as the work
+  §2.5 cites does.
 * ``TopK(percent, feedback)``  TopK of §2.3, optionally with error feedback (§2.4):
   ``"none"``, ``"ef"`` (Seide: one global error buffer), ``"ef21"`` (the previously sent
   value), ``"aqsgd"`` (§2.5: one buffer per training sample; ``forward`` then takes the
@@ -20,6 +23,11 @@ Compressors (the operators of §2.2 - §2.5):
 * ``Reuse()`` (gradients only): the gradient is sent at the indices the activation's TopK
   kept (§3.2, Table 5, which fine-tuning needs to converge).
 * ``None``: no compression in that direction.
+
+What the next stage receives: the decompressed message for plain compression and for EF
+(the receiver has no buffer of its own); the receiver's reconstruction for EF21 (its copy
+of ``g``) and AQ-SGD (its copy of the sample's buffer rows), which equals the sender's
+buffer after the update since both take the same fp32 additions.
 
 Rows: ``rows="sample"`` treats each sample (all dims but the first) as one row, as for the
 CNN boundaries; ``rows="last"`` treats the last dimension as the row (one token of a
@@ -37,9 +45,9 @@ from dataclasses import dataclass
 
 import torch
 
-from . import (mpc_aqsgd_compress, mpc_ef21_topk_compress, mpc_ef_topk_compress,
-               mpc_quant_compress, mpc_quant_decompress, mpc_topk_compress,
-               mpc_topk_decompress, mpc_topk_gather)
+from . import (mpc_aqsgd_compress, mpc_aqsgd_quant_compress, mpc_ef21_topk_compress,
+               mpc_ef_topk_compress, mpc_quant_compress, mpc_quant_decompress,
+               mpc_topk_compress, mpc_topk_decompress, mpc_topk_gather)
 from .synth import k_of
 
 __all__ = ["Quant", "TopK", "Reuse", "CompressionBoundary", "with_boundaries"]
@@ -49,6 +57,11 @@ __all__ = ["Quant", "TopK", "Reuse", "CompressionBoundary", "with_boundaries"]
 class Quant:
     bits: int
     stochastic: bool = False
+    feedback: str = "none"  # "none" | "aqsgd"
+
+    def __post_init__(self):
+        if self.feedback not in ("none", "aqsgd"):
+            raise ValueError("quantisation feedback must be none or aqsgd")
 
 
 @dataclass(frozen=True)
@@ -99,9 +112,9 @@ class CompressionBoundary(torch.nn.Module):
             raise ValueError("Reuse() compresses gradients only")
         if isinstance(backward, Reuse) and not isinstance(forward, TopK):
             raise ValueError("Reuse() needs a TopK forward compressor")
-        if isinstance(backward, TopK) and backward.feedback != "none":
+        if isinstance(backward, (TopK, Quant)) and backward.feedback != "none":
             raise ValueError("feedback applies to the forward (activation) compressor")
-        if isinstance(forward, TopK) and forward.feedback == "aqsgd" and aqsgd_samples < 1:
+        if getattr(forward, "feedback", None) == "aqsgd" and aqsgd_samples < 1:
             raise ValueError("AQ-SGD needs aqsgd_samples, the number of training samples")
         self.fw = forward
         self.bw = backward
@@ -139,11 +152,13 @@ class CompressionBoundary(torch.nn.Module):
         r = _as_rows(x.detach(), self.rows)
         R, L = r.shape
         idx = None
-        if isinstance(c, Quant):
+        fb = c.feedback if self.training else "none"
+        if fb == "aqsgd":
+            y, idx = self._aqsgd(r, c, sample_ids)
+        elif isinstance(c, Quant):
             y = self._quant(r, c, 0)
         else:
             k = k_of(L, c.percent)
-            fb = c.feedback if self.training else "none"
             if fb == "none":
                 vals, idx = mpc_topk_compress(r, k)
             elif fb == "ef":
@@ -154,24 +169,36 @@ class CompressionBoundary(torch.nn.Module):
                 if self.state is None or self.state.shape != r.shape:
                     self.state = torch.zeros_like(r)
                 vals, idx = mpc_ef21_topk_compress(r, self.state, k)
-            else:  # aqsgd
-                if sample_ids is None:
-                    raise ValueError("AQ-SGD needs the batch's sample ids")
-                ids = sample_ids.to(device=r.device, dtype=torch.int64).contiguous()
-                if R % ids.numel():
-                    raise ValueError("rows must split evenly over the sample ids")
-                rps = R // ids.numel()
-                shape = (self.aqsgd_samples, rps, L)
-                if self.state is None or tuple(self.state.shape) != shape:
-                    self.state = torch.zeros(shape, device=r.device)
-                vals, idx = mpc_aqsgd_compress(r.reshape(ids.numel(), rps, L), self.state,
-                                               ids, k)
-                vals = vals.reshape(R, k)
-                idx = idx.reshape(R, k)
-            y = mpc_topk_decompress(vals, idx, L)
+            if fb == "ef21":
+                y = self.state.clone()  # the receiver's g' = g + C(x - g)
+            else:
+                y = mpc_topk_decompress(vals, idx, L)
         if self.training:
             self.step += 1
         return y.reshape(x.shape), idx
+
+    def _aqsgd(self, r: torch.Tensor, c, sample_ids):
+        """AQ-SGD (§2.5): the change against the samples' buffer rows is compressed and
+        both copies of the buffer take it; the next stage receives the updated rows."""
+        if sample_ids is None:
+            raise ValueError("AQ-SGD needs the batch's sample ids")
+        R, L = r.shape
+        ids = sample_ids.to(device=r.device, dtype=torch.int64).contiguous()
+        if R % ids.numel():
+            raise ValueError("rows must split evenly over the sample ids")
+        n, rps = ids.numel(), R // ids.numel()
+        shape = (self.aqsgd_samples, rps, L)
+        if self.state is None or tuple(self.state.shape) != shape:
+            self.state = torch.zeros(shape, device=r.device)
+        idx = None
+        if isinstance(c, Quant):
+            mpc_aqsgd_quant_compress(r.reshape(n, rps, L), self.state, ids, c.bits,
+                                     stochastic=c.stochastic, seed=self._seed(0))
+        else:
+            _, idx = mpc_aqsgd_compress(r.reshape(n, rps, L), self.state, ids,
+                                        k_of(L, c.percent))
+            idx = idx.reshape(R, -1)
+        return self.state[ids].reshape(R, L), idx
 
     def _compress_backward(self, gy: torch.Tensor, idx):
         c = self.bw

@@ -465,6 +465,101 @@ mpc_status mpc_quant_decompress(const uint32_t* codes, const float* scale, const
   return ok();
 }
 
+namespace {
+
+// Shared argument checks of the two quantised AQ-SGD calls.
+mpc_status check_aqsgd_quant(int64_t num_samples, int64_t n_ids, int64_t rps, int64_t L,
+                             int bits, int64_t* rows) {
+  if (n_ids < 0) return set_error(MPC_ERR_INVALID_ARG, "n_ids < 0");
+  if (rps < 1) return set_error(MPC_ERR_INVALID_ARG, "rows_per_sample < 1");
+  if (num_samples < 1) return set_error(MPC_ERR_INVALID_ARG, "num_samples < 1");
+  if (n_ids > INT64_MAX / rps) return set_error(MPC_ERR_INVALID_ARG, "rows overflow");
+  *rows = n_ids * rps;
+  MPC_TRY(check_shape(*rows, L, 1));
+  if (!valid_bits(bits))
+    return set_error(MPC_ERR_INVALID_ARG, "bits=%d not in 1..16 or 32", bits);
+  if (L > 0x7fffffffLL / 32) return set_error(MPC_ERR_INVALID_ARG, "row_len too large");
+  if (num_samples > INT64_MAX / rps / L)
+    return set_error(MPC_ERR_INVALID_ARG, "buffer size overflows");
+  return ok();
+}
+
+size_t aqsgd_delta_bytes(int64_t rows, int64_t L) {
+  return (static_cast<size_t>(rows) * static_cast<size_t>(L) * 4 + 255) / 256 * 256;
+}
+
+}  // namespace
+
+size_t mpc_aqsgd_quant_workspace_bytes(int64_t n_ids, int64_t rows_per_sample, int64_t row_len,
+                                       int bits) {
+  if (n_ids <= 0 || rows_per_sample < 1 || row_len < 1 || !valid_bits(bits)) return 0;
+  if (n_ids > INT64_MAX / rows_per_sample) return 0;
+  const int64_t rows = n_ids * rows_per_sample;
+  if (rows > INT64_MAX / 4 / row_len) return 0;
+  return aqsgd_delta_bytes(rows, row_len) + mpc::quant_workspace_bytes(rows, row_len, bits);
+}
+
+mpc_status mpc_aqsgd_quant_compress(const float* x, float* buf, int64_t num_samples,
+                                    const int64_t* sample_ids, int64_t n_ids,
+                                    int64_t rows_per_sample, int64_t row_len, int bits,
+                                    mpc_rounding mode, uint64_t seed, uint32_t* codes,
+                                    float* scale, float* minv, void* ws, size_t ws_bytes,
+                                    mpc_stream_t stream) {
+  int64_t rows = 0;
+  MPC_TRY(check_aqsgd_quant(num_samples, n_ids, rows_per_sample, row_len, bits, &rows));
+  if (mode != MPC_ROUND_NEAREST && mode != MPC_ROUND_STOCHASTIC)
+    return set_error(MPC_ERR_INVALID_ARG, "rounding mode %d", static_cast<int>(mode));
+  if (rows == 0) return ok();
+  MPC_TRY(check_ptr(x, 4, "x"));
+  MPC_TRY(check_ptr(buf, 4, "buf"));
+  MPC_TRY(check_ptr(sample_ids, 8, "sample_ids"));
+  MPC_TRY(check_ptr(codes, 4, "codes"));
+  MPC_TRY(check_ptr(scale, 4, "scale"));
+  MPC_TRY(check_ptr(minv, 4, "minv"));
+  const size_t need = mpc_aqsgd_quant_workspace_bytes(n_ids, rows_per_sample, row_len, bits);
+  if (ws == nullptr || ws_bytes < need)
+    return set_error(MPC_ERR_WORKSPACE, "workspace of %zu bytes needed", need);
+  MPC_TRY(check_ptr(ws, 8, "ws"));
+  Device d;
+  MPC_TRY(current_device(&d));
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  float* delta = static_cast<float*>(ws);
+  const size_t dbytes = aqsgd_delta_bytes(rows, row_len);
+  cudaError_t e = mpc::launch_aqsgd_delta(x, buf, sample_ids, n_ids, rows_per_sample, row_len,
+                                          num_samples, delta, d.status, s);
+  if (e != cudaSuccess) return cuda_error(e, "aqsgd_delta launch");
+  MPC_TRY(mpc_quant_compress(delta, rows, row_len, bits, mode, seed, codes, scale, minv,
+                             static_cast<char*>(ws) + dbytes, ws_bytes - dbytes, stream));
+  const int64_t W = static_cast<int64_t>(mpc_quant_codes_words(1, row_len, bits));
+  e = mpc::launch_aqsgd_dequant_add(codes, scale, minv, buf, sample_ids, n_ids, rows_per_sample,
+                                    row_len, W, bits, num_samples, d.status, s);
+  if (e != cudaSuccess) return cuda_error(e, "aqsgd_dequant_add launch");
+  return ok();
+}
+
+mpc_status mpc_aqsgd_quant_decompress(const uint32_t* codes, const float* scale,
+                                      const float* minv, float* buf_recv, int64_t num_samples,
+                                      const int64_t* sample_ids, int64_t n_ids,
+                                      int64_t rows_per_sample, int64_t row_len, int bits,
+                                      mpc_stream_t stream) {
+  int64_t rows = 0;
+  MPC_TRY(check_aqsgd_quant(num_samples, n_ids, rows_per_sample, row_len, bits, &rows));
+  if (rows == 0) return ok();
+  MPC_TRY(check_ptr(codes, 4, "codes"));
+  MPC_TRY(check_ptr(scale, 4, "scale"));
+  MPC_TRY(check_ptr(minv, 4, "minv"));
+  MPC_TRY(check_ptr(buf_recv, 4, "buf_recv"));
+  MPC_TRY(check_ptr(sample_ids, 8, "sample_ids"));
+  Device d;
+  MPC_TRY(current_device(&d));
+  const int64_t W = static_cast<int64_t>(mpc_quant_codes_words(1, row_len, bits));
+  cudaError_t e = mpc::launch_aqsgd_dequant_add(codes, scale, minv, buf_recv, sample_ids, n_ids,
+                                                rows_per_sample, row_len, W, bits, num_samples,
+                                                d.status, reinterpret_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_error(e, "aqsgd_dequant_add launch");
+  return ok();
+}
+
 mpc_status mpc_get_status(mpc_stream_t stream) {
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   cudaError_t e = cudaStreamSynchronize(s);

@@ -58,6 +58,16 @@ cudaError_t launch_topk_grid(int mode, const TopkGridArgs& a, int num_sms, cudaS
 cudaError_t launch_topk_decompress(const float* vals, const int32_t* idx, int64_t rows,
                                    int64_t L, int64_t k, float* y, int aligned, int num_sms,
                                    cudaStream_t s);
+// AQ-SGD with quantisation (§2.5), aqsgd_quant.cu: d = x - buf[id, r], and
+// buf[id, r] += Dequant(codes).
+cudaError_t launch_aqsgd_delta(const float* x, const float* buf, const int64_t* ids, int64_t n_ids,
+                               int64_t rps, int64_t L, int64_t num_samples, float* d,
+                               unsigned* status, cudaStream_t s);
+cudaError_t launch_aqsgd_dequant_add(const uint32_t* codes, const float* scale, const float* minv,
+                                     float* buf, const int64_t* ids, int64_t n_ids, int64_t rps,
+                                     int64_t L, int64_t W, int bits, int64_t num_samples,
+                                     unsigned* status, cudaStream_t s);
+
 // EF-mixed (§2.4): the steps between its two TopK calls (topk_efmix.cu).
 cudaError_t launch_efmix_mark(float* err, const int32_t* idx, int64_t rows, int64_t L, int64_t k,
                               float* saved, int restore, cudaStream_t s);

@@ -15,6 +15,12 @@ def test_block_arguments():
     with pytest.raises(ValueError):
         m.CompressionBoundary(m.TopK(10, feedback="aqsgd"), None)
     with pytest.raises(ValueError):
+        m.CompressionBoundary(m.Quant(4, feedback="aqsgd"), None)
+    with pytest.raises(ValueError):
+        m.CompressionBoundary(m.TopK(10), m.Quant(4, feedback="aqsgd"), aqsgd_samples=4)
+    with pytest.raises(ValueError):
+        m.Quant(4, feedback="ef")
+    with pytest.raises(ValueError):
         m.TopK(10, feedback="other")
     with pytest.raises(ValueError):
         m.CompressionBoundary(m.TopK(10), None, rows="column")

@@ -76,7 +76,9 @@ def test_feedback_over_steps(mpc, fb):
         k = k_of(512, 10)
         f = oracle.ef_topk_compress if fb == "ef" else oracle.ef21_topk_compress
         v, i = f(xn, state, k)
-        assert_bits_equal(y.cpu().numpy(), oracle.topk_decompress(v, i, 512), "%s step %d" % (fb, step))
+        # EF's receiver takes the message; EF21's takes its copy of g' = g + C(x - g)
+        want = oracle.topk_decompress(v, i, 512) if fb == "ef" else state
+        assert_bits_equal(y.cpu().numpy(), want, "%s step %d" % (fb, step))
         assert_bits_equal(B.state.cpu().numpy(), state, "%s state step %d" % (fb, step))
         assert torch.equal(gx, torch.ones_like(gx))  # no gradient compressor
 
@@ -92,10 +94,35 @@ def test_aqsgd_per_sample_buffer(mpc):
         xn = rng.standard_normal((4, rps, L)).astype(np.float32)
         y, _ = run(B, torch.from_numpy(xn).cuda(), torch.zeros(4, rps, L, device="cuda"),
                    torch.from_numpy(ids).cuda())
-        v, i = oracle.aqsgd_compress(xn, buf, ids, k_of(L, 30))
-        assert_bits_equal(y.cpu().numpy().reshape(4 * rps, L), oracle.topk_decompress(v, i, L),
-                          "aqsgd step %d" % step)
+        oracle.aqsgd_compress(xn, buf, ids, k_of(L, 30))
+        # the next stage receives its copy of the samples' updated buffer rows
+        assert_bits_equal(y.cpu().numpy(), buf[ids], "aqsgd step %d" % step)
         assert_bits_equal(B.state.cpu().numpy(), buf, "buffer step %d" % step)
+
+
+@pytest.mark.parametrize("bits,sr", [(4, False), (8, True)])
+def test_aqsgd_quant_per_sample_buffer(mpc, bits, sr):
+    """AQ-SGD with the quantiser (§2.5's cited work): the change against each sample's
+    buffer is quantised; the next stage receives the updated buffer rows."""
+    S, L = 12, 2 * 8 * 8
+    B = mpc.CompressionBoundary(mpc.Quant(bits, sr, feedback="aqsgd"), mpc.Quant(8),
+                                aqsgd_samples=S, seed=3)
+    buf = np.zeros((S, 1, L), np.float32)
+    rng = np.random.default_rng(2)
+    base = rng.standard_normal((S, 2, 8, 8)).astype(np.float32)
+    for step in range(3):
+        ids = rng.permutation(S)[:5].astype(np.int64)
+        xn = (base[ids] + 0.1 * rng.standard_normal((5, 2, 8, 8))).astype(np.float32)
+        gn = rng.standard_normal((5, 2, 8, 8)).astype(np.float32)
+        y, gx = run(B, torch.from_numpy(xn).cuda(), torch.from_numpy(gn).cuda(),
+                    torch.from_numpy(ids).cuda())
+        seed_fw = (((3 << 1) | 0) << 32) | step
+        oracle.aqsgd_quant_compress(xn.reshape(5, 1, L), buf, ids, bits, sr, seed_fw)
+        assert_bits_equal(y.cpu().numpy().reshape(5, 1, L), buf[ids], "aqsgd-q step %d" % step)
+        assert_bits_equal(B.state.cpu().numpy(), buf, "buffer step %d" % step)
+        c, s_, m = oracle.quant_compress(gn.reshape(5, L), 8, False, 0)
+        assert_bits_equal(gx.cpu().numpy().reshape(5, L),
+                          oracle.quant_decompress(c, s_, m, L, 8), "gradient step %d" % step)
 
 
 @pytest.mark.parametrize("bits,sr", [(2, False), (4, True), (6, False), (8, True)])
