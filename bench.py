@@ -60,6 +60,8 @@ def parse_args():
     p.add_argument("--impl", choices=("ours", "reference"), default="ours")
     p.add_argument("--no-operators", action="store_true", help="skip the per-operator table")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--branches", type=int, default=5, choices=(1, 2, 3, 5, 9),
+                   help="concurrent streams inside the step graph (1 = all launches in order)")
     return p.parse_args()
 
 
@@ -310,12 +312,14 @@ class Step:
         self.vals = {p: torch.empty((R, self.ks[p]), device=device) for p in TOPK_PCTS}
         self.idx = {p: torch.empty((R, self.ks[p]), dtype=torch.int32, device=device)
                     for p in TOPK_PCTS}
-        self.y = torch.empty((R, L), device=device)
-        self.gy = torch.empty((R, L), device=device)
+        # every pair has its own outputs, so that pairs on different streams share nothing
+        QS = [(b, sr) for b in BITS for sr in (False, True)]
+        self.y = {p: torch.empty((R, L), device=device) for p in TOPK_PCTS}
+        self.gy = {q: torch.empty((R, L), device=device) for q in QS}
         W = {b: mpc.mpc_quant_codes_words(R, L, b) // R for b in BITS}
-        self.codes = {b: torch.empty((R, W[b]), dtype=torch.int32, device=device) for b in BITS}
-        self.scale = {b: torch.empty(R, device=device) for b in BITS}
-        self.minv = {b: torch.empty(R, device=device) for b in BITS}
+        self.codes = {q: torch.empty((R, W[q[0]]), dtype=torch.int32, device=device) for q in QS}
+        self.scale = {q: torch.empty(R, device=device) for q in QS}
+        self.minv = {q: torch.empty(R, device=device) for q in QS}
         self.seed = seed
         self.ops = []  # (name, bytes) in launch order
         for p in TOPK_PCTS:
@@ -330,9 +334,14 @@ class Step:
                 self.ops.append(("quant_decompress " + tag, algorithmic_bytes(R, L, bits=b, op="dequant")))
         self.input_bytes = 9 * 4 * R * L  # 9 compress+decompress pairs
 
-    def launch(self, slot: int, step: int, events=None, x=None, g=None, around=None):
+    def launch(self, slot: int, step: int, events=None, x=None, g=None, around=None, side=None,
+               y=None, gy=None):
         """Enqueue the step's 18 launches.  events: one event recorded after each launch;
-        around: (i, ev0, ev1) records ev0 just before launch i and ev1 just after it."""
+        around: (i, ev0, ev1) records ev0 just before launch i and ev1 just after it.
+        side: streams for concurrent branches (the nine pairs are independent; BRANCH_OF
+        maps a pair to its branch, branch 0 being the current stream).  The branches fork
+        from and join back into the current stream.  y, gy: outputs to use instead of the
+        step's own, by TopK percent and by (bits, stochastic)."""
         m = self.mpc
         x = self.xs[slot] if x is None else x
         g = self.gs[slot] if g is None else g
@@ -349,16 +358,63 @@ class Step:
                 next(e).record()
             n[0] += 1
 
-        for p in TOPK_PCTS:
-            op(lambda: m.mpc_ef_topk_compress(x, self.errs[p], self.ks[p], self.vals[p], self.idx[p]))
-            op(lambda: m.mpc_topk_decompress(self.vals[p], self.idx[p], L, y=self.y))
+        ys = {**self.y, **(y or {})}
+        gys = {**self.gy, **(gy or {})}
+        nb = 1 + len(side or [])
+        seq = []  # (branch, launch) in the order of self.ops
+        for i, p in enumerate(TOPK_PCTS):
+            br = BRANCH_OF[nb](i, None)
+            seq.append((br, lambda p=p: m.mpc_ef_topk_compress(x, self.errs[p], self.ks[p],
+                                                               self.vals[p], self.idx[p])))
+            seq.append((br, lambda p=p: m.mpc_topk_decompress(self.vals[p], self.idx[p], L,
+                                                              y=ys[p])))
         for b in BITS:
             for sr in (False, True):
-                op(lambda: m.mpc_quant_compress(g, b, stochastic=sr, seed=(self.seed << 32) | step,
-                                                codes=self.codes[b], scale=self.scale[b],
-                                                minv=self.minv[b]))
-                op(lambda: m.mpc_quant_decompress(self.codes[b], self.scale[b], self.minv[b], L, b,
-                                                  y=self.gy))
+                q = (b, sr)
+                br = BRANCH_OF[nb](len(seq) // 2, sr)
+                seq.append((br, lambda q=q: m.mpc_quant_compress(
+                    g, q[0], stochastic=q[1], seed=(self.seed << 32) | step, codes=self.codes[q],
+                    scale=self.scale[q], minv=self.minv[q])))
+                seq.append((br, lambda q=q: m.mpc_quant_decompress(
+                    self.codes[q], self.scale[q], self.minv[q], L, q[0], y=gys[q])))
+        if not side:
+            for _, fn in seq:
+                op(fn)
+            return
+        main = torch.cuda.current_stream()
+        streams = [main] + list(side)
+        fork = torch.cuda.Event()
+        fork.record(main)
+        for s in side:
+            s.wait_event(fork)
+        for br, fn in seq:
+            with torch.cuda.stream(streams[br]):
+                fn()
+        for s in side:
+            main.wait_stream(s)
+
+
+# Branch of pair i (0-2 the TopK pairs, 3-8 the quantisation pairs; sr = stochastic
+# rounding) for a step of n concurrent branches.
+BRANCH_OF = {
+    1: lambda i, sr: 0,
+    2: lambda i, sr: 0 if i < 3 else 1,
+    3: lambda i, sr: 0 if i < 3 else 1 + int(sr),
+    5: lambda i, sr: i if i < 3 else 3 + int(sr),
+    9: lambda i, sr: i,
+}
+
+BRANCH_TEXT = {
+    1: "the 18 launches in order on one stream",
+    2: "two concurrent branches (the three TopK pairs; the six quantisation pairs), each in "
+       "order, forked from and joined into one stream",
+    3: "three concurrent branches (the three TopK pairs; the nearest quantisation pairs; the "
+       "stochastic ones), each in order, forked from and joined into one stream",
+    5: "five concurrent branches (each TopK pair; the nearest quantisation pairs; the "
+       "stochastic ones), each in order, forked from and joined into one stream",
+    9: "nine concurrent branches (one per compress+decompress pair), forked from and joined "
+       "into one stream",
+}
 
 
 def make_event(external: bool):
@@ -384,6 +440,7 @@ def run_ours(args, rank, local, world):
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=device)
     flush_sink = torch.empty((), dtype=torch.int64, device=device)
     stream = torch.cuda.Stream(device)
+    side = [torch.cuda.Stream(device) for _ in range(args.branches - 1)]
     torch.cuda.synchronize()
 
     def flush_l2(i):
@@ -397,6 +454,7 @@ def run_ours(args, rank, local, world):
     with torch.cuda.stream(stream):
         for w in range(2):
             st.launch(w % POOL, w)
+            st.launch(w % POOL, w, side=side)
     stream.synchronize()
     assert mpc.mpc_get_status(stream) == 0, mpc.mpc_last_error()
 
@@ -414,7 +472,7 @@ def run_ours(args, rank, local, world):
             st.launch(slot, slot, **kw)
         return g
 
-    plain = [capture(slot) for slot in range(POOL)]
+    plain = [capture(slot, side=side) for slot in range(POOL)]
     evsets = [[make_event(True) for _ in range(n_ops)] for _ in range(POOL)]
     keep.append(evsets)
     evented = [capture(slot, events=evsets[slot]) for slot in range(POOL)]
@@ -505,7 +563,7 @@ def run_ours(args, rank, local, world):
               for j in range(n_ops)}
 
     # end to end through the Python API: host inputs in, two outputs back, no graphs
-    e2e = run_e2e(args, st, stream, world, device)
+    e2e = run_e2e(args, st, stream, side, world, device)
 
     operators = None
     if not args.no_operators and rank == 0:
@@ -524,59 +582,94 @@ def run_ours(args, rank, local, world):
             "config": {"workload": WORKLOAD, "rows": R, "row_len": L,
                        "topk_percents": list(TOPK_PCTS), "bits": list(BITS),
                        "rounding": ["nearest", "stochastic"], "launches_per_step": n_ops,
-                       "step": "one CUDA graph per step (no event nodes inside)", "l2": "256 MiB buffer "
+                       "step": "one CUDA graph per step (no event nodes inside); " + BRANCH_TEXT[args.branches],
+                       "l2": "256 MiB buffer "
                        "written then read before each timed step, outside the timed interval "
                        "(inputs cold, no dirty lines left by the flush)", "parallelism":
                        "replicas" if world > 1 else "single GPU"},
             "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
             "gpu_launches": n_ops * args.steps, "clocks": clocks,
             "wall_s": round(wall, 3), "per_op": per_op,
-            "per_op_timing": "an event after every launch inside the step graph (second pass; "
-                             "each interval includes the ~5 us of an event node)",
+            "per_op_timing": "an event after every launch inside a graph of the 18 launches in "
+                             "order on one stream (second pass; each interval includes the ~5 us "
+                             "of an event node)",
             "operators": operators,
         }
         print(json.dumps(line), flush=True)
 
 
-def run_e2e(args, st, stream, world, device):
+def run_e2e(args, st, stream, side, world, device):
+    """The step end to end through the Python API: every step copies its two inputs from
+    pinned host memory to the device and two of its results back, inside the timed
+    region.  Copies and compute are pipelined over two slots (inputs and read-back
+    outputs double-buffered; step s+1's inputs go up while step s computes and step
+    s-1's results come down), each copy on its own stream; the compute of a slot is the
+    step's API calls captured once into a CUDA graph (its branches as in the headline)."""
     mpc = st.mpc
     hx = [t.cpu().pin_memory() for t in st.xs]
     hg = [t.cpu().pin_memory() for t in st.gs]
-    dx = torch.empty_like(st.xs[0])
-    dg = torch.empty_like(st.gs[0])
-    hy = torch.empty((R, L), pin_memory=True)
-    hgy = torch.empty((R, L), pin_memory=True)
-    k10 = 10
+    k10, q8 = 10, (8, True)  # read back: the K=10% activation, the 8-bit stochastic gradient
+    dx = [torch.empty_like(st.xs[0]) for _ in range(2)]
+    dg = [torch.empty_like(st.gs[0]) for _ in range(2)]
+    dy = [torch.empty((R, L), device=device) for _ in range(2)]
+    dgy = [torch.empty((R, L), device=device) for _ in range(2)]
+    hy = [torch.empty((R, L), pin_memory=True) for _ in range(2)]
+    hgy = [torch.empty((R, L), pin_memory=True) for _ in range(2)]
+    up = [torch.cuda.Stream(device) for _ in range(2)]
+    down = [torch.cuda.Stream(device) for _ in range(2)]
+    ev = lambda: [torch.cuda.Event() for _ in range(2)]  # noqa: E731
+    x_in, g_in, done, y_out, g_out = ev(), ev(), ev(), ev(), ev()
+
+    graphs = []
+    for slot in range(2):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            st.launch(slot, slot, x=dx[slot], g=dg[slot], side=side,
+                      y={k10: dy[slot]}, gy={q8: dgy[slot]})
+        graphs.append(g)
 
     def one(s):
-        dx.copy_(hx[s % POOL], non_blocking=True)
-        dg.copy_(hg[s % POOL], non_blocking=True)
-        st.launch(0, s, x=dx, g=dg)
-        # outputs read back: the K=10% decompressed activation and the 8-bit gradient
-        mpc.mpc_topk_decompress(st.vals[k10], st.idx[k10], L, y=st.y)
-        hy.copy_(st.y, non_blocking=True)
-        hgy.copy_(st.gy, non_blocking=True)
+        b = s % 2
+        for stm, dst, src, e in ((up[0], dx[b], hx[s % POOL], x_in[b]),
+                                 (up[1], dg[b], hg[s % POOL], g_in[b])):
+            stm.wait_event(done[b])  # the slot's previous compute has read it
+            with torch.cuda.stream(stm):
+                dst.copy_(src, non_blocking=True)
+                e.record(stm)
+        for e in (x_in[b], g_in[b], y_out[b], g_out[b]):
+            stream.wait_event(e)
+        with torch.cuda.stream(stream):
+            graphs[b].replay()
+            done[b].record(stream)
+        for stm, dst, src, e in ((down[0], hy[b], dy[b], y_out[b]),
+                                 (down[1], hgy[b], dgy[b], g_out[b])):
+            stm.wait_event(done[b])
+            with torch.cuda.stream(stm):
+                dst.copy_(src, non_blocking=True)
+                e.record(stm)
 
     steps = max(3, min(args.steps, 50))
-    with torch.cuda.stream(stream):
-        for s in range(3):
-            one(s)
-    stream.synchronize()
+    for s in range(3):
+        one(s)
+    torch.cuda.synchronize()
     barrier(world)
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
-    with torch.cuda.stream(stream):
-        e0.record(stream)
-        for s in range(steps):
-            one(s)
-        e1.record(stream)
-    stream.synchronize()
+    e0.record(stream)
+    for s in range(steps):
+        one(s)
+    for e in y_out + g_out:
+        stream.wait_event(e)
+    e1.record(stream)
+    torch.cuda.synchronize()
     barrier(world)
     secs = e0.elapsed_time(e1) / 1e3
     units, secs = aggregate(st.input_bytes * steps, secs, world, device)
     return {"value": round(units / secs / 1e9, 2), "unit": UNIT,
             "h2d_bytes_per_step": 2 * 4 * R * L, "d2h_bytes_per_step": 2 * 4 * R * L,
-            "steps": steps, "api": "python binding, no graphs"}
+            "steps": steps, "api": "python binding calls of one step captured into a CUDA "
+            "graph per input slot; per step two H2D copies from pinned memory and two D2H "
+            "copies of results on copy streams, pipelined over two slots"}
 
 
 def time_op(fn, stream, flush, reps=5):
