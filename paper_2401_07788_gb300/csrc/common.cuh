@@ -106,21 +106,31 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
+// The retry loop of mbar_wait_bounded, out of line: a first try that succeeds
+// (the common case once the copy has landed) costs no more than the try.
+static __device__ __noinline__ bool mbar_wait_retry(uint64_t* bar, uint32_t parity, uint32_t limit,
+                                                    unsigned* status) {
+  const uint64_t deadline = global_ns() + 64ull * limit;
+  for (uint32_t i = 1; i < limit; ++i) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (global_ns() > deadline) break;
+  }
+  set_status(status, STATUS_TIMEOUT);
+  return false;
+}
+
 // Wait for phase `parity` of `bar` to complete: at most `limit` tries, and no
 // new try once about 64 ns x `limit` have passed since the first one (a try
 // itself ends within about 1 ms).
 // Returns false, and records STATUS_TIMEOUT, if it gave up.
 __device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity,
                                                   uint32_t limit, unsigned* status) {
-  uint64_t deadline = 0;
-  for (uint32_t i = 0; i < limit; ++i) {
-    if (mbar_try_wait(bar, parity)) return true;
-    const uint64_t now = global_ns();
-    if (i == 0) deadline = now + 64ull * limit;
-    else if (now > deadline) break;
+  if (limit > 0 && mbar_try_wait(bar, parity)) return true;
+  if (limit <= 1) {
+    set_status(status, STATUS_TIMEOUT);
+    return false;
   }
-  set_status(status, STATUS_TIMEOUT);
-  return false;
+  return mbar_wait_retry(bar, parity, limit, status);
 }
 
 // Bulk copy of `bytes` (multiple of 16, both addresses 16-byte aligned) from

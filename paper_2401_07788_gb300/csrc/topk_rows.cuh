@@ -845,12 +845,20 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
     }
     __syncwarp();
     {
+      // at most 128 kept entries a chunk: up to four warp-wide rounds, the
+      // later ones only when the chunk keeps that many
       const int colbase = static_cast<int>(c0) + 4 * (j * NT + warp * 32);
-      for (uint32_t t = lane; t < tot; t += 32) {
-        const uint32_t p = pos + t;
-        if (p < kk32) {
-          vrow[p] = sval[t];
-          irow[p] = colbase + soff[t];
+      const uint32_t lim = min(tot, kk32 > pos ? kk32 - pos : 0u);
+      float* vdst = vrow + pos;
+      int32_t* idst = irow + pos;
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        if (32u * u < lim) {
+          const uint32_t t = 32u * u + lane;
+          if (t < lim) {
+            vdst[t] = sval[t];
+            idst[t] = colbase + soff[t];
+          }
         }
       }
     }
