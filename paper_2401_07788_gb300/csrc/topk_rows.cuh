@@ -562,7 +562,7 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
       // it are the candidates for T, pushed to every CTA of the row at their
       // place in the row's candidate table ------------------------------------
       uint32_t wab = 0;
-#pragma unroll 2
+#pragma unroll 1
       for (int j = 0; j < QPT; ++j) {
         uint32_t ab = 0;
         if (j < jv) {
