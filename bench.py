@@ -13,13 +13,17 @@ one boundary crossing of every operator the workload sweeps, on that step's tens
 value = sum over the 9 compress+decompress pairs of the input bytes (4 x 128 x 32768) /
 device time of the step.  Each step is one CUDA graph of the 18 library launches (one
 graph per slot of a pool of 4 pre-drawn steps, so inputs differ from step to step), with
-no event nodes inside; L2 is flushed before every timed step by writing and then
+no event nodes inside; the nine pairs are independent and run as concurrent branches of
+the graph (--branches).  L2 is flushed before every timed step by writing and then
 reading a 256 MiB buffer (so the step's inputs are cold and the flush leaves no dirty
-lines for the first launch to write back), outside the timed interval.  Per-launch times come from a second timed pass
-whose graphs record an event after every launch, and the dominant launch's duration
-(for `roofline`) from a third pass with one event pair around that launch only.  `e2e` runs the same steps through the Python API without graphs, with the
-step's inputs copied from pinned host memory and two outputs copied back inside the
-timed region.  `operators` times every operator of the path on its own workload.
+lines for the first launch to write back), outside the timed interval.  Per-launch
+shares come from a second timed pass whose graphs run the 18 launches in order and
+record an event after every launch; the dominant launch's duration (for `roofline`)
+from a third pass that launches it alone after each flush, between two events on its
+stream, behind a GPU-side sleep so that the host's enqueue never delays it.  `e2e` runs
+the steps through the Python API with the step's inputs copied from pinned host memory
+and two outputs copied back inside the timed region.  `operators` times every operator
+of the path on its own workload.
 
 `--impl reference` times the CPU oracle (single-threaded C) on a bounded sample of the
 same step: 16 of the 128 rows.
@@ -334,10 +338,10 @@ class Step:
                 self.ops.append(("quant_decompress " + tag, algorithmic_bytes(R, L, bits=b, op="dequant")))
         self.input_bytes = 9 * 4 * R * L  # 9 compress+decompress pairs
 
-    def launch(self, slot: int, step: int, events=None, x=None, g=None, around=None, side=None,
-               y=None, gy=None):
+    def launch(self, slot: int, step: int, events=None, x=None, g=None, side=None,
+               y=None, gy=None, only=None):
         """Enqueue the step's 18 launches.  events: one event recorded after each launch;
-        around: (i, ev0, ev1) records ev0 just before launch i and ev1 just after it.
+        only: enqueue launch `only` alone (timing of one launch on its own).
         side: streams for concurrent branches (the nine pairs are independent; BRANCH_OF
         maps a pair to its branch, branch 0 being the current stream).  The branches fork
         from and join back into the current stream.  y, gy: outputs to use instead of the
@@ -349,11 +353,7 @@ class Step:
         n = [0]
 
         def op(fn):
-            if around is not None and around[0] == n[0]:
-                around[1].record()
             fn()
-            if around is not None and around[0] == n[0]:
-                around[2].record()
             if e is not None:
                 next(e).record()
             n[0] += 1
@@ -377,6 +377,9 @@ class Step:
                     scale=self.scale[q], minv=self.minv[q])))
                 seq.append((br, lambda q=q: m.mpc_quant_decompress(
                     self.codes[q], self.scale[q], self.minv[q], L, q[0], y=gys[q])))
+        if only is not None:
+            seq[only][1]()
+            return
         if not side:
             for _, fn in seq:
                 op(fn)
@@ -461,7 +464,8 @@ def run_ours(args, rank, local, world):
     # One graph per pool slot.  Event nodes inside a graph cost ~5 us each, so the
     # headline steps replay event-free graphs; per-launch times come from a second
     # timed pass with an event after every launch (shares of the step), and the
-    # dominant launch's duration from a third pass with one event pair around it.
+    # dominant launch's duration from a third pass that launches it alone between two
+    # events (time_alone).
     if make_event(external=True) is None:
         raise RuntimeError("torch.cuda.Event(external=True) is required")
     keep = []  # events referenced by graph nodes must outlive the graphs
@@ -526,15 +530,7 @@ def run_ours(args, rank, local, world):
 
     timed_pass(evented, read_ops)
     dom = max(range(n_ops), key=lambda j: op_ms[j])
-    pairs = [(make_event(True), make_event(True)) for _ in range(POOL)]
-    keep.append(pairs)
-    around = [capture(slot, around=(dom, pairs[slot][0], pairs[slot][1])) for slot in range(POOL)]
-    dom_ms = [0.0]
-
-    def read_dom(j, start, end):
-        dom_ms[0] += pairs[j % POOL][0].elapsed_time(pairs[j % POOL][1])
-
-    timed_pass(around, read_dom)
+    dom_ms = time_alone(st, dom, stream, flush_l2, min(args.steps, 300), args.warmup)
     status = mpc.mpc_get_status(stream)
     if status != 0:
         raise RuntimeError("device status %d: %s" % (status, mpc.mpc_last_error()))
@@ -545,7 +541,7 @@ def run_ours(args, rank, local, world):
     # roofline of the dominant kernel (largest share of the step)
     peak, peak_kind = hbm_peak()
     name, nbytes = st.ops[dom]
-    avg_ms = dom_ms[0] / args.steps
+    avg_ms = dom_ms
     achieved = nbytes / (avg_ms / 1e3) / 1e9
     kern = "topk_cta_kernel" if "topk_compress" in name else (
         "topk_decompress_rows_kernel" if "decompress K" in name else (
@@ -557,7 +553,8 @@ def run_ours(args, rank, local, world):
                 "avg_launch_us": round(avg_ms * 1e3, 2),
                 "share_of_step": round(op_ms[dom] / max(sum(op_ms), 1e-9), 4),
                 "peak_source": peak_kind,
-                "timing": "one event pair around this launch inside the step graph"}
+                "timing": "launched alone after each L2 flush, between two events on its "
+                          "stream, behind a GPU-side sleep (median of %d)" % min(args.steps, 300)}
     per_op = {st.ops[j][0]: {"avg_us": round(op_ms[j] / args.steps * 1e3, 2),
                              "GBps": round(st.ops[j][1] / (op_ms[j] / args.steps / 1e3) / 1e9, 1)}
               for j in range(n_ops)}
@@ -596,6 +593,30 @@ def run_ours(args, rank, local, world):
             "operators": operators,
         }
         print(json.dumps(line), flush=True)
+
+
+def time_alone(st, i, stream, flush_l2, n, warmup):
+    """Median device time (ms) of launch i of the step on its own, on cold inputs: after
+    each L2 flush a GPU-side sleep of ~50 us lets the host enqueue the two events and
+    the launch before the stream reaches them, so the interval holds the launch alone."""
+    with torch.cuda.stream(stream):
+        for w in range(warmup):
+            flush_l2(w)
+            st.launch(w % POOL, w, only=i)
+        stream.synchronize()
+        pairs = []
+        for s in range(n):
+            flush_l2(s)
+            torch.cuda._sleep(100_000)
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            st.launch(s % POOL, s, only=i)
+            b.record(stream)
+            pairs.append((a, b))
+        stream.synchronize()
+    ts = [a.elapsed_time(b) for a, b in pairs]
+    return statistics.median(ts)
 
 
 def run_e2e(args, st, stream, side, world, device):
