@@ -30,6 +30,7 @@ struct TopkRowArgs {
   int aligned;            // 1: every row start is 16-byte aligned (bulk copies allowed)
   uint32_t spin_limit;    // polls before a wait gives up
   unsigned* status;       // device status word
+  int wide_cta;           // 1: rows of 8193..32768 entries may take one wide CTA each
 };
 
 // Largest row the on-chip row path handles (cluster of 8 CTAs x 8192).

@@ -202,11 +202,14 @@ template <int NT, int NBINS, class Sh>
 __device__ __forceinline__ BinPick cluster_pick(const uint32_t* hist, uint32_t* gsum, uint32_t C,
                                                 uint32_t crank, uint32_t kr, Sh& sh, int tid,
                                                 int lane, int warp) {
-  constexpr int G = NBINS / NT;
-  static_assert(G * NT == NBINS && G * kMaxCluster <= 128, "bin groups");
+  constexpr int NG = NT < NBINS ? NT : NBINS;  // bin groups: thread t < NG owns group t
+  constexpr int G = NBINS / NG;
+  static_assert(G * NG == NBINS && G * kMaxCluster <= 128, "bin groups");
   uint32_t gs = 0;
+  if (tid < NG) {
 #pragma unroll
-  for (int b = 0; b < G; ++b) gs += hist[NBINS - 1 - (tid * G + b)];
+    for (int b = 0; b < G; ++b) gs += hist[NBINS - 1 - (tid * G + b)];
+  }
   uint32_t total = gs;
   if (C > 1) {
     uint32_t* mine = gsum + crank * NT + tid;
@@ -283,7 +286,8 @@ __device__ __forceinline__ void row_sync(uint32_t C) {
 }
 
 template <int MODE, int NT, int SCAP, bool FULL>
-__global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const TopkRowArgs a) {
+__global__ void __launch_bounds__(NT, (NT == 128 ? 6 : NT == 256 ? 4 : NT == 512 ? 2 : 1))
+    topk_cta_kernel(const TopkRowArgs a) {
   pdl_begin();
   constexpr int NW = NT / 32;
   constexpr int NQ = SCAP / 4;     // float4 slots per slice
@@ -291,7 +295,10 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
   constexpr int NCH = SCAP / 128;  // 128-entry chunks per slice
   constexpr int G = kNB / NT;      // bins of a thread's group in the first histogram
   constexpr int GW = G / 2;        // packed words of a group (two 16-bit counts each)
-  static_assert(G == 4 || G == 8, "bin groups of 4 or 8");
+  // A wide CTA (512 or 1024 threads) holds a whole row: no cluster, and the
+  // histogram is read where it was built.
+  constexpr bool kWide = NT >= 512;
+  static_assert(G == 4 || G == 8 || (kWide && (G == 1 || G == 2)), "bin groups");
   static_assert(SCAP < 65536, "per-CTA bin counts fit 16 bits");
   using Sh = CtaShared<NT, SCAP>;
   __shared__ Sh sh;
@@ -447,8 +454,14 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
     if (scale > 0.0f) {
       // Every CTA pushes its histogram, packed two 16-bit counts to a word, to
       // every CTA of the row; thread t owns group t of G bins (groups ranked
-      // high to low).
-      {
+      // high to low).  A wide CTA folds the zeros into bin 0 and reads its
+      // histogram in place.
+      if constexpr (kWide) {
+        if (warp == 0) {
+          const uint32_t z = __reduce_add_sync(kFull, sh.u.hist[kNB + lane]);
+          if (lane == 0) sh.u.hist[0] += z;
+        }
+      } else {
         const int b0 = kNB - G * (tid + 1);
         uint32_t w[GW];
 #pragma unroll
@@ -473,15 +486,20 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
       row_sync(C);
       // counts of group g's bins (ascending) summed over the row
       auto group_bins = [&](int g, uint32_t (&cnt)[G]) {
+        if constexpr (kWide) {
 #pragma unroll
-        for (int b = 0; b < G; ++b) cnt[b] = 0;
-        for (uint32_t r = 0; r < C; ++r) {
-          const uint32_t* src = table + (r * NT + g) * GW;
+          for (int b = 0; b < G; ++b) cnt[b] = sh.u.hist[kNB - G * (g + 1) + b];
+        } else {
 #pragma unroll
-          for (int i = 0; i < GW; ++i) {
-            const uint32_t wv = src[i];
-            cnt[2 * i] += wv & 0xffffu;
-            cnt[2 * i + 1] += wv >> 16;
+          for (int b = 0; b < G; ++b) cnt[b] = 0;
+          for (uint32_t r = 0; r < C; ++r) {
+            const uint32_t* src = table + (r * NT + g) * GW;
+#pragma unroll
+            for (int i = 0; i < GW; ++i) {
+              const uint32_t wv = src[i];
+              cnt[2 * i] += wv & 0xffffu;
+              cnt[2 * i + 1] += wv >> 16;
+            }
           }
         }
       };
@@ -533,7 +551,11 @@ __global__ void __launch_bounds__(NT, (NT == 256 ? 4 : 6)) topk_cta_kernel(const
         const int gB = (kNB - 1 - Bw) / G;
         const int ib = Bw - (kNB - G * (gB + 1));
         uint32_t cr = 0;
-        if (lane < static_cast<int>(C)) {
+        if constexpr (kWide) {
+          (void)gB;
+          (void)ib;
+          cr = lane == 0 ? mw : 0u;
+        } else if (lane < static_cast<int>(C)) {
           const uint32_t wv = table[(lane * NT + gB) * GW + ib / 2];
           cr = (ib & 1) ? (wv >> 16) : (wv & 0xffffu);
         }
@@ -1234,7 +1256,7 @@ template <int MODE, int NT, int SCAP, bool FULL>
 cudaError_t run_cta(const TopkRowArgs& a, int C, cudaStream_t s) {
   auto kernel = topk_cta_kernel<MODE, NT, SCAP, FULL>;
   const int smem = cta_smem_bytes(NT, SCAP, C);
-  cudaError_t err = ensure_dynamic_smem(kernel, cta_smem_bytes(NT, SCAP, kMaxCluster));
+  cudaError_t err = ensure_dynamic_smem(kernel, cta_smem_bytes(NT, SCAP, NT >= 512 ? 1 : kMaxCluster));
   if (err != cudaSuccess) return err;
   return launch_kernel(kernel, dim3(static_cast<unsigned>(a.rows * C)), dim3(NT), smem, s,
                        static_cast<unsigned>(C), a);
@@ -1266,6 +1288,18 @@ cudaError_t run_mode(const TopkRowArgs& a0, int num_sms, cudaStream_t s) {
   if (L <= 4096) {
     a.slice = (L + 3) / 4 * 4;
     return run_cta_any<MODE, 128, 4096>(a, 1, s);
+  }
+  // Rows up to 32768 entries take one wide CTA each (512 threads and 2 CTAs
+  // per SM up to 16384, else 1024 threads and one CTA per SM) when that fills
+  // most of the GPU in a single wave: no cluster barriers on the way.  With
+  // more rows the smaller clustered CTAs of several waves pack better.
+  if (a.wide_cta && L <= 16384 && a.rows >= num_sms && a.rows <= 2 * num_sms) {
+    a.slice = (L + 3) / 4 * 4;
+    return run_cta_any<MODE, 512, 16384>(a, 1, s);
+  }
+  if (a.wide_cta && L <= 32768 && 4 * a.rows >= 3 * num_sms && a.rows <= num_sms) {
+    a.slice = (L + 3) / 4 * 4;
+    return run_cta_any<MODE, 1024, 32768>(a, 1, s);
   }
   int64_t C = (L + 8191) / 8192;
   while (a.rows * C < 2 * num_sms && C < kMaxCluster && L / (2 * C) >= 2048) C *= 2;

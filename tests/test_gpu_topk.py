@@ -173,3 +173,69 @@ def test_long_row_decompress_tiles(mpc):
         vals = rng.standard_normal((R, k)).astype(np.float32)
         y = mpc.mpc_topk_decompress(dev(vals), dev(idx), L)
         assert_bits_equal(y.cpu().numpy(), oracle.topk_decompress(vals, idx, L), "k=%d" % k)
+
+
+# Rows of 8193..32768 entries with enough rows to fill the GPU take one wide CTA each
+# (512 threads up to 16384 entries, else 1024); the knob value 3 keeps them on clusters.
+WIDE = [(160, 8193), (160, 12345), (160, 16384), (120, 16385), (116, 20000), (120, 32768)]
+
+
+@pytest.mark.parametrize("R,L", WIDE)
+@pytest.mark.parametrize("path", [0, 3])
+def test_topk_wide_rows(mpc, R, L, path):
+    try:
+        mpc.mpc_set_knob(mpc.MPC_KNOB_TOPK_PATH, path)
+        for kind in ("normal", "relu", "ties", "zeros", "outlier"):
+            x = rows_of(kind, R, L, seed=L + R)
+            xd = dev(x)
+            for k in (1, L // 20, L // 3, L - 1):
+                v, i = mpc.mpc_topk_compress(xd, k)
+                check_status(mpc)
+                ov, oi = oracle.topk_compress(x, k)
+                assert_bits_equal(i.cpu().numpy(), oi, "idx %s L=%d k=%d" % (kind, L, k))
+                assert_bits_equal(v.cpu().numpy(), ov, "vals %s L=%d k=%d" % (kind, L, k))
+    finally:
+        mpc.mpc_set_knob(mpc.MPC_KNOB_TOPK_PATH, 0)
+
+
+@pytest.mark.parametrize("R,L", [(160, 16384), (120, 32768), (116, 24001)])
+def test_ef_ef21_wide_rows(mpc, R, L):
+    rng = np.random.default_rng(L)
+    k = max(1, L // 10)
+    e_host = np.zeros((R, L), np.float32)
+    g_host = np.zeros((R, L), np.float32)
+    e_dev = torch.zeros((R, L), dtype=torch.float32, device="cuda")
+    g_dev = torch.zeros((R, L), dtype=torch.float32, device="cuda")
+    x = np.maximum(rng.standard_normal((R, L)), 0).astype(np.float32)
+    for step in range(3):
+        v, i = mpc.mpc_ef_topk_compress(dev(x), e_dev, k)
+        check_status(mpc)
+        ov, oi = oracle.ef_topk_compress(x, e_host, k)
+        assert_bits_equal(i.cpu().numpy(), oi, "EF idx step %d" % step)
+        assert_bits_equal(v.cpu().numpy(), ov, "EF vals step %d" % step)
+        assert_bits_equal(e_dev.cpu().numpy(), e_host, "EF err step %d" % step)
+        v, i = mpc.mpc_ef21_topk_compress(dev(x), g_dev, k)
+        check_status(mpc)
+        ov, oi = oracle.ef21_topk_compress(x, g_host, k)
+        assert_bits_equal(i.cpu().numpy(), oi, "EF21 idx step %d" % step)
+        assert_bits_equal(v.cpu().numpy(), ov, "EF21 vals step %d" % step)
+        assert_bits_equal(g_dev.cpu().numpy(), g_host, "EF21 g step %d" % step)
+        x = (x + 0.1 * rng.standard_normal((R, L))).astype(np.float32)
+
+
+def test_aqsgd_wide_rows(mpc):
+    """AQ-SGD rows of 16384 entries, 160 of them (8 samples x 20 rows): one wide CTA a row."""
+    rng = np.random.default_rng(3)
+    S, rps, n, L = 24, 20, 8, 16384
+    k = L * 30 // 100
+    buf = rng.standard_normal((S, rps, L)).astype(np.float32)
+    buf_dev = dev(buf)
+    for step in range(2):
+        ids = rng.permutation(S)[:n].astype(np.int64)
+        x = (buf[ids] + 0.05 * rng.standard_normal((n, rps, L))).astype(np.float32)
+        v, i = mpc.mpc_aqsgd_compress(dev(x), buf_dev, dev(ids), k)
+        check_status(mpc)
+        ov, oi = oracle.aqsgd_compress(x, buf, ids, k)
+        assert_bits_equal(i.cpu().numpy(), oi, "AQ-SGD idx step %d" % step)
+        assert_bits_equal(v.cpu().numpy(), ov, "AQ-SGD vals step %d" % step)
+        assert_bits_equal(buf_dev.cpu().numpy(), buf, "AQ-SGD buffer step %d" % step)
