@@ -813,7 +813,7 @@ __global__ void __launch_bounds__(NT, (NT == 128 ? 6 : NT == 256 ? 4 : NT == 512
   int32_t* irow = a.idx + row * k;
   const uint32_t kk32 = static_cast<uint32_t>(min64(k, 0x7fffffff));
   const unsigned lt = lanemask_lt();
-#pragma unroll 2
+#pragma unroll 1
   for (int j = 0; j < jv; ++j) {
     const int q = j * NT + tid;
     const float4 v4 = s4[q];
@@ -848,20 +848,17 @@ __global__ void __launch_bounds__(NT, (NT == 128 ? 6 : NT == 256 ? 4 : NT == 512
     const int e0 = 4 * q;
     const float val[4] = {v4.x, v4.y, v4.z, v4.w};
     const int col = static_cast<int>(c0) + e0;
-    // The kept entries are staged in the chunk's own float4 slots (every lane
-    // has read its slot) with their column offsets, then written out with
+    // The column offsets of the kept entries are staged in column order, then
+    // the entries are read back from the chunk's slots and written out with
     // coalesced stores.
-    float* sval = reinterpret_cast<float*>(s4 + j * NT + warp * 32);
+    const float* sval = reinterpret_cast<const float*>(s4 + j * NT + warp * 32);
     uint8_t* soff = sh.woff[warp];
     __syncwarp();
     {
       uint32_t r = pre;
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
-        if (kp[i]) {
-          sval[r] = val[i];
-          soff[r] = static_cast<uint8_t>(4 * lane + i);
-        }
+        if (kp[i]) soff[r] = static_cast<uint8_t>(4 * lane + i);
         r += kp[i] ? 1u : 0u;
       }
     }
@@ -878,8 +875,9 @@ __global__ void __launch_bounds__(NT, (NT == 128 ? 6 : NT == 256 ? 4 : NT == 512
         if (32u * u < lim) {
           const uint32_t t = 32u * u + lane;
           if (t < lim) {
-            vdst[t] = sval[t];
-            idst[t] = colbase + soff[t];
+            const uint32_t o = soff[t];
+            vdst[t] = sval[o];
+            idst[t] = colbase + static_cast<int>(o);
           }
         }
       }
