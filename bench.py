@@ -64,7 +64,7 @@ def parse_args():
     p.add_argument("--impl", choices=("ours", "reference"), default="ours")
     p.add_argument("--no-operators", action="store_true", help="skip the per-operator table")
     p.add_argument("--no-cpu-baseline", action="store_true")
-    p.add_argument("--branches", type=int, default=5, choices=(1, 2, 3, 5, 9),
+    p.add_argument("--branches", type=int, default=6, choices=(1, 2, 3, 5, 6, 9),
                    help="concurrent streams inside the step graph (1 = all launches in order)")
     return p.parse_args()
 
@@ -404,6 +404,7 @@ BRANCH_OF = {
     2: lambda i, sr: 0 if i < 3 else 1,
     3: lambda i, sr: 0 if i < 3 else 1 + int(sr),
     5: lambda i, sr: i if i < 3 else 3 + int(sr),
+    6: lambda i, sr: i if i < 3 else 3 + (i - 3) // 2,
     9: lambda i, sr: i,
 }
 
@@ -415,6 +416,8 @@ BRANCH_TEXT = {
        "stochastic ones), each in order, forked from and joined into one stream",
     5: "five concurrent branches (each TopK pair; the nearest quantisation pairs; the "
        "stochastic ones), each in order, forked from and joined into one stream",
+    6: "six concurrent branches (each TopK pair; the 2-, 4- and 8-bit quantisation pairs), "
+       "each in order, forked from and joined into one stream",
     9: "nine concurrent branches (one per compress+decompress pair), forked from and joined "
        "into one stream",
 }

@@ -181,3 +181,48 @@ def test_sweep_sampled_rows(mpc, synth, log2n, L):
         assert_bits_equal(sq[rows].cpu().numpy(), os_, "scale b=%d" % bits)
     del x
     torch.cuda.empty_cache()
+
+
+def rel_err(x, y) -> float:
+    x = np.asarray(x, np.float64)
+    y = np.asarray(y, np.float64)
+    return float(np.linalg.norm(x - y) / np.linalg.norm(x))
+
+
+def test_compression_error_norms(mpc, synth):
+    """Relative compression error ||x - x_hat|| / ||x|| (computed in double) of every
+    operator on the CNN boundary: the GPU's within 1e-6 relative of the oracle's (they are
+    bit-identical, so the norms agree exactly), and each one inside the range its
+    operator allows (TopK below the energy of the dropped tail; b-bit quantisation below
+    half a step per entry)."""
+    c = synth.CNN
+    R, L = c["rows"], c["row_len"]
+    x = synth.relu_normal(c["shape"], 3, "cuda").view(R, L)
+    xn = x.cpu().numpy()
+    for p in c["topk_percents"]:
+        k = synth.k_of(L, p)
+        v, i = mpc.mpc_topk_compress(x, k)
+        y = mpc.mpc_topk_decompress(v, i, L)
+        ok(mpc)
+        ov, oi = oracle.topk_compress(xn, k)
+        e_gpu = rel_err(xn, y.cpu().numpy())
+        e_orc = rel_err(xn, oracle.topk_decompress(ov, oi, L))
+        assert abs(e_gpu - e_orc) <= 1e-6 * e_orc
+        # the dropped entries are the L - k smallest magnitudes of each row
+        srt = np.sort(np.abs(xn.astype(np.float64)), axis=1)[:, : L - k]
+        assert abs(e_gpu - np.sqrt((srt ** 2).sum()) / np.linalg.norm(xn.astype(np.float64))) <= 1e-9
+    g = synth.normal((R, L), 77, "cuda", std=1e-3)
+    gn = g.cpu().numpy()
+    for bits in c["bits"]:
+        for sr in (False, True):
+            cq, sq, mq = mpc.mpc_quant_compress(g, bits, stochastic=sr, seed=5)
+            y = mpc.mpc_quant_decompress(cq, sq, mq, L, bits)
+            ok(mpc)
+            oc, os_, om = oracle.quant_compress(gn, bits, sr, 5)
+            e_gpu = rel_err(gn, y.cpu().numpy())
+            e_orc = rel_err(gn, oracle.quant_decompress(oc, os_, om, L, bits))
+            assert abs(e_gpu - e_orc) <= 1e-6 * e_orc
+            # nearest: |x - y| <= scale / 2 (+ rounding); stochastic: < scale
+            bound = (0.5 if not sr else 1.0) * np.asarray(os_, np.float64) * np.sqrt(L) * 1.0001
+            rows = np.linalg.norm(gn.astype(np.float64) - y.cpu().numpy(), axis=1)
+            assert (rows <= bound).all(), "b=%d sr=%d" % (bits, sr)
