@@ -113,9 +113,7 @@ __device__ __forceinline__ int block_max(int v, int* red, int lane, int warp) {
   v = __reduce_max_sync(kFull, v);
   if (lane == 0) red[warp] = v;
   __syncthreads();
-  int r = red[0];
-#pragma unroll
-  for (int i = 1; i < NT / 32; ++i) r = max(r, red[i]);
+  const int r = __reduce_max_sync(kFull, lane < NT / 32 ? red[lane] : red[0]);
   __syncthreads();
   return r;
 }
@@ -125,9 +123,7 @@ __device__ __forceinline__ int block_min(int v, int* red, int lane, int warp) {
   v = __reduce_min_sync(kFull, v);
   if (lane == 0) red[warp] = v;
   __syncthreads();
-  int r = red[0];
-#pragma unroll
-  for (int i = 1; i < NT / 32; ++i) r = min(r, red[i]);
+  const int r = __reduce_min_sync(kFull, lane < NT / 32 ? red[lane] : red[0]);
   __syncthreads();
   return r;
 }
@@ -137,10 +133,9 @@ __device__ __forceinline__ uint32_t block_excl_scan(uint32_t v, uint32_t* red, i
   const uint32_t inc = warp_inclusive_scan(v, lane);
   if (lane == 31) red[warp] = inc;
   __syncthreads();
-  uint32_t base = 0;
-#pragma unroll
-  for (int i = 0; i < NT / 32; ++i)
-    if (i < warp) base += red[i];
+  // the warps' totals, one per lane, scanned: this warp's base is the sum before it
+  const uint32_t t = lane < NT / 32 ? red[lane] : 0u;
+  const uint32_t base = __shfl_sync(kFull, warp_inclusive_scan(t, lane) - t, warp);
   __syncthreads();
   return base + inc - v;
 }
@@ -511,17 +506,13 @@ __global__ void __launch_bounds__(NT, (NT == 128 ? 6 : NT == 256 ? 4 : NT == 512
       const uint32_t incl = warp_inclusive_scan(total, lane);
       if (lane == 31) sh.ured[warp] = incl;
       __syncthreads();
-      // the warp whose groups hold the kr-th entry (every thread finds the same)
-      uint32_t wbase = 0;
-      int ws = NW - 1;
-#pragma unroll
-      for (int w = 0; w < NW; ++w) {
-        const uint32_t u = sh.ured[w];
-        if (ws == NW - 1 && w < NW - 1) {
-          if (wbase + u >= kr) ws = w;
-          else wbase += u;
-        }
-      }
+      // the warp whose groups hold the kr-th entry (every warp finds the same):
+      // a scan of the warps' totals, one per lane
+      const uint32_t wu = lane < NW ? sh.ured[lane] : 0u;
+      const uint32_t wi = warp_inclusive_scan(wu, lane);
+      const unsigned reach = __ballot_sync(kFull, lane < NW - 1 && wi >= kr);
+      const int ws = reach ? __ffs(reach) - 1 : NW - 1;
+      const uint32_t wbase = __shfl_sync(kFull, wi - wu, ws);
       if (warp == ws) {
         // that warp finds the bin, this CTA's entries in it and those of the
         // CTAs before it, and the bin's first and last keys
