@@ -238,21 +238,22 @@ __global__ void __launch_bounds__(32 * kQWarps) quant_warp_kernel(const QuantArg
 // ---------------------------------------------------------------------------
 // Cluster of CTAs per row (or, with a workspace, CTAs over one row's chunks)
 // ---------------------------------------------------------------------------
+template <int NT>
 struct QuantShared {
-  uint32_t redmin[kQNT / 32];
-  uint32_t redmax[kQNT / 32];
+  uint32_t redmin[NT / 32];
+  uint32_t redmax[NT / 32];
   uint32_t mm_min[8];  // per-CTA extrema of the row, pushed by every CTA of the cluster
   uint32_t mm_max[8];
   uint64_t bars[kQNV];  // one per slice chunk
 };
 
-template <int BITS, bool SR>
-__global__ void __launch_bounds__(kQNT) quant_cta_kernel(const QuantArgs a, int spr) {
+template <int BITS, bool SR, int NT>
+__global__ void __launch_bounds__(NT) quant_cta_kernel(const QuantArgs a, int spr) {
   pdl_begin();
-  __shared__ QuantShared sh;
-  __shared__ uint32_t gbuf[BITS == 0 ? (kQNT / 32) * 64 : 1];  // width-b packing, per warp
+  __shared__ QuantShared<NT> sh;
+  __shared__ uint32_t gbuf[BITS == 0 ? (NT / 32) * 64 : 1];  // width-b packing, per warp
   const int bits = BITS == 0 ? a.bits : BITS;
-  extern __shared__ __align__(16) float sx[];  // kQSCAP floats
+  extern __shared__ __align__(16) float sx[];  // 4 x NT x kQNV floats
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const bool from_ws = a.ws != nullptr;
   const uint32_t C = from_ws ? 1u : cluster_size();
@@ -263,20 +264,20 @@ __global__ void __launch_bounds__(kQNT) quant_cta_kernel(const QuantArgs a, int 
   const int n = static_cast<int>(max64(0, min64(a.slice, L - c0)));
   const float* xr = a.x + row * L;
 
-  // The slice arrives in chunks of one float4 per thread (4 x kQNT entries),
+  // The slice arrives in chunks of one float4 per thread (4 x NT entries),
   // each on its own mbarrier and issued by its own lane of warp 0; the
   // extrema are taken chunk by chunk as the chunks land.
   bool failed = false;
-  const int jmax = (n + 4 * kQNT - 1) / (4 * kQNT);
+  const int jmax = (n + 4 * NT - 1) / (4 * NT);
   if (a.aligned && warp == 0 && lane < jmax) {
-    const uint32_t bytes = static_cast<uint32_t>(min(4 * kQNT, n - 4 * kQNT * lane)) * 4u;
+    const uint32_t bytes = static_cast<uint32_t>(min(4 * NT, n - 4 * NT * lane)) * 4u;
     mbar_init(&sh.bars[lane], 1);
     fence_mbar_init();
     mbar_arrive_expect_tx(&sh.bars[lane], bytes);
-    bulk_g2s(sx + 4 * kQNT * lane, xr + c0 + 4 * kQNT * lane, bytes, &sh.bars[lane]);
+    bulk_g2s(sx + 4 * NT * lane, xr + c0 + 4 * NT * lane, bytes, &sh.bars[lane]);
   }
   if (!a.aligned)
-    for (int e = tid; e < n; e += kQNT) sx[e] = xr[c0 + e];
+    for (int e = tid; e < n; e += NT) sx[e] = xr[c0 + e];
   __syncthreads();
   uint32_t kmin = 0xffffffffu, kmax = 0u;
 #pragma unroll
@@ -286,7 +287,7 @@ __global__ void __launch_bounds__(kQNT) quant_cta_kernel(const QuantArgs a, int 
         mbar_wait_bounded(&sh.bars[v], 0, kDrainPolls, nullptr);
         failed = true;
       }
-      const int q = v * kQNT + tid;
+      const int q = v * NT + tid;
       const float4 f = reinterpret_cast<const float4*>(sx)[q];
       const float xs[4] = {f.x, f.y, f.z, f.w};
 #pragma unroll
@@ -318,8 +319,8 @@ __global__ void __launch_bounds__(kQNT) quant_cta_kernel(const QuantArgs a, int 
     }
     __syncthreads();
     if (warp == 0) {
-      uint32_t a0 = lane < kQNT / 32 ? sh.redmin[lane] : 0xffffffffu;
-      uint32_t a1 = lane < kQNT / 32 ? sh.redmax[lane] : 0u;
+      uint32_t a0 = lane < NT / 32 ? sh.redmin[lane] : 0xffffffffu;
+      uint32_t a1 = lane < NT / 32 ? sh.redmax[lane] : 0u;
       a0 = __reduce_min_sync(kFull, a0);
       a1 = __reduce_max_sync(kFull, a1);
       // push this slice's extrema into every CTA of the cluster (itself included)
@@ -346,7 +347,7 @@ __global__ void __launch_bounds__(kQNT) quant_cta_kernel(const QuantArgs a, int 
   if (!failed) {
 #pragma unroll
     for (int v = 0; v < kQNV; ++v) {
-      const int q = v * kQNT + tid;
+      const int q = v * NT + tid;
       const int64_t e0 = 4 * q;  // slice-relative
       const float4 f = reinterpret_cast<const float4*>(sx)[q];
       const float xs[4] = {f.x, f.y, f.z, f.w};
@@ -355,7 +356,7 @@ __global__ void __launch_bounds__(kQNT) quant_cta_kernel(const QuantArgs a, int 
         // start on multiples of 128 entries, so the codes start on a word
         // (this slice owns the words of its entries only: slices start on
         // multiples of 128 entries, so no word is shared with the next one)
-        const int64_t chunk = 128 * (v * (kQNT / 32) + warp);
+        const int64_t chunk = 128 * (v * (NT / 32) + warp);
         if (chunk < nv) {
           float u[4] = {0.f, 0.f, 0.f, 0.f};
           if (SR) uniform4(a.seed, static_cast<uint64_t>(row * L + c0 + e0), u);
@@ -595,6 +596,20 @@ cudaError_t run_quant_warp(const QuantArgs& a, int num_sms, cudaStream_t s) {
                        dim3(32 * kQWarps), 0, s, 0u, a);
 }
 
+// One CTA of NT threads per row, the whole row (<= 4 x NT x kQNV entries) in
+// shared memory.
+template <int BITS, bool SR, int NT>
+cudaError_t run_quant_wide(const QuantArgs& a0, cudaStream_t s) {
+  QuantArgs a = a0;
+  auto kernel = quant_cta_kernel<BITS, SR, NT>;
+  const int smem = 4 * NT * kQNV * 4;
+  cudaError_t err = ensure_dynamic_smem(kernel, smem);
+  if (err != cudaSuccess) return err;
+  a.slice = (a.L + 127) / 128 * 128;
+  if (a.rows > 0x7fffffffLL) return cudaErrorInvalidValue;
+  return launch_kernel(kernel, dim3(static_cast<unsigned>(a.rows)), dim3(NT), smem, s, 1u, a, 1);
+}
+
 template <int BITS, bool SR>
 cudaError_t run_quant_bits(const QuantArgs& a0, int num_sms, cudaStream_t s) {
   QuantArgs a = a0;
@@ -606,7 +621,16 @@ cudaError_t run_quant_bits(const QuantArgs& a0, int num_sms, cudaStream_t s) {
     if (L <= 1024) return run_quant_warp<BITS, 8, SR>(a, num_sms, s);
     return run_quant_warp<BITS, 16, SR>(a, num_sms, s);
   }
-  auto kernel = quant_cta_kernel<BITS, SR>;
+  // Rows of 8193..32768 entries take one wide CTA each (512 threads and two
+  // CTAs per SM up to 16384, else 1024 threads and one per SM) when that
+  // fills the GPU in one wave: the row's extrema then need no cluster barrier.
+  if (a.ws == nullptr && L > kQSCAP && L <= 4 * kQSCAP && a.rows >= num_sms &&
+      a.rows <= 2 * num_sms && L <= 2 * kQSCAP)
+    return run_quant_wide<BITS, SR, 2 * kQNT>(a, s);
+  if (a.ws == nullptr && L > kQSCAP && L <= 4 * kQSCAP && 4 * a.rows >= 3 * num_sms &&
+      a.rows <= num_sms)
+    return run_quant_wide<BITS, SR, 4 * kQNT>(a, s);
+  auto kernel = quant_cta_kernel<BITS, SR, kQNT>;
   const int smem = kQSCAP * 4;
   cudaError_t err = ensure_dynamic_smem(kernel, smem);
   if (err != cudaSuccess) return err;

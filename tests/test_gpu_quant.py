@@ -75,3 +75,17 @@ def test_quant_seed_changes_codes(mpc):
     b = mpc.mpc_quant_compress(x, 4, stochastic=True, seed=1)[0]
     c = mpc.mpc_quant_compress(x, 4, stochastic=True, seed=2)[0]
     assert torch.equal(a, b) and not torch.equal(a, c)
+
+
+# Rows of 8193..32768 entries with enough rows to fill the GPU in one wave take one wide
+# CTA each (512 threads up to 16384 entries, else 1024): every width, both roundings,
+# aligned and unaligned rows, degenerate rows.
+@pytest.mark.parametrize("R,L", [(160, 8193), (160, 16384), (200, 12345), (120, 16385),
+                                 (116, 20001), (128, 32768)])
+def test_quant_wide_rows(mpc, R, L):
+    for kind in ("normal", "relu", "equal"):
+        x = rows_of(kind, R, L, seed=L)
+        for bits in (1, 2, 4, 6, 8, 13, 16, 32):
+            run_both(mpc, x, bits, False, seed=0)
+        for bits in (2, 6, 8):
+            run_both(mpc, x, bits, True, seed=(7 << 32) | L)
