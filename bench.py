@@ -24,7 +24,8 @@ through 8 copies (twice the L2) so that each launch reads cold inputs, and, for
 reference, from single launches between two events (which adds ~5 us to any launch).  `e2e` runs
 the steps through the Python API with the step's inputs copied from pinned host memory
 and two outputs copied back inside the timed region.  `operators` times every operator
-of the path on its own workload.
+of the path on its own workload: a CUDA graph of 8 x (L2 flush, launch) against a graph
+of the 8 flushes alone, the difference divided by 8.
 
 `--impl reference` times the CPU oracle (single-threaded C) on a bounded sample of the
 same step: 16 of the 128 rows.
@@ -763,22 +764,42 @@ def run_e2e(args, st, stream, side, world, device):
             "copies of results on copy streams, pipelined over two slots"}
 
 
-def time_op(fn, stream, flush, reps=5):
-    """Median device time (ms) of fn over reps, L2 flushed before each."""
-    ts = []
+def time_op(fn, stream, flush, reps=8):
+    """Device time (ms) of one launch of fn on cold inputs, inside a CUDA graph: a graph of
+    reps x (L2 flush, launch) against a graph of the reps flushes alone, the difference
+    divided by reps (median of three), so that no event sits next to the launch."""
+    sink = torch.empty((), dtype=torch.int64, device=flush.device)
+
+    def fl():
+        flush.fill_(1)
+        torch.sum(flush.view(torch.int64), dim=0, out=sink)
+
     with torch.cuda.stream(stream):
         fn()
-        for r in range(reps):
-            flush.fill_(r)
-            flush.view(torch.int64).sum()
+        fl()
+        stream.synchronize()
+        g1 = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g1, stream=stream):
+            for _ in range(reps):
+                fl()
+                fn()
+        g0 = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g0, stream=stream):
+            for _ in range(reps):
+                fl()
+
+        def run(g):
+            g.replay()
             a = torch.cuda.Event(enable_timing=True)
             b = torch.cuda.Event(enable_timing=True)
             a.record(stream)
-            fn()
+            g.replay()
             b.record(stream)
             stream.synchronize()
-            ts.append(a.elapsed_time(b))
-    return statistics.median(ts)
+            return a.elapsed_time(b)
+
+        d = [run(g1) - run(g0) for _ in range(3)]
+    return max(statistics.median(d) / reps, 1e-4)
 
 
 def measure_operators(mpc, synth, device, stream, peak):
@@ -871,35 +892,35 @@ def measure_operators(mpc, synth, device, stream, peak):
         for pct in (1, 10, 50):
             ks = synth.k_of(Ls, pct)
             vs, is_ = mpc.mpc_topk_compress(xv, ks)
-            rec("topk_compress 2^28 L=%d K=%d%%" % (Ls, pct), time_op(lambda: mpc.mpc_topk_compress(xv, ks, vs, is_), stream, flush, 3),
+            rec("topk_compress 2^28 L=%d K=%d%%" % (Ls, pct), time_op(lambda: mpc.mpc_topk_compress(xv, ks, vs, is_), stream, flush),
                 algorithmic_bytes(Rs, Ls, k=ks, op="topk"))
             if pct == 10:
                 gvs = mpc.mpc_topk_gather(xv, is_)
-                rec("topk_gather 2^28 L=%d K=10%%" % Ls, time_op(lambda: mpc.mpc_topk_gather(xv, is_, vals=gvs), stream, flush, 3),
+                rec("topk_gather 2^28 L=%d K=10%%" % Ls, time_op(lambda: mpc.mpc_topk_gather(xv, is_, vals=gvs), stream, flush),
                     algorithmic_bytes(Rs, Ls, k=ks, op="topk_gather"))
                 del gvs
                 ys = torch.empty_like(xv)
-                rec("topk_decompress 2^28 L=%d K=10%%" % Ls, time_op(lambda: mpc.mpc_topk_decompress(vs, is_, Ls, y=ys), stream, flush, 3),
+                rec("topk_decompress 2^28 L=%d K=10%%" % Ls, time_op(lambda: mpc.mpc_topk_decompress(vs, is_, Ls, y=ys), stream, flush),
                     algorithmic_bytes(Rs, Ls, k=ks, op="topk_decompress"))
                 es = torch.zeros_like(xv)
-                rec("ef_topk_compress 2^28 L=%d K=10%%" % Ls, time_op(lambda: mpc.mpc_ef_topk_compress(xv, es, ks, vs, is_), stream, flush, 3),
+                rec("ef_topk_compress 2^28 L=%d K=10%%" % Ls, time_op(lambda: mpc.mpc_ef_topk_compress(xv, es, ks, vs, is_), stream, flush),
                     algorithmic_bytes(Rs, Ls, k=ks, op="ef_topk"))
                 del ys, es
             del vs, is_
         for b in BITS + (6,):
             cq, sq, mq = mpc.mpc_quant_compress(xv, b)
-            rec("quant_compress 2^28 L=%d %d-bit" % (Ls, b), time_op(lambda: mpc.mpc_quant_compress(xv, b, codes=cq, scale=sq, minv=mq), stream, flush, 3),
+            rec("quant_compress 2^28 L=%d %d-bit" % (Ls, b), time_op(lambda: mpc.mpc_quant_compress(xv, b, codes=cq, scale=sq, minv=mq), stream, flush),
                 algorithmic_bytes(Rs, Ls, bits=b, op="quant"))
             if b == 6:
                 ys = torch.empty_like(xv)
-                rec("quant_decompress 2^28 L=%d 6-bit" % Ls, time_op(lambda: mpc.mpc_quant_decompress(cq, sq, mq, Ls, 6, y=ys), stream, flush, 3),
+                rec("quant_decompress 2^28 L=%d 6-bit" % Ls, time_op(lambda: mpc.mpc_quant_decompress(cq, sq, mq, Ls, 6, y=ys), stream, flush),
                     algorithmic_bytes(Rs, Ls, bits=6, op="dequant"))
                 del ys
             if b == 4:
-                rec("quant_compress 2^28 L=%d 4-bit stochastic" % Ls, time_op(lambda: mpc.mpc_quant_compress(xv, 4, True, 7, codes=cq, scale=sq, minv=mq), stream, flush, 3),
+                rec("quant_compress 2^28 L=%d 4-bit stochastic" % Ls, time_op(lambda: mpc.mpc_quant_compress(xv, 4, True, 7, codes=cq, scale=sq, minv=mq), stream, flush),
                     algorithmic_bytes(Rs, Ls, bits=4, op="quant"))
                 ys = torch.empty_like(xv)
-                rec("quant_decompress 2^28 L=%d 4-bit" % Ls, time_op(lambda: mpc.mpc_quant_decompress(cq, sq, mq, Ls, 4, y=ys), stream, flush, 3),
+                rec("quant_decompress 2^28 L=%d 4-bit" % Ls, time_op(lambda: mpc.mpc_quant_decompress(cq, sq, mq, Ls, 4, y=ys), stream, flush),
                     algorithmic_bytes(Rs, Ls, bits=4, op="dequant"))
                 del ys
     del xs
