@@ -1282,11 +1282,11 @@ cudaError_t run_mode(const TopkRowArgs& a0, int num_sms, cudaStream_t s) {
   // per SM up to 16384, else 1024 threads and one CTA per SM) when that fills
   // most of the GPU in a single wave: no cluster barriers on the way.  With
   // more rows the smaller clustered CTAs of several waves pack better.
-  if (a.wide_cta && L <= 16384 && a.rows >= num_sms && a.rows <= 2 * num_sms) {
+  if (a.wide_cta && L > 8192 && L <= 16384 && a.rows >= num_sms && a.rows <= 2 * num_sms) {
     a.slice = (L + 3) / 4 * 4;
     return run_cta_any<MODE, 512, 16384>(a, 1, s);
   }
-  if (a.wide_cta && L <= 32768 && 4 * a.rows >= 3 * num_sms && a.rows <= num_sms) {
+  if (a.wide_cta && L > 8192 && L <= 32768 && 4 * a.rows >= 3 * num_sms && a.rows <= num_sms) {
     a.slice = (L + 3) / 4 * 4;
     return run_cta_any<MODE, 1024, 32768>(a, 1, s);
   }

@@ -177,7 +177,8 @@ def test_long_row_decompress_tiles(mpc):
 
 # Rows of 8193..32768 entries with enough rows to fill the GPU take one wide CTA each
 # (512 threads up to 16384 entries, else 1024); the knob value 3 keeps them on clusters.
-WIDE = [(160, 8193), (160, 12345), (160, 16384), (120, 16385), (116, 20000), (120, 32768)]
+WIDE = [(160, 8192), (160, 8193), (160, 12345), (160, 16384), (120, 16385), (116, 20000),
+        (120, 32768), (300, 9000)]
 
 
 @pytest.mark.parametrize("R,L", WIDE)
