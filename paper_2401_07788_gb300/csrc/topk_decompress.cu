@@ -95,17 +95,17 @@ __global__ void __launch_bounds__(kDecThreads)
 
 // Rows of up to 65536 entries: a CTA owns either whole rows [r0, r0 + nrows)
 // (rpc rows, rpc * row_len <= kRowsPerCta) or the column range
-// [part * width, part * width + width) of one row (ppr parts per row).  It
-// zero-fills its region, then stores the kept values that fall in it; a part
-// reads its row's whole payload (from L2 after the first part) and keeps its
-// own, with 16-byte loads several deep so the payload costs few round trips.
+// [part * pw, part * pw + pw) of one row (ppr parts per row).  It zero-fills
+// its region, then stores the kept values that fall in it; a part brackets
+// its own payload entries with one round of probes of the row's ascending
+// indices and reads that range with 16-byte loads several deep.
 constexpr int64_t kRowsPerCta = 16384;
 constexpr int64_t kPartWidth = 8192;
 
 __global__ void __launch_bounds__(kDecThreads)
     topk_decompress_rows_kernel(const float* __restrict__ vals, const int32_t* __restrict__ idx,
                                 int64_t rows, int64_t L, int64_t k, float* __restrict__ y,
-                                int64_t rpc, int64_t ppr, int aligned, int vec) {
+                                int64_t rpc, int64_t ppr, int64_t pw, int aligned, int vec) {
   pdl_begin();
   const int tid = threadIdx.x;
   int64_t r0, nrows, c0, ncols;
@@ -117,8 +117,8 @@ __global__ void __launch_bounds__(kDecThreads)
   } else {
     r0 = blockIdx.x / ppr;
     nrows = 1;
-    c0 = (blockIdx.x % ppr) * kPartWidth;
-    ncols = min64(kPartWidth, L - c0);
+    c0 = (blockIdx.x % ppr) * pw;
+    ncols = min64(pw, L - c0);
   }
   float* dst = y + r0 * L + c0;
   if (ppr == 1) {
@@ -147,11 +147,25 @@ __global__ void __launch_bounds__(kDecThreads)
   const uint32_t k32 = static_cast<uint32_t>(k);
   const float* vr = vals + e_begin;
   const int32_t* ir = idx + e_begin;
+  // A part of a long row needs the payload entries of its columns only: one
+  // round of evenly spaced probes of the ascending indices brackets them (to
+  // within one probe spacing each side; the column test drops the rest).
+  uint32_t e_lo = 0, e_hi = nk;
+  if (ppr > 1 && nk >= 4 * kDecThreads) {
+    const uint32_t stride = (nk + kDecThreads - 1) / kDecThreads;
+    const uint32_t p = static_cast<uint32_t>(tid) * stride;
+    const bool in = p < nk;
+    const int64_t v = in ? static_cast<int64_t>(ir[p]) : 0;
+    const uint32_t c_lo = static_cast<uint32_t>(__syncthreads_count(in && v < c0));
+    const uint32_t c_hi = static_cast<uint32_t>(__syncthreads_count(in && v < c0 + ncols));
+    e_lo = c_lo > 0 ? (c_lo - 1) * stride : 0u;
+    e_hi = min(nk, c_hi * stride);
+  }
   if (vec) {
     // 4 entries per 16-byte load, kU loads in flight per thread
     constexpr int kU = 4;
-    const uint32_t n4 = nk / 4;
-    for (uint32_t b = tid; b < n4; b += kDecThreads * kU) {
+    const uint32_t n4 = min(nk / 4, (e_hi + 3) / 4);
+    for (uint32_t b = e_lo / 4 + tid; b < n4; b += kDecThreads * kU) {
       int4 iv[kU];
       float4 fv[kU];
 #pragma unroll
@@ -178,13 +192,13 @@ __global__ void __launch_bounds__(kDecThreads)
         }
       }
     }
-    for (uint32_t e = 4 * n4 + tid; e < nk; e += kDecThreads) {
+    for (uint32_t e = 4 * (nk / 4) + tid; e < e_hi; e += kDecThreads) {
       const uint32_t lr = (ppr == 1) ? e / k32 : 0u;
       const int64_t col = static_cast<int64_t>(ir[e]) - c0;
       if (col >= 0 && col < ncols) dst[static_cast<int64_t>(lr) * L + col] = vr[e];
     }
   } else {
-    for (uint32_t e = tid; e < nk; e += kDecThreads) {
+    for (uint32_t e = e_lo + tid; e < e_hi; e += kDecThreads) {
       const uint32_t lr = (ppr == 1) ? e / k32 : 0u;
       const int64_t col = static_cast<int64_t>(ir[e]) - c0;
       if (col >= 0 && col < ncols) dst[static_cast<int64_t>(lr) * L + col] = vr[e];
@@ -276,10 +290,9 @@ __global__ void __launch_bounds__(kDecThreads)
 cudaError_t launch_topk_decompress(const float* vals, const int32_t* idx, int64_t rows,
                                    int64_t L, int64_t k, float* y, int aligned, int num_sms,
                                    cudaStream_t s) {
-  (void)num_sms;
   if (rows <= 0) return cudaSuccess;
   if (L <= 65536) {
-    int64_t rpc = 1, ppr = 1, blocks;
+    int64_t rpc = 1, ppr = 1, pw = kPartWidth, blocks;
     if (L <= kRowsPerCta) {
       rpc = max64(1, min64(rows, kRowsPerCta / L));
       blocks = (rows + rpc - 1) / rpc;
@@ -287,13 +300,25 @@ cudaError_t launch_topk_decompress(const float* vals, const int32_t* idx, int64_
       ppr = (L + kPartWidth - 1) / kPartWidth;
       blocks = rows * ppr;
     }
+    // Too few blocks for the GPU: rows of 4096 entries or more split into
+    // narrower parts (at least 2048 columns, multiples of 4) up to about two
+    // blocks per SM.
+    if (blocks < 2 * num_sms && L >= 4096) {
+      const int64_t want = min64((L + 2047) / 2048, (2 * num_sms + rows - 1) / rows);
+      if (want > ppr) {
+        rpc = 1;
+        pw = ((L + want - 1) / want + 3) / 4 * 4;
+        ppr = (L + pw - 1) / pw;
+        blocks = rows * ppr;
+      }
+    }
     if (blocks > 0x7fffffffLL) return cudaErrorInvalidValue;
     // 16-byte payload loads when every block's payload range is 16-byte aligned
     const int vec = (k % 4 == 0) && (reinterpret_cast<uintptr_t>(vals) % 16 == 0) &&
                     (reinterpret_cast<uintptr_t>(idx) % 16 == 0);
     return launch_kernel(topk_decompress_rows_kernel, dim3(static_cast<unsigned>(blocks)),
-                         dim3(kDecThreads), 0, s, 0u, vals, idx, rows, L, k, y, rpc, ppr, aligned,
-                         vec);
+                         dim3(kDecThreads), 0, s, 0u, vals, idx, rows, L, k, y, rpc, ppr, pw,
+                         aligned, vec);
   }
   int64_t rpc = 1, tpr = 1, blocks;
   if (L <= kTile) {
