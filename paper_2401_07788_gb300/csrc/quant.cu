@@ -179,7 +179,7 @@ __device__ __forceinline__ void store_codes_any(uint64_t piece, int bits, int la
 // One warp per row
 // ---------------------------------------------------------------------------
 template <int BITS, int NVW, bool SR>
-__global__ void __launch_bounds__(32 * kQWarps) quant_warp_kernel(const QuantArgs a) {
+__global__ void __launch_bounds__(32 * kQWarps, NVW <= 8 ? 4 : 2) quant_warp_kernel(const QuantArgs a) {
   pdl_begin();
   __shared__ uint32_t gbuf[BITS == 0 ? kQWarps * 64 : 1];  // width-b packing, per warp
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
