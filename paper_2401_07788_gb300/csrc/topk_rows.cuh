@@ -924,11 +924,20 @@ __device__ __forceinline__ float* state_row(const TopkRowArgs& a, int64_t row, b
   return a.aux + srow * a.L;
 }
 
+// Rows staged per row buffer of the warp kernel: x, plus the err / state row
+// except for rows of 513..768 entries (NVW 6), where that row is read through
+// L2 (measured: with it staged one CTA fits an SM and the kernel runs ~25 %
+// slower; for other lengths the staged row is faster).
+__host__ __device__ constexpr int warp_row_buffers(int mode, int nvw) { return (mode == kPlain || nvw == 6) ? 1 : 2; }
+
 template <int MODE, int NVW, int WPC, bool FULL>
 __global__ void __launch_bounds__(32 * WPC) topk_warp_kernel(const TopkRowArgs a) {
   pdl_begin();
   constexpr int RCAP = 128 * NVW;
-  constexpr int NBUF = (MODE == kPlain) ? 1 : 2;  // x (+ err / state) per row
+  // x, and the err / state row, are staged per row in the warp's buffers;
+  // rows of 513..768 entries instead prefetch the err / state row into L2 and
+  // read it from there: staged, it would leave room for one CTA per SM
+  constexpr int NBUF = warp_row_buffers(MODE, NVW);
   __shared__ WarpShared wsh[WPC];
   extern __shared__ __align__(16) float dyn[];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -959,7 +968,10 @@ __global__ void __launch_bounds__(32 * WPC) topk_warp_kernel(const TopkRowArgs a
       fence_proxy_async_smem();
       mbar_arrive_expect_tx(&sh.bar[b], bytes * NBUF);
       bulk_g2s(buf, a.x + r * L, bytes, &sh.bar[b]);
-      if (MODE != kPlain) bulk_g2s(buf + RCAP, ar, bytes, &sh.bar[b]);
+      if (MODE != kPlain) {
+        if (NBUF == 2) bulk_g2s(buf + RCAP, ar, bytes, &sh.bar[b]);
+        else bulk_prefetch_l2(ar, bytes);
+      }
     }
     return true;
   };
@@ -982,7 +994,6 @@ __global__ void __launch_bounds__(32 * WPC) topk_warp_kernel(const TopkRowArgs a
       continue;
     }
     float* xs = wbase + b * (RCAP * NBUF);
-    float* as = xs + RCAP;
     if (a.aligned) {
       const uint32_t par = (phases >> b) & 1u;
       const bool got = mbar_wait_bounded(&sh.bar[b], par, a.spin_limit, a.status);
@@ -998,12 +1009,22 @@ __global__ void __launch_bounds__(32 * WPC) topk_warp_kernel(const TopkRowArgs a
       const float* xrow = a.x + row * L;
       for (int e = lane; e < n; e += 32) {
         xs[e] = xrow[e];
-        if (MODE != kPlain) as[e] = arow[e];
+        if (MODE != kPlain && NBUF == 2) xs[RCAP + e] = arow[e];
       }
       __syncwarp();
     }
     float4* x4 = reinterpret_cast<float4*>(xs);
-    const float4* a4 = reinterpret_cast<const float4*>(as);
+    // the err / state entries 4q..4q+3 of this row (+0 past its end), from the
+    // staged copy or through L2
+    auto aux4 = [&](int q) -> float4 {
+      if (NBUF == 2) return reinterpret_cast<const float4*>(xs + RCAP)[q];
+      const int e0 = 4 * q;
+      if (a.aligned && (FULL || e0 + 4 <= n)) return *reinterpret_cast<const float4*>(arow + e0);
+      float t[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) t[i] = (e0 + i < n) ? arow[e0 + i] : 0.0f;
+      return make_float4(t[0], t[1], t[2], t[3]);
+    };
 
     // ---- ranked values (in place), the largest finite magnitude, any NaN -------
     int kmax = -1, kall = -1;
@@ -1012,7 +1033,7 @@ __global__ void __launch_bounds__(32 * WPC) topk_warp_kernel(const TopkRowArgs a
       const int q = v * 32 + lane;
       float4 val = x4[q];
       if (MODE != kPlain) {
-        val = ranked4<MODE>(val, a4[q]);
+        val = ranked4<MODE>(val, aux4(q));
         x4[q] = val;
       }
       int kk[4];
@@ -1181,7 +1202,7 @@ __global__ void __launch_bounds__(32 * WPC) topk_warp_kernel(const TopkRowArgs a
         const float val[4] = {v4.x, v4.y, v4.z, v4.w};
         float st[4] = {0.f, 0.f, 0.f, 0.f};
         if (MODE == kDelta) {
-          const float4 sv = a4[q];
+          const float4 sv = aux4(q);
           st[0] = sv.x;
           st[1] = sv.y;
           st[2] = sv.z;
@@ -1221,7 +1242,7 @@ __global__ void __launch_bounds__(32 * WPC) topk_warp_kernel(const TopkRowArgs a
 template <int MODE, int NVW, bool FULL>
 cudaError_t run_warp(const TopkRowArgs& a, int num_sms, cudaStream_t s) {
   // Eight warps per CTA, four when a warp's two row buffers exceed 12 KiB.
-  constexpr int NBUF = (MODE == kPlain) ? 1 : 2;
+  constexpr int NBUF = warp_row_buffers(MODE, NVW);
   constexpr int WBYTES = 2 * 128 * NVW * 4 * NBUF;
   constexpr int WPC = WBYTES > 12 * 1024 ? 4 : 8;
   auto kernel = topk_warp_kernel<MODE, NVW, WPC, FULL>;
