@@ -66,6 +66,9 @@ def parse_args():
     p.add_argument("--impl", choices=("ours", "reference"), default="ours")
     p.add_argument("--no-operators", action="store_true", help="skip the per-operator table")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--sweep", action="store_true",
+                   help="only the size sweep: N = 2^20..2^30 entries, L in {768, 4096, 65536, N}; "
+                        "prints one JSON line with the table (not the benchmark line)")
     p.add_argument("--branches", type=int, default=6, choices=(1, 2, 3, 5, 6, 9),
                    help="concurrent streams inside the step graph (1 = all launches in order)")
     return p.parse_args()
@@ -822,6 +825,13 @@ def measure_operators(mpc, synth, device, stream, peak):
         algorithmic_bytes(32, 16384, k=k, op="topk"))
     rec("topk_decompress 32x16384 K=10%", time_op(lambda: mpc.mpc_topk_decompress(v, i, 16384, y=y), stream, flush),
         algorithmic_bytes(32, 16384, k=k, op="topk_decompress"))
+    g1 = synth.normal((32, 16384), 1, device, std=1e-3)
+    c1, s1, m1 = mpc.mpc_quant_compress(g1, 8)
+    rec("quant_compress 32x16384 8-bit", time_op(lambda: mpc.mpc_quant_compress(g1, 8, codes=c1, scale=s1, minv=m1), stream, flush),
+        algorithmic_bytes(32, 16384, bits=8, op="quant"))
+    rec("quant_decompress 32x16384 8-bit", time_op(lambda: mpc.mpc_quant_decompress(c1, s1, m1, 16384, 8, y=y), stream, flush),
+        algorithmic_bytes(32, 16384, bits=8, op="dequant"))
+    del g1
     # index reuse at the CNN stage boundary: gradient values at the activation's Top10%
     xg = synth.relu_normal((R, L), 3, device)
     gg = synth.normal((R, L), 4, device, std=1e-3)
@@ -1014,11 +1024,76 @@ def run_reference(args, rank, world):
     print(json.dumps(line), flush=True)
 
 
+def run_sweep():
+    """The size sweep of the bandwidth study: N = 2^20..2^30 N(0,1) entries as rows of
+    L in {768, 4096, 65536, N} (N itself only up to 2^26, the on-chip row path's reach
+    being 65536 and the grid path's workspace growing with the row); TopK and EF-TopK at
+    K = 1, 10, 50 %, 2/4/8-bit quantisation and 4-bit dequantisation, each launch timed
+    inside a CUDA graph on cold inputs as in `operators`."""
+    import paper_2401_07788_gb300 as mpc
+    from paper_2401_07788_gb300 import synth
+
+    device = torch.device("cuda", 0)
+    torch.cuda.set_device(device)
+    stream = torch.cuda.Stream(device)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=device)
+    peak, _ = hbm_peak()
+    table = []
+    for log2n in range(20, 31):
+        N = 1 << log2n
+        xs = synth.normal((N,), log2n, device)
+        for Ls in (768, 4096, 65536) + ((N,) if log2n <= 26 else ()):
+            Rs = N // Ls
+            if Rs < 1:
+                continue
+            xv = xs[: Rs * Ls].view(Rs, Ls)
+            entries = []
+            for pct in (1, 10, 50):
+                ks = synth.k_of(Ls, pct)
+                vs, is_ = mpc.mpc_topk_compress(xv, ks)
+                ws = None
+                need = mpc.mpc_topk_workspace_bytes(Rs, Ls, ks)
+                if need:
+                    ws = torch.empty(need, dtype=torch.uint8, device=device)
+                entries.append(("topk K=%d%%" % pct, time_op(lambda: mpc.mpc_topk_compress(xv, ks, vs, is_, ws=ws), stream, flush),
+                                algorithmic_bytes(Rs, Ls, k=ks, op="topk")))
+                es = torch.zeros_like(xv)
+                entries.append(("ef_topk K=%d%%" % pct, time_op(lambda: mpc.mpc_ef_topk_compress(xv, es, ks, vs, is_, ws=ws), stream, flush),
+                                algorithmic_bytes(Rs, Ls, k=ks, op="ef_topk")))
+                del es, vs, is_, ws
+            for b in ((2, 4, 8) if Ls <= 0x7fffffff // 32 else ()):  # the quantiser's row limit
+                cq, sq, mq = mpc.mpc_quant_compress(xv, b)
+                entries.append(("quant %d-bit" % b, time_op(lambda: mpc.mpc_quant_compress(xv, b, codes=cq, scale=sq, minv=mq), stream, flush),
+                                algorithmic_bytes(Rs, Ls, bits=b, op="quant")))
+                if b == 4:
+                    ys = torch.empty_like(xv)
+                    entries.append(("dequant 4-bit", time_op(lambda: mpc.mpc_quant_decompress(cq, sq, mq, Ls, 4, y=ys), stream, flush),
+                                    algorithmic_bytes(Rs, Ls, bits=4, op="dequant")))
+                    del ys
+                del cq, sq, mq
+            for name, ms, nbytes in entries:
+                gbs = nbytes / (ms / 1e3) / 1e9
+                table.append({"log2n": log2n, "row_len": Ls, "op": name, "us": round(ms * 1e3, 2),
+                              "GBps": round(gbs, 1), "frac": round(gbs / peak, 4)})
+        del xs
+        torch.cuda.empty_cache()
+    st = mpc.mpc_get_status(stream)
+    if st != 0:
+        raise RuntimeError("device status %d: %s" % (st, mpc.mpc_last_error()))
+    print(json.dumps({"sweep": table, "peak": peak, "unit": "GB/s", "timing": "each launch "
+                      "inside a CUDA graph on cold inputs (flush-and-launch graph against a "
+                      "flush-only graph)"}), flush=True)
+
+
 def main():
     args = parse_args()
     rank, local, world = dist_env()
     if args.impl == "reference":
         run_reference(args, rank, world)
+        return
+    if args.sweep:
+        if rank == 0:
+            run_sweep()
         return
     run_ours(args, rank, local, world)
     if world > 1:
