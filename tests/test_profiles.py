@@ -1,0 +1,38 @@
+"""The committed ncu traffic table that bench.py reads for roofline.traffic: it parses,
+names a source digest, and holds a per-launch DRAM figure for every operator of the
+benchmark step (no GPU needed)."""
+
+import importlib.util
+import os
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _bench():
+    spec = importlib.util.spec_from_file_location("bench", os.path.join(ROOT, "bench.py"))
+    mod = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(mod)
+    return mod
+
+
+def test_traffic_table_parses():
+    lines = open(os.path.join(ROOT, "profiles", "dram_traffic.txt")).read().splitlines()
+    digests = [ln.split()[1] for ln in lines if ln.startswith("source_digest ")]
+    assert len(digests) == 1 and len(digests[0]) == 16
+    entries = {ln.split()[0]: float(ln.split()[1]) for ln in lines
+               if ln.strip() and not ln.startswith("#") and not ln.startswith("source_digest")}
+    b = _bench()
+    kern = lambda o: ("topk_cta_kernel" if "topk_compress" in o else  # noqa: E731
+                      "topk_decompress_rows_kernel" if "decompress K" in o else
+                      "quant_cta_kernel" if "quant_compress" in o else "dequant_rows_kernel")
+    ops = ["ef_topk_compress K=%d%%" % p for p in b.TOPK_PCTS]
+    ops += ["topk_decompress K=%d%%" % p for p in b.TOPK_PCTS]
+    for bits in b.BITS:
+        for sr in ("nearest", "stochastic"):
+            ops += ["quant_compress %d-bit %s" % (bits, sr), "quant_decompress %d-bit %s" % (bits, sr)]
+    for o in ops:
+        key = kern(o) + ":" + o.replace(" ", "_")
+        assert key in entries and entries[key] > 0, key
+    # inputs read once: an error-feedback TopK launch reads x and err, 2 x 16.8 MB
+    ef = entries["topk_cta_kernel:ef_topk_compress_K=5%"]
+    assert 2 * 4 * b.R * b.L * 0.99 <= ef <= 2 * 4 * b.R * b.L * 1.05
