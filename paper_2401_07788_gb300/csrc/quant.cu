@@ -465,18 +465,49 @@ __global__ void __launch_bounds__(256)
 // Rows with a 16-byte aligned output and L % 4 == 0: every thread writes whole
 // float4s, consecutive lanes consecutive float4s (512-byte warp stores), from
 // the one code word that holds their 4 codes; bpr blocks per row, kDqU float4
-// per thread.
+// per thread.  Short rows (rpb > 1): a block covers rpb whole rows, its
+// 256 x kDqU slots laid over them in order, the row of a slot found by the
+// exact product (slot * rmul) >> 20 (slot < 1024 and n4 <= 512).
 constexpr int kDqU = 4;
 
 template <int BITS>
 __global__ void __launch_bounds__(256)
     dequant_rows_kernel(const uint32_t* __restrict__ codes, const float* __restrict__ scale,
                         const float* __restrict__ minv, int64_t L, int64_t W, int bpr,
-                        float* __restrict__ y) {
+                        float* __restrict__ y, int64_t rows, int rpb, uint32_t rmul) {
   pdl_begin();
+  const int64_t n4 = L / 4;
+  if (rpb > 1) {
+    const int64_t r0 = static_cast<int64_t>(blockIdx.x) * rpb;
+    const uint32_t slots = static_cast<uint32_t>(min64(rpb, rows - r0) * n4);
+    uint32_t w[kDqU];
+    int64_t rr[kDqU];
+    int64_t ff[kDqU];
+#pragma unroll
+    for (int u = 0; u < kDqU; ++u) {
+      const uint32_t t = u * 256 + threadIdx.x;
+      const uint32_t ri = (t * rmul) >> 20;
+      rr[u] = r0 + ri;
+      ff[u] = t - static_cast<int64_t>(ri) * n4;
+      w[u] = (t < slots) ? codes[rr[u] * W + ((ff[u] * 4 * BITS) >> 5)] : 0u;
+    }
+#pragma unroll
+    for (int u = 0; u < kDqU; ++u) {
+      const uint32_t t = u * 256 + threadIdx.x;
+      if (t < slots) {
+        const float sc = scale[rr[u]], m = minv[rr[u]];
+        const uint32_t word = w[u] >> ((ff[u] * 4 * BITS) & 31);
+        float o[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+          o[q] = fadd(m, fmul(static_cast<float>((word >> (BITS * q)) & ((1u << BITS) - 1u)), sc));
+        reinterpret_cast<float4*>(y + rr[u] * L)[ff[u]] = make_float4(o[0], o[1], o[2], o[3]);
+      }
+    }
+    return;
+  }
   const int64_t row = blockIdx.x / bpr;
   const int64_t f0 = static_cast<int64_t>(blockIdx.x % bpr) * (256 * kDqU);
-  const int64_t n4 = L / 4;
   const uint32_t* cr = codes + row * W;
   float4* yr = reinterpret_cast<float4*>(y + row * L);
   const float sc = scale[row], m = minv[row];
@@ -561,10 +592,22 @@ void launch_dequant(const uint32_t* codes, const float* scale, const float* minv
                     int64_t L, int64_t W, int64_t wpr, float* y, int aligned, unsigned grid,
                     cudaStream_t s) {
   if (aligned && L % 4 == 0) {
-    const int64_t bpr = (L / 4 + 256 * kDqU - 1) / (256 * kDqU);
+    const int64_t n4 = L / 4;
+    if (n4 <= 128 * kDqU) {
+      // short rows: whole rows per block
+      const int64_t rpb = (256 * kDqU) / n4;
+      const int64_t blocks = (rows + rpb - 1) / rpb;
+      const uint32_t rmul = static_cast<uint32_t>(((int64_t{1} << 20) + n4 - 1) / n4);
+      if (blocks < 0x7fffffffLL) {
+        launch_kernel(dequant_rows_kernel<BITS>, dim3(static_cast<unsigned>(blocks)), dim3(256), 0,
+                      s, 0u, codes, scale, minv, L, W, 1, y, rows, static_cast<int>(rpb), rmul);
+        return;
+      }
+    }
+    const int64_t bpr = (n4 + 256 * kDqU - 1) / (256 * kDqU);
     if (bpr > 0 && rows * bpr < 0x7fffffffLL) {
       launch_kernel(dequant_rows_kernel<BITS>, dim3(static_cast<unsigned>(rows * bpr)), dim3(256), 0,
-                    s, 0u, codes, scale, minv, L, W, static_cast<int>(bpr), y);
+                    s, 0u, codes, scale, minv, L, W, static_cast<int>(bpr), y, rows, 1, 0u);
       return;
     }
   }
