@@ -36,3 +36,20 @@ def test_traffic_table_parses():
     # inputs read once: an error-feedback TopK launch reads x and err, 2 x 16.8 MB
     ef = entries["topk_cta_kernel:ef_topk_compress_K=5%"]
     assert 2 * 4 * b.R * b.L * 0.99 <= ef <= 2 * 4 * b.R * b.L * 1.05
+
+
+def test_step_branch_layouts():
+    """Every concurrent-branch layout of the benchmark step puts each of its nine pairs on
+    a branch that exists, keeps a pair's two launches together (one branch per pair) and
+    uses every branch; one branch is the launches in order."""
+    b = _bench()
+    for nb, f in b.BRANCH_OF.items():
+        got = []
+        for i in range(9):
+            sr = None if i < 3 else bool((i - 3) % 2)
+            br = f(i, sr)
+            assert 0 <= br < nb, (nb, i, br)
+            got.append(br)
+        assert sorted(set(got)) == list(range(nb)), (nb, got)
+        assert nb in b.BRANCH_TEXT
+    assert set(b.BRANCH_OF[1](i, None if i < 3 else False) for i in range(9)) == {0}
