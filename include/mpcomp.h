@@ -10,7 +10,7 @@
  * Conventions for every entry point
  * ---------------------------------
  *  - Tensors are row-major fp32 matrices [rows][row_len]; each operator acts on
- *    every row independently (the paper's "input vector", §2.2, §2.3).
+ *    every row independently (the vector the paper compresses, §2.2, §2.3).
  *  - Every pointer argument is CUDA device memory owned by the caller, except
  *    where a comment says otherwise.  The library allocates no device memory.
  *  - Every call is asynchronous on `stream` (a cudaStream_t; NULL = legacy
@@ -76,8 +76,8 @@ int mpc_version(void);
  * multi-pass path that keeps counters and candidates in the workspace. */
 size_t mpc_topk_workspace_bytes(int64_t rows, int64_t row_len, int64_t k);
 
-/* TopK compress (§2.3: "selects the largest K% values (in absolute value)
- * from the input vector").
+/* TopK compress (§2.3: keep the K% entries of each row with the largest
+ * magnitudes).
  *   x     [rows][row_len] fp32, read only.
  *   k     entries kept per row, 1 <= k <= row_len (the caller turns K% into k).
  *   vals  [rows][k] fp32, out;  idx [rows][k] int32, out (ascending per row).
@@ -88,7 +88,8 @@ mpc_status mpc_topk_compress(const float* x, int64_t rows, int64_t row_len, int6
                              float* vals, int32_t* idx, void* ws, size_t ws_bytes,
                              mpc_stream_t stream);
 
-/* TopK decompress (§2.3: "setting other values to zero"):
+/* TopK decompress (§2.3: the kept values back at their columns, zero
+ * elsewhere):
  *   y [rows][row_len] = +0 everywhere except y[r][idx[r][i]] = vals[r][i].
  * idx must be strictly ascending in each row and within [0, row_len) (as
  * produced by the compress calls); entries that are not are skipped, never
@@ -119,9 +120,9 @@ mpc_status mpc_ef_topk_compress(const float* x, float* err, int64_t rows, int64_
                                 int64_t k, float* vals, int32_t* idx, void* ws,
                                 size_t ws_bytes, mpc_stream_t stream);
 
-/* EF-mixed TopK (§2.4: "the largest K/2% values from the input vector X and
- * K/2% of the current error buffer", then "the input vector and buffer are
- * added and sent, resulting in the same K% non-zero values").  Reading: the
+/* EF-mixed TopK (§2.4: half of the K% budget goes to the largest entries of
+ * the input and half to the largest of the error buffer; input and buffer are
+ * summed and sent on those K% positions).  Reading: the
  * input's share is its ceil(k/2) largest |x|; the buffer's share is its
  * floor(k/2) largest |err| among the entries the input's share did not take
  * (so exactly k entries are sent); ties go to the lower index.  Then
@@ -190,8 +191,8 @@ size_t mpc_quant_codes_words(int64_t rows, int64_t row_len, int bits);
  * single-pass kernel handles). */
 size_t mpc_quant_workspace_bytes(int64_t rows, int64_t row_len, int bits);
 
-/* Quantise (§2.2: "mapped to [0;1] interval with min-max scaling and then
- * quantized"), per row, with L = 2^bits - 1:
+/* Quantise (§2.2: each row scaled to [0, 1] by its minimum and maximum, then
+ * rounded to one of 2^bits levels), per row, with L = 2^bits - 1:
  *   mn, mx = row minimum and maximum (-0 ordered below +0);
  *   scale = (mx - mn) / L;  inv = L / (mx - mn);  t = (x - mn) * inv;
  *   q = clamp(round_half_even(t), 0, L)            (MPC_ROUND_NEAREST) or
@@ -211,8 +212,8 @@ mpc_status mpc_quant_compress(const float* x, int64_t rows, int64_t row_len, int
                               float* scale, float* minv, void* ws, size_t ws_bytes,
                               mpc_stream_t stream);
 
-/* Dequantise (§2.2: "Decompression transforms these values back to original
- * scale"): y = minv + float(q) * scale, two fp32 round-to-nearest operations
+/* Dequantise (§2.2: the codes mapped back to the row's original range):
+ * y = minv + float(q) * scale, two fp32 round-to-nearest operations
  * (bits = 32: y = the raw bits). */
 mpc_status mpc_quant_decompress(const uint32_t* codes, const float* scale,
                                 const float* minv, int64_t rows, int64_t row_len, int bits,

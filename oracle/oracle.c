@@ -108,8 +108,8 @@ void orc_topk_compress(const float* x, int64_t rows, int64_t row_len, int64_t k,
     free(work);
 }
 
-/* "setting other values to zero": a dense row of +0 with the kept values put
- * back at their indices. */
+/* Decompression (§2.3): a dense row of +0 with the kept values put back at
+ * their indices. */
 void orc_topk_decompress(const float* vals, const int32_t* idx, int64_t rows,
                          int64_t row_len, int64_t k, float* y)
 {
@@ -366,7 +366,7 @@ void orc_quant_compress(const float* x, int64_t rows, int64_t row_len, int bits,
     }
 }
 
-/* "Decompression transforms these values back to original scale":
+/* Decompression (§2.2), the codes mapped back to the row's range:
  * y = min + q * scale. */
 void orc_quant_decompress(const uint32_t* codes, const float* scale, const float* minv,
                           int64_t rows, int64_t row_len, int bits, float* y)
