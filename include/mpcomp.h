@@ -52,7 +52,7 @@ typedef struct CUstream_st* mpc_stream_t;
 typedef enum {
     MPC_OK = 0,
     MPC_ERR_INVALID_ARG = 1, /* bad size, null or misaligned pointer, bad enum */
-    MPC_ERR_UNSUPPORTED = 2, /* valid request this build does not implement */
+    MPC_ERR_UNSUPPORTED = 2, /* valid request the library does not implement */
     MPC_ERR_WORKSPACE = 3,   /* workspace missing or smaller than required */
     MPC_ERR_CUDA = 4,        /* a CUDA runtime call or launch failed */
     MPC_ERR_TIMEOUT = 5,     /* a device-side wait gave up (see mpc_get_status) */
