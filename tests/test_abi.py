@@ -109,3 +109,32 @@ def test_knobs(lib):
     assert lib.mpc_set_knob(3, 2) == 1  # programmatic dependent launch: 0 or 1
     assert lib.mpc_set_knob(3, 0) == 0
     assert lib.mpc_set_knob(3, 1) == 0
+
+
+def test_aqsgd_quant_validation(lib):
+    p = ctypes.c_void_p(0x1000)
+    q = ctypes.c_void_p(0x100000)
+
+    def comp(num_samples=10, ids=p, n_ids=2, rps=3, L=16, bits=4, mode=0, ws=q, ws_bytes=1 << 20):
+        return lib.mpc_aqsgd_quant_compress(p, p, num_samples, ids, n_ids, rps, L, bits, mode, 0,
+                                            p, p, p, ws, ws_bytes, None)
+
+    # the workspace holds d (rows x row_len fp32, rounded up to 256 bytes), plus the
+    # quantiser's own for rows longer than its on-chip path
+    assert lib.mpc_aqsgd_quant_workspace_bytes(2, 3, 16, 4) == 512  # 6 x 16 x 4 = 384 -> 512
+    assert lib.mpc_aqsgd_quant_workspace_bytes(4, 2, 256, 4) == 8 * 256 * 4
+    assert lib.mpc_aqsgd_quant_workspace_bytes(1, 1, 100000, 4) == 400128 + 8
+    assert lib.mpc_aqsgd_quant_workspace_bytes(2, 3, 16, 17) == 0
+    assert lib.mpc_aqsgd_quant_workspace_bytes(0, 3, 16, 4) == 0
+    assert comp(bits=17) == 1 and comp(bits=0) == 1
+    assert comp(mode=7) == 1
+    assert comp(num_samples=0) == 1 and comp(rps=0) == 1 and comp(n_ids=-1) == 1
+    assert comp(ids=ctypes.c_void_p(0x1004)) == 1       # sample ids misaligned
+    assert comp(ws=None) == 3 and comp(ws_bytes=255) == 3  # workspace missing or short
+    assert comp(n_ids=0, ws=None, ws_bytes=0) == 0      # nothing to do
+    dec = lambda **kw: lib.mpc_aqsgd_quant_decompress(  # noqa: E731
+        p, p, p, p, kw.get("num_samples", 10), kw.get("ids", p), kw.get("n_ids", 2), 3, 16,
+        kw.get("bits", 4), None)
+    assert dec(bits=33) == 1 and dec(num_samples=0) == 1
+    assert dec(ids=ctypes.c_void_p(0x1002)) == 1
+    assert dec(n_ids=0) == 0
