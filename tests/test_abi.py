@@ -138,3 +138,23 @@ def test_aqsgd_quant_validation(lib):
     assert dec(bits=33) == 1 and dec(num_samples=0) == 1
     assert dec(ids=ctypes.c_void_p(0x1002)) == 1
     assert dec(n_ids=0) == 0
+
+
+def test_gather_and_efmix_validation(lib):
+    p = ctypes.c_void_p(0x1000)
+    # index reuse: the payload shape rules of TopK
+    assert lib.mpc_topk_gather(p, 2, 16, p, 0, p, None) == 1      # k = 0
+    assert lib.mpc_topk_gather(p, 2, 16, p, 17, p, None) == 1     # k > row_len
+    assert lib.mpc_topk_gather(None, 2, 16, p, 4, p, None) == 1   # g NULL
+    assert lib.mpc_topk_gather(p, 0, 16, p, 4, p, None) == 0      # no rows
+    # EF-mixed: the two shares' index and saved-value arrays (256-byte rounded) come first
+    k = 7
+    share = -(-(3 * ((k + 1) // 2) * 4) // 256) * 256
+    assert lib.mpc_efmix_workspace_bytes(3, 64, k) >= 2 * share
+    assert lib.mpc_efmix_workspace_bytes(3, 64, 0) == 0
+    need = lib.mpc_efmix_workspace_bytes(3, 64, k)
+    ws = ctypes.c_void_p(0x100000)
+    call = lambda ws, n: lib.mpc_efmix_topk_compress(p, p, 3, 64, k, p, p, ws, n, None)  # noqa: E731
+    assert call(None, 0) == 3                       # workspace missing
+    assert call(ws, need - 1) == 3                  # workspace short
+    assert call(ctypes.c_void_p(0x100010), need) == 1  # workspace not 256-byte aligned
