@@ -23,6 +23,9 @@
  *    are recorded in a per-process device status word and reported by
  *    mpc_get_status(); the outputs of the failing call are then unspecified.
  *  - No C++ exception crosses this interface.
+ *  - The library looks up per-device addresses of its device variables once
+ *    per device and keeps them: it supports the device's primary context only
+ *    (the CUDA runtime's), and no cudaDeviceReset while it is loaded.
  *
  * TopK payload: for each row, the k kept entries as `vals[rows][k]` (fp32, the
  * exact bits of the kept value, sign included) and `idx[rows][k]` (int32 column
@@ -265,12 +268,14 @@ mpc_status mpc_aqsgd_quant_decompress(const uint32_t* codes, const float* scale,
  * of 8 * MPC_QUANT_NOALLOC_MAX_ROWS bytes (512 KiB) that every device loading
  * the library keeps until the process exits.  rows > MPC_QUANT_NOALLOC_MAX_ROWS
  * returns MPC_ERR_INVALID_ARG and launches nothing.
+ * Only calls whose rows are longer than 65536 entries (the two-pass path)
+ * use the array; shorter rows run exactly as in mpc_quant_compress.
  * The first call on a device looks up the array's device address (with that
  * device current); make that first call outside any CUDA stream capture.
- * Every call shares the one array: calls whose kernels may overlap on the GPU
- * (different streams without ordering) race and give undefined results; calls
- * ordered on one stream are safe.  No cudaMalloc, cudaFree or allocating
- * library routine is called. */
+ * Every call with rows longer than 65536 entries shares the one array: such
+ * calls whose kernels may overlap on the GPU (different streams without
+ * ordering) race and give undefined results; calls ordered on one stream are
+ * safe.  No cudaMalloc, cudaFree or allocating library routine is called. */
 #define MPC_QUANT_NOALLOC_MAX_ROWS 65536
 mpc_status mpc_quant_compress_noalloc(const float* x, int64_t rows, int64_t row_len, int bits,
                                       mpc_rounding mode, uint64_t seed, uint32_t* codes,

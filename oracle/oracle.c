@@ -317,8 +317,9 @@ static uint32_t get_code(const uint32_t* row_codes, int64_t j, int bits)
     return (uint32_t)(both & ((1ull << bits) - 1u));
 }
 
-/* "Input vector with floating values is mapped to [0;1] interval with min-max
- * scaling and then quantized": with L = 2^bits - 1 intervals,
+/* §2.2: each row is shifted by its minimum and divided by its range, which
+ * puts it in [0, 1], and then rounded onto 2^bits evenly spaced levels; with
+ * L = 2^bits - 1 intervals,
  *   scale = (max - min) / L,  inv = L / (max - min),
  *   t = (x - min) * inv,  q = round(t)  or  floor(t + u),  clamped to [0, L].
  * A row whose range is 0, or whose range or inv is infinite, sends all-zero

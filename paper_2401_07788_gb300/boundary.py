@@ -1,5 +1,5 @@
-"""Compression block between pipeline stages (§2.1, Figure 1): activations are compressed
-in the forward pass and the gradients of those activations in the backward pass, so that
+"""Compression block between pipeline stages (§2.1, Figure 1): the forward pass sends a
+compressed activation across the cut and the backward pass a compressed gradient, so that
 a model cut into stages trains as it would if the stages ran on separate devices that
 exchange compressed messages.
 

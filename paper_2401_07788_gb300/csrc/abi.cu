@@ -371,7 +371,6 @@ mpc_status mpc_quant_compress(const float* x, int64_t rows, int64_t row_len, int
     return set_error(MPC_ERR_INVALID_ARG, "bits=%d not in 1..16 or 32", bits);
   if (mode != MPC_ROUND_NEAREST && mode != MPC_ROUND_STOCHASTIC)
     return set_error(MPC_ERR_INVALID_ARG, "rounding mode %d", static_cast<int>(mode));
-  if (row_len > 0x7fffffffLL / 32) return set_error(MPC_ERR_INVALID_ARG, "row_len too large");
   if (rows == 0) return ok();
   MPC_TRY(check_ptr(x, 4, "x"));
   MPC_TRY(check_ptr(codes, 4, "codes"));
@@ -411,7 +410,6 @@ mpc_status mpc_quant_compress_noalloc(const float* x, int64_t rows, int64_t row_
     return set_error(MPC_ERR_INVALID_ARG, "bits=%d not in 1..16 or 32", bits);
   if (mode != MPC_ROUND_NEAREST && mode != MPC_ROUND_STOCHASTIC)
     return set_error(MPC_ERR_INVALID_ARG, "rounding mode %d", static_cast<int>(mode));
-  if (row_len > 0x7fffffffLL / 32) return set_error(MPC_ERR_INVALID_ARG, "row_len too large");
   if (rows > mpc::quant_noalloc_max_rows())
     return set_error(MPC_ERR_INVALID_ARG,
                      "rows=%lld exceeds the %lld rows of the static scratch of "
@@ -450,7 +448,6 @@ mpc_status mpc_quant_decompress(const uint32_t* codes, const float* scale, const
   MPC_TRY(check_shape(rows, row_len, 1));
   if (!valid_bits(bits))
     return set_error(MPC_ERR_INVALID_ARG, "bits=%d not in 1..16 or 32", bits);
-  if (row_len > 0x7fffffffLL / 32) return set_error(MPC_ERR_INVALID_ARG, "row_len too large");
   if (rows == 0) return ok();
   MPC_TRY(check_ptr(codes, 4, "codes"));
   MPC_TRY(check_ptr(scale, 4, "scale"));
@@ -480,7 +477,6 @@ mpc_status check_aqsgd_quant(int64_t num_samples, int64_t n_ids, int64_t rps, in
   MPC_TRY(check_shape(*rows, L, 1));
   if (!valid_bits(bits))
     return set_error(MPC_ERR_INVALID_ARG, "bits=%d not in 1..16 or 32", bits);
-  if (L > 0x7fffffffLL / 32) return set_error(MPC_ERR_INVALID_ARG, "row_len too large");
   if (num_samples > INT64_MAX / rps / L)
     return set_error(MPC_ERR_INVALID_ARG, "buffer size overflows");
   return ok();

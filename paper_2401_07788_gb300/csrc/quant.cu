@@ -686,6 +686,7 @@ cudaError_t run_quant_bits(const QuantArgs& a0, int num_sms, cudaStream_t s) {
   } else {
     a.slice = kQSCAP;
     spr = (L + kQSCAP - 1) / kQSCAP;
+    if (a.rows > 0x7fffffffLL / spr) return cudaErrorInvalidValue;  // before any launch
     uint32_t* mm = static_cast<uint32_t*>(a.ws);
     minmax_init_kernel<<<static_cast<unsigned>(min64((a.rows + 255) / 256, 1024)), 256, 0, s>>>(mm, a.rows);
     quant_minmax_kernel<<<static_cast<unsigned>(a.rows * spr), kQNT, 0, s>>>(a.x, L, static_cast<int>(spr), a.slice, mm);
@@ -810,9 +811,11 @@ cudaError_t launch_quant_compress_noalloc(const QuantArgs& a0, int num_sms, cuda
     scratch = g_noalloc_ptr[dev];
   }
   QuantArgs a = a0;
-  // The two-pass path starts by writing every row's {min, max} slot, so no
-  // state of an earlier call is read.
-  a.ws = (a.bits == 32) ? nullptr : scratch;
+  // Only rows longer than the single-pass kernels take (the two-pass path)
+  // use the scratch; the others run exactly as mpc_quant_compress does.  The
+  // two-pass path starts by writing every row's {min, max} slot, so no state
+  // of an earlier call is read.
+  a.ws = quant_workspace_bytes(a.rows, a.L, a.bits) > 0 ? scratch : nullptr;
   return launch_quant_compress(a, num_sms, s);
 }
 

@@ -52,3 +52,22 @@ def assert_bits_equal(got: np.ndarray, want: np.ndarray, what: str) -> None:
         i = tuple(bad[0])
         raise AssertionError("%s: %d mismatches, first at %s: got %r want %r"
                              % (what, len(bad), i, got[i], want[i]))
+
+
+def row_blocks(fn, n_rows: int, *arrays, threads: int = 16):
+    """Run ``fn(*blocks)`` on row blocks of ``arrays`` in threads and stack the results.
+
+    For oracle calls that treat rows independently and whose results do not depend on a
+    row's position in the call (TopK, error feedback, EF21, nearest quantisation; not
+    stochastic rounding, whose counter runs over the flat index of the call).  The oracle
+    is a C library called through ctypes, which releases the GIL, so blocks run on
+    separate cores.  Arrays updated in place are passed as views of their row blocks."""
+    from concurrent.futures import ThreadPoolExecutor
+
+    step = max(1, -(-n_rows // threads))
+    spans = [(r, min(n_rows, r + step)) for r in range(0, n_rows, step)]
+    with ThreadPoolExecutor(len(spans)) as ex:
+        outs = list(ex.map(lambda s: fn(*(a[s[0]:s[1]] for a in arrays)), spans))
+    if outs and isinstance(outs[0], tuple):
+        return tuple(np.concatenate(parts, axis=0) for parts in zip(*outs))
+    return outs

@@ -7,7 +7,7 @@ import pytest
 import torch
 
 import oracle
-from gpu_cases import assert_bits_equal
+from gpu_cases import assert_bits_equal, row_blocks
 
 pytestmark = pytest.mark.gpu
 
@@ -58,21 +58,23 @@ def test_cnn_small_boundary(mpc, synth):
 
 @pytest.mark.parametrize("seed", [0, 9])
 def test_cnn_boundary_ef_and_quant(mpc, synth, seed):
-    """[128,128,16,16]: EF-TopK at 5/10/30% with the error carried over drifting steps;
-    2/4/8-bit gradients, nearest and stochastic (seed (config_seed << 32) | step)."""
+    """[128,128,16,16] for all 50 steps of the workload: EF-TopK at 5/10/30% with the
+    error carried over the drifting steps, and 2/4/8-bit gradients, nearest and stochastic
+    (seed (config_seed << 32) | step); every output compared at every step."""
     c = synth.CNN
     R, L = c["rows"], c["row_len"]
     gen = synth.generator(seed, "cuda")
     x = synth.relu_normal(c["shape"], seed, "cuda", gen=gen).view(R, L)
     errs = {p: torch.zeros((R, L), device="cuda") for p in c["topk_percents"]}
     errs_host = {p: np.zeros((R, L), np.float32) for p in c["topk_percents"]}
-    for step in range(3):
+    for step in range(c["steps"]):
         xn = x.cpu().numpy()
         for p in c["topk_percents"]:
             k = synth.k_of(L, p)
             v, i = mpc.mpc_ef_topk_compress(x, errs[p], k)
             ok(mpc)
-            ov, oi = oracle.ef_topk_compress(xn, errs_host[p], k)
+            ov, oi = row_blocks(lambda xb, eb: oracle.ef_topk_compress(xb, eb, k), R, xn,
+                                errs_host[p])
             assert_bits_equal(i.cpu().numpy(), oi, "idx K=%d step %d" % (p, step))
             assert_bits_equal(v.cpu().numpy(), ov, "vals K=%d step %d" % (p, step))
             assert_bits_equal(errs[p].cpu().numpy(), errs_host[p], "err K=%d step %d" % (p, step))
@@ -83,16 +85,21 @@ def test_cnn_boundary_ef_and_quant(mpc, synth, seed):
                 sd = (seed << 32) | step
                 cq, sq, mq = mpc.mpc_quant_compress(g, bits, stochastic=sr, seed=sd)
                 ok(mpc)
-                oc, os_, om = oracle.quant_compress(gn, bits, sr, sd)
-                assert_bits_equal(cq.cpu().numpy().view(np.uint32), oc, "codes b=%d" % bits)
-                assert_bits_equal(sq.cpu().numpy(), os_, "scale b=%d" % bits)
-                assert_bits_equal(mq.cpu().numpy(), om, "minv b=%d" % bits)
+                if sr:
+                    oc, os_, om = oracle.quant_compress(gn, bits, sr, sd)
+                else:
+                    oc, os_, om = row_blocks(lambda gb: oracle.quant_compress(gb, bits), R, gn)
+                what = "b=%d sr=%d step %d" % (bits, sr, step)
+                assert_bits_equal(cq.cpu().numpy().view(np.uint32), oc, "codes " + what)
+                assert_bits_equal(sq.cpu().numpy(), os_, "scale " + what)
+                assert_bits_equal(mq.cpu().numpy(), om, "minv " + what)
         x = synth.drift(x, c["drift"], gen)
 
 
 def test_lm_boundary_ef21_and_quant(mpc, synth):
-    """GPT-2 boundary [8,1024,768] with outlier channels: EF21-TopK 10% per token, g_0 = 0,
-    over drifting steps; 4-bit per-token gradient quantisation."""
+    """GPT-2 boundary [8,1024,768] with outlier channels, all 20 steps of the workload:
+    EF21-TopK 10% per token, g_0 = 0, over drifting steps, and 4-bit per-token gradient
+    quantisation of each step's gradient."""
     c = synth.LM
     R, L = c["rows"], c["row_len"]
     k = synth.k_of(L, c["topk_percent"])
@@ -100,49 +107,58 @@ def test_lm_boundary_ef21_and_quant(mpc, synth):
     gen = synth.generator(1, "cuda")
     g_dev = torch.zeros((R, L), device="cuda")
     g_host = np.zeros((R, L), np.float32)
-    for step in range(3):
+    for step in range(c["steps"]):
         xn = x.cpu().numpy()
         v, i = mpc.mpc_ef21_topk_compress(x, g_dev, k)
         ok(mpc)
-        ov, oi = oracle.ef21_topk_compress(xn, g_host, k)
+        ov, oi = row_blocks(lambda xb, gb: oracle.ef21_topk_compress(xb, gb, k), R, xn, g_host)
         assert_bits_equal(i.cpu().numpy(), oi, "idx step %d" % step)
         assert_bits_equal(v.cpu().numpy(), ov, "vals step %d" % step)
         assert_bits_equal(g_dev.cpu().numpy(), g_host, "g step %d" % step)
+        gr = synth.normal((R, L), 2 + step, "cuda", std=1e-4)
+        cq, sq, mq = mpc.mpc_quant_compress(gr, 4)
+        y = mpc.mpc_quant_decompress(cq, sq, mq, L, 4)
+        ok(mpc)
+        oc, os_, om = row_blocks(lambda gb: oracle.quant_compress(gb, 4), R, gr.cpu().numpy())
+        assert_bits_equal(cq.cpu().numpy().view(np.uint32), oc, "codes step %d" % step)
+        assert_bits_equal(y.cpu().numpy(), oracle.quant_decompress(oc, os_, om, L, 4),
+                          "dequant step %d" % step)
         x = synth.drift(x, c["drift"], gen)
-    gr = synth.normal((R, L), 2, "cuda", std=1e-4)
-    cq, sq, mq = mpc.mpc_quant_compress(gr, 4)
-    y = mpc.mpc_quant_decompress(cq, sq, mq, L, 4)
-    ok(mpc)
-    oc, os_, om = oracle.quant_compress(gr.cpu().numpy(), 4)
-    assert_bits_equal(cq.cpu().numpy().view(np.uint32), oc, "codes")
-    assert_bits_equal(y.cpu().numpy(), oracle.quant_decompress(oc, os_, om, L, 4), "dequant")
 
 
 def test_aqsgd_boundary_full_buffer(mpc, synth):
-    """Per-sample buffer [4096,512,1024] (2^31 entries, 64-bit offsets): 16 ids per step,
-    Top30% of the change; the gathered rows are checked against the oracle and rows of
-    samples not drawn stay bit-identical."""
+    """Per-sample buffer [4096,512,1024] (2^31 entries, 64-bit offsets), 10 steps of 16 ids,
+    Top30% of the change: the gathered rows are checked against the oracle at every step,
+    the receiver's copy of the buffer (updated from the payload alone) stays bit-identical
+    to the sender's, and rows of samples not drawn stay bit-identical."""
     c = synth.AQSGD
     S, rps, L = c["num_samples"], c["rows_per_sample"], c["row_len"]
     k = synth.k_of(L, c["topk_percent"])
     buf = synth.normal((S, rps, L), 0, "cuda")
+    recv = buf.clone()
     watch = torch.tensor([0, 1, S // 2, S - 1], device="cuda")
     gen = synth.generator(5, "cuda")
-    for step in range(2):
-        ids = synth.sample_ids(S, c["ids_per_step"], 100 + step, "cuda")
-        x = buf[ids] + c["noise"] * torch.randn((ids.numel(), rps, L), generator=gen, device="cuda")
+    n = c["ids_per_step"]
+    for step in range(10):
+        ids = synth.sample_ids(S, n, 100 + step, "cuda")
+        x = buf[ids] + c["noise"] * torch.randn((n, rps, L), generator=gen, device="cuda")
         rows_before = buf[ids].cpu().numpy()
         untouched = watch[~torch.isin(watch, ids)]
         keep = buf[untouched].clone()
         v, i = mpc.mpc_aqsgd_compress(x, buf, ids, k)
+        mpc.mpc_aqsgd_decompress(v, i, recv, ids)
         ok(mpc)
         local = rows_before.copy()
-        ov, oi = oracle.aqsgd_compress(x.cpu().numpy(), local, np.arange(ids.numel()), k)
+        ov, oi = row_blocks(
+            lambda xb, lb: oracle.aqsgd_compress(xb, lb, np.arange(xb.shape[0]), k), n,
+            x.cpu().numpy(), local)
         assert_bits_equal(i.cpu().numpy(), oi, "idx step %d" % step)
         assert_bits_equal(v.cpu().numpy(), ov, "vals step %d" % step)
         assert_bits_equal(buf[ids].cpu().numpy(), local, "buffer rows step %d" % step)
+        assert torch.equal(recv[ids].view(torch.int32), buf[ids].view(torch.int32)), step
         assert torch.equal(buf[untouched], keep)
-    del buf
+    assert torch.equal(recv.view(torch.int32), buf.view(torch.int32))
+    del buf, recv
     torch.cuda.empty_cache()
 
 
