@@ -2,33 +2,34 @@
 """Benchmark of libmpcomp: compress+decompress GB/s (input bytes) and the fraction of HBM
 bandwidth per operator, on one GB300.
 
-Workload (the CNN stage boundary, [128,128,16,16] fp32 = 128 rows x 32768): one step is
-one boundary crossing of every operator the workload sweeps, on that step's tensors:
-  forward : error-feedback TopK at K = 5, 10, 30 % (one error buffer per K, carried
-            across steps) of the activation ReLU(N(0,1)) drifting by 0.1*N(0,1) per step,
-            each followed by TopK decompression;
-  backward: 2/4/8-bit min-max quantisation of the gradient N(0, sigma=1e-3), round to
-            nearest and stochastic (seed (seed << 32) | step), each followed by
-            dequantisation.
-value = sum over the 9 compress+decompress pairs of the input bytes (4 x 128 x 32768) /
-device time of the step.  Each step is one CUDA graph of the 18 library launches (one
-graph per slot of a pool of 4 pre-drawn steps, so inputs differ from step to step), with
-no event nodes inside; the nine pairs are independent and run as concurrent branches of
-the graph (--branches).  L2 is flushed before every timed step by writing and then
-reading a 256 MiB buffer (so the step's inputs are cold and the flush leaves no dirty
-lines for the first launch to write back), outside the timed interval.  Per-launch
-shares come from a second timed pass whose graphs run the 18 launches in order and
-record an event after every launch; the dominant launch's duration (for `roofline`)
-from 200 launches of it in a row between two events on its stream, the inputs cycling
-through 8 copies (twice the L2) so that each launch reads cold inputs, and, for
-reference, from single launches between two events (which adds ~5 us to any launch).  `e2e` runs
-the steps through the Python API with the step's inputs copied from pinned host memory
-and two outputs copied back inside the timed region.  `operators` times every operator
-of the path on its own workload: a CUDA graph of 8 x (L2 flush, launch) against a graph
-of the 8 flushes alone, the difference divided by 8.
+Headline workload: the bandwidth sweep at its largest size, one N(0,1) fp32 tensor of
+2^30 entries (4 GiB), reshaped to rows of 768, 4096 and 65536 entries and to one
+whole-tensor row.  One step runs, for each of the four row lengths, every
+compress+decompress pair of the sweep on that step's tensor:
+  TopK at K = 1, 10, 50 %, each followed by TopK decompression;
+  error-feedback TopK at K = 1, 10, 50 % (one error buffer per row length and K, carried
+  across steps), each followed by decompression of its payload;
+  2/4/8-bit min-max quantisation (round to nearest), each followed by dequantisation.
+That is 36 pairs (72 library calls) per step, in order on one stream; two input tensors
+alternate from step to step.  value = 36 x 4 x 2^30 input bytes per step / device time of
+the step (CUDA events on the stream, max over ranks).  Every input is 4 GiB, far larger
+than the 126 MB L2, so no L2 flush is needed between steps.  An event after every call
+gives each call's duration inside the timed region; `roofline` reports the call with the
+largest share of the step: its algorithmic bytes (inputs and buffers read once, payload
+and buffers written once) / its average duration, against the measured copy bandwidth.
+`e2e` runs the same steps through the same calls with the input tensor copied from
+pinned host memory and the last dequantised tensor copied back every step (pipelined over
+two slots).  `per_op` lists every call of the step.
 
-`--impl reference` times the CPU oracle (single-threaded C) on a bounded sample of the
-same step: 16 of the 128 rows.
+Secondary keys: `cnn_boundary_step`, the CNN stage boundary [128,128,16,16] (EF-TopK at
+5/10/30 % and 2/4/8-bit quantisation, nearest and stochastic, with their
+decompressions; one CUDA graph per step); `whole_tensor`, whole-tensor rows of 2^27,
+2^28 and 2^29 entries; `operators`, every operator on its own workload (the small CNN,
+transformer and AQ-SGD boundaries, index reuse, EF-mixed, stochastic and 6-bit codes).
+
+`--impl reference` and `cpu_baseline` time the CPU oracle (single-threaded C) on a
+bounded sample of the same step: a few rows of each row length and a whole-tensor row of
+2^20 entries.
 """
 
 from __future__ import annotations
@@ -50,27 +51,33 @@ import torch  # noqa: E402
 
 METRIC = "compress+decompress GB/s (input bytes) and % of HBM roofline per operator at 1 GB300"
 UNIT = "GB/s"
-WORKLOAD = "CNN stage boundary [128,128,16,16] fp32"
+LOG2N = 30
+SWEEP_LENS = (768, 4096, 65536, None)  # None: the whole tensor as one row
+SWEEP_PCTS = (1, 10, 50)
+SWEEP_BITS = (2, 4, 8)
+# the CNN stage boundary (secondary key)
 R, L = 128, 32768
 TOPK_PCTS = (5, 10, 30)
 BITS = (2, 4, 8)
 POOL = 4
-SAMPLE_ROWS = 16
 
 
 def parse_args():
     p = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     p.add_argument("--gpus", type=int, default=1)
-    p.add_argument("--steps", type=int, default=1000)
-    p.add_argument("--warmup", type=int, default=10)
+    p.add_argument("--steps", type=int, default=10)
+    p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    p.add_argument("--log2n", type=int, default=LOG2N,
+                   help="entries of the headline tensor, log2 (the workload is 2^30)")
     p.add_argument("--no-operators", action="store_true", help="skip the per-operator table")
+    p.add_argument("--no-secondary", action="store_true",
+                   help="skip the CNN-boundary step and the whole-tensor table")
+    p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
-    p.add_argument("--sweep", action="store_true",
-                   help="only the size sweep: N = 2^20..2^30 entries, L in {768, 4096, 65536, N}; "
-                        "prints one JSON line with the table (not the benchmark line)")
+    p.add_argument("--cnn-steps", type=int, default=200)
     p.add_argument("--branches", type=int, default=6, choices=(1, 2, 3, 5, 6, 9),
-                   help="concurrent streams inside the step graph (1 = all launches in order)")
+                   help="concurrent streams inside the CNN-boundary step graph")
     return p.parse_args()
 
 
@@ -274,23 +281,19 @@ class ClockSampler:
 
 
 # ---------------------------------------------------------------------------------------
-# the workload
+# algorithmic bytes and the kernels behind each call
 # ---------------------------------------------------------------------------------------
 
 def algorithmic_bytes(R_, L_, k=None, bits=None, op=""):
-    """Minimum HBM bytes of one launch: inputs and buffers read once, payload and buffers
-    written once."""
+    """Minimum HBM bytes of one call: inputs and buffers read once, payload and buffers
+    written once (the buffer of EF21 / AQ-SGD counted as read and written in full)."""
     N = R_ * L_
-    if op == "ef_topk":
+    if op in ("ef_topk", "delta_topk", "efmix_topk"):  # x, buffer read; buffer, payload written
         return 12 * N + 8 * k * R_
     if op == "topk":
         return 4 * N + 8 * k * R_
     if op == "topk_decompress":
         return 8 * k * R_ + 4 * N
-    if op == "delta_topk":  # EF21 / AQ-SGD: state written only where kept
-        return 8 * N + 12 * k * R_
-    if op == "efmix_topk":  # x and err read, err written, payload written
-        return 12 * N + 8 * k * R_
     if op == "topk_gather":  # indices read, values gathered, payload written
         return 12 * k * R_
     if op == "aqsgd_decompress":
@@ -303,6 +306,366 @@ def algorithmic_bytes(R_, L_, k=None, bits=None, op=""):
         return 4 * N + (N * bits + 7) // 8 + 8 * R_
     raise ValueError(op)
 
+
+ROW_PATH_MAX = 65536  # longest row of the on-chip TopK and single-pass quantisation kernels
+
+
+def kernels_of(op: str, L_: int) -> list:
+    """The library kernels one call launches, in order (the launch count is their number)."""
+    if op in ("topk", "ef_topk"):
+        if L_ <= 1024:
+            return ["topk_warp_kernel"]
+        if L_ <= ROW_PATH_MAX:
+            return ["topk_cta_kernel"]
+        return ["g_init", "g_sample"] + ["g_hist", "g_pick"] * 4 + ["g_count", "g_select",
+                                                                   "g_scan", "g_write"]
+    if op == "topk_decompress":
+        return ["topk_decompress_rows_kernel" if L_ <= ROW_PATH_MAX else "topk_decompress_kernel"]
+    if op == "quant":
+        if L_ <= 2048:
+            return ["quant_warp_kernel"]
+        if L_ <= ROW_PATH_MAX:
+            return ["quant_cta_kernel"]
+        return ["minmax_init_kernel", "quant_minmax_kernel", "quant_cta_kernel"]
+    if op == "dequant":
+        return ["dequant_rows_kernel"]
+    raise ValueError(op)
+
+
+# ---------------------------------------------------------------------------------------
+# the headline step: the bandwidth sweep at 2^30 entries
+# ---------------------------------------------------------------------------------------
+
+def headline_call_names(log2n: int = LOG2N) -> list:
+    """Names of the calls of one headline step, in launch order (no device needed)."""
+    N = 1 << log2n
+    names = []
+    for Ls in SWEEP_LENS:
+        tag = "L=%s" % ("N" if Ls is None else Ls)
+        for feedback in (False, True):
+            for p in SWEEP_PCTS:
+                names.append(("ef_topk_compress %s K=%d%%" if feedback else "topk_compress %s K=%d%%")
+                             % (tag, p))
+                names.append("topk_decompress %s K=%d%%%s" % (tag, p, " (EF)" if feedback else ""))
+        for b in SWEEP_BITS:
+            names += ["quant_compress %s %d-bit" % (tag, b), "quant_decompress %s %d-bit" % (tag, b)]
+    assert N > 0
+    return names
+
+
+class Call:
+    __slots__ = ("name", "op", "L", "fn", "nbytes", "in_bytes", "kernels")
+
+    def __init__(self, name, op, L_, fn, nbytes, in_bytes):
+        self.name, self.op, self.L, self.fn = name, op, L_, fn
+        self.nbytes, self.in_bytes = nbytes, in_bytes
+        self.kernels = kernels_of(op, L_)
+
+
+class SweepStep:
+    """Buffers and the 72 calls of one step of the sweep at N entries.  Every call takes
+    the step's input tensor x (N entries) and the dense output y (N entries), so the same
+    calls serve the device-resident and the end-to-end runs."""
+
+    def __init__(self, mpc, synth, device, log2n: int, seed: int):
+        self.mpc = mpc
+        N = 1 << log2n
+        self.N = N
+        self.xs = [synth.normal((N,), 1000 * seed + log2n + 17 * t, device) for t in range(2)]
+        self.y = torch.empty(N, device=device)
+        self.seed = seed
+        shapes = []
+        for Ls in SWEEP_LENS:
+            Lr = N if Ls is None else Ls
+            shapes.append((N // Lr, Lr))
+        self.shapes = shapes
+        max_pay = max(Rr * synth.k_of(Lr, p) for Rr, Lr in shapes for p in SWEEP_PCTS)
+        self.vals = torch.empty(max_pay, device=device)
+        self.idx = torch.empty(max_pay, dtype=torch.int32, device=device)
+        max_words = max(mpc.mpc_quant_codes_words(Rr, Lr, b) for Rr, Lr in shapes for b in SWEEP_BITS)
+        self.codes = torch.empty(max_words, dtype=torch.int32, device=device)
+        max_rows = max(Rr for Rr, _ in shapes)
+        self.scale = torch.empty(max_rows, device=device)
+        self.minv = torch.empty(max_rows, device=device)
+        tws = max(mpc.mpc_topk_workspace_bytes(Rr, Lr, synth.k_of(Lr, p))
+                  for Rr, Lr in shapes for p in SWEEP_PCTS)
+        qws = max(mpc.mpc_quant_workspace_bytes(Rr, Lr, b) for Rr, Lr in shapes for b in SWEEP_BITS)
+        self.tws = torch.empty(max(tws, 256), dtype=torch.uint8, device=device)
+        self.qws = torch.empty(max(qws, 256), dtype=torch.uint8, device=device)
+        self.errs = {}
+        self.calls = []
+        m = mpc
+        for Rr, Lr in shapes:
+            tag = "L=%s" % ("N" if Lr == N else Lr)
+            n = Rr * Lr
+            for feedback in (False, True):
+                for p in SWEEP_PCTS:
+                    k = synth.k_of(Lr, p)
+                    v = self.vals[: Rr * k].view(Rr, k)
+                    i = self.idx[: Rr * k].view(Rr, k)
+                    if feedback:
+                        e = torch.zeros((Rr, Lr), device=device)
+                        self.errs[(Lr, p)] = e
+                        fn = (lambda x, y, Rr=Rr, Lr=Lr, k=k, v=v, i=i, e=e: m.mpc_ef_topk_compress(
+                            x[: Rr * Lr].view(Rr, Lr), e, k, v, i, ws=self.tws))
+                        self.calls.append(Call("ef_topk_compress %s K=%d%%" % (tag, p), "ef_topk", Lr,
+                                               fn, algorithmic_bytes(Rr, Lr, k=k, op="ef_topk"), 4 * n))
+                    else:
+                        fn = (lambda x, y, Rr=Rr, Lr=Lr, k=k, v=v, i=i: m.mpc_topk_compress(
+                            x[: Rr * Lr].view(Rr, Lr), k, v, i, ws=self.tws))
+                        self.calls.append(Call("topk_compress %s K=%d%%" % (tag, p), "topk", Lr, fn,
+                                               algorithmic_bytes(Rr, Lr, k=k, op="topk"), 4 * n))
+                    fn = (lambda x, y, Rr=Rr, Lr=Lr, v=v, i=i: m.mpc_topk_decompress(
+                        v, i, Lr, y=y[: Rr * Lr].view(Rr, Lr)))
+                    self.calls.append(Call("topk_decompress %s K=%d%%%s" % (tag, p, " (EF)" if feedback else ""),
+                                           "topk_decompress", Lr, fn,
+                                           algorithmic_bytes(Rr, Lr, k=k, op="topk_decompress"), 0))
+            for b in SWEEP_BITS:
+                W = m.mpc_quant_codes_words(Rr, Lr, b) // Rr
+                c = self.codes[: Rr * W].view(Rr, W)
+                sc, mn = self.scale[:Rr], self.minv[:Rr]
+                fn = (lambda x, y, Rr=Rr, Lr=Lr, b=b, c=c, sc=sc, mn=mn: m.mpc_quant_compress(
+                    x[: Rr * Lr].view(Rr, Lr), b, codes=c, scale=sc, minv=mn, ws=self.qws))
+                self.calls.append(Call("quant_compress %s %d-bit" % (tag, b), "quant", Lr, fn,
+                                       algorithmic_bytes(Rr, Lr, bits=b, op="quant"), 4 * n))
+                fn = (lambda x, y, Rr=Rr, Lr=Lr, b=b, c=c, sc=sc, mn=mn: m.mpc_quant_decompress(
+                    c, sc, mn, Lr, b, y=y[: Rr * Lr].view(Rr, Lr)))
+                self.calls.append(Call("quant_decompress %s %d-bit" % (tag, b), "dequant", Lr, fn,
+                                       algorithmic_bytes(Rr, Lr, bits=b, op="dequant"), 0))
+        assert [c.name for c in self.calls] == headline_call_names(log2n)
+        self.input_bytes = sum(c.in_bytes for c in self.calls)
+        self.launches = sum(len(c.kernels) for c in self.calls)
+
+    def run(self, x, y, events=None):
+        for j, c in enumerate(self.calls):
+            c.fn(x, y)
+            if events is not None:
+                events[j].record()
+
+
+def run_headline(args, rank, local, world):
+    import paper_2401_07788_gb300 as mpc
+    from paper_2401_07788_gb300 import synth
+
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    init_dist(world, "nccl")
+    mpc.lib()
+    st = SweepStep(mpc, synth, device, args.log2n, rank % 10)
+    n_calls = len(st.calls)
+    stream = torch.cuda.Stream(device)
+    with torch.cuda.stream(stream):
+        for w in range(max(1, args.warmup)):
+            st.run(st.xs[w % 2], st.y)
+    stream.synchronize()
+    status = mpc.mpc_get_status(stream)
+    if status != 0:
+        raise RuntimeError("device status %d: %s" % (status, mpc.mpc_last_error()))
+
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(n_calls)] for _ in range(args.steps)]
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    barrier(world)
+    torch.cuda.synchronize()
+    sampler = ClockSampler(local)
+    sampler.__enter__()
+    t0 = time.perf_counter()
+    with torch.cuda.stream(stream):
+        for s in range(args.steps):
+            starts[s].record(stream)
+            st.run(st.xs[s % 2], st.y, evs[s])
+    stream.synchronize()
+    wall = time.perf_counter() - t0
+    sampler.__exit__(None, None, None)
+    clocks = sampler.summary()
+    barrier(world)
+    status = mpc.mpc_get_status(stream)
+    if status != 0:
+        raise RuntimeError("device status %d: %s" % (status, mpc.mpc_last_error()))
+    op_ms = [0.0] * n_calls
+    dev_ms = 0.0
+    for s in range(args.steps):
+        prev = starts[s]
+        for j in range(n_calls):
+            op_ms[j] += prev.elapsed_time(evs[s][j])
+            prev = evs[s][j]
+        dev_ms += starts[s].elapsed_time(evs[s][-1])
+    units, secs = aggregate(st.input_bytes * args.steps, dev_ms / 1e3, world, device)
+    value = units / secs / 1e9
+
+    peak, peak_kind = hbm_peak()
+    per_op = {}
+    for j, c in enumerate(st.calls):
+        us = op_ms[j] / args.steps * 1e3
+        gbs = c.nbytes / (us / 1e6) / 1e9
+        per_op[c.name] = {"us": round(us, 1), "GBps": round(gbs, 1), "frac": round(gbs / peak, 4),
+                          "launches": len(c.kernels)}
+    dom = max(range(n_calls), key=lambda j: op_ms[j])
+    c = st.calls[dom]
+    avg_ms = op_ms[dom] / args.steps
+    achieved = c.nbytes / (avg_ms / 1e3) / 1e9
+    roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                "frac": round(achieved / peak, 4),
+                "traffic": recorded_traffic(c.name),
+                "op": c.name, "kernels": sorted(set(c.kernels)), "launches_per_call": len(c.kernels),
+                "algorithmic_bytes": c.nbytes, "avg_call_us": round(avg_ms * 1e3, 1),
+                "share_of_step": round(op_ms[dom] / max(sum(op_ms), 1e-9), 4),
+                "peak_source": peak_kind + " (MEASURED_PEAKS.json hbm_gbs, copy bandwidth)"
+                if peak_kind == "measured" else peak_kind,
+                "timing": "CUDA events on the launching stream before and after the call, "
+                          "inside the timed steps, averaged over the steps"}
+
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(args, st, stream, world, device)
+
+    cnn = whole = operators = None
+    if not args.no_secondary:
+        cnn = run_cnn_step(args, mpc, synth, device, world)
+        if rank == 0:
+            whole = measure_whole_tensor(mpc, synth, device, stream, peak)
+    if not args.no_operators and rank == 0:
+        operators = measure_operators(mpc, synth, device, stream, peak)
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(budget_s=10.0)
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": round(value, 2), "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(secs * 1e3 / args.steps, 3), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": {"workload": "bandwidth sweep at 2^%d entries: one N(0,1) fp32 tensor of "
+                                   "%d entries as rows of 768, 4096, 65536 and one whole-tensor row"
+                                   % (args.log2n, st.N),
+                       "entries": st.N, "row_lens": [Lr for _, Lr in st.shapes],
+                       "rows": [Rr for Rr, _ in st.shapes],
+                       "topk_percents": list(SWEEP_PCTS), "ef_topk_percents": list(SWEEP_PCTS),
+                       "bits": list(SWEEP_BITS), "rounding": "nearest",
+                       "pairs_per_step": n_calls // 2, "calls_per_step": n_calls,
+                       "input_bytes_per_step": st.input_bytes,
+                       "l2": "no flush: every input is %d bytes, larger than the 126 MB L2" % (4 * st.N),
+                       "parallelism": "replicas" if world > 1 else "single GPU"},
+            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
+            "gpu_launches": st.launches * args.steps, "clocks": clocks,
+            "wall_s": round(wall, 3), "per_op": per_op,
+            "cnn_boundary_step": cnn, "whole_tensor": whole, "operators": operators,
+        }
+        print(json.dumps(line), flush=True)
+
+
+def run_e2e(args, st, stream, world, device):
+    """The headline steps end to end: every step copies its input tensor from pinned host
+    memory to the device and the last dequantised tensor back, inside the timed region,
+    through the same calls.  Copies and compute are pipelined over two slots (step s+1's
+    input goes up while step s computes and step s-1's result comes down), each copy on its
+    own stream."""
+    N = st.N
+    hx = st.xs[0].cpu().pin_memory()
+    hy = [torch.empty(N, pin_memory=True) for _ in range(2)]
+    dx = [torch.empty(N, device=device) for _ in range(2)]
+    dy = [torch.empty(N, device=device) for _ in range(2)]
+    up, down = torch.cuda.Stream(device), torch.cuda.Stream(device)
+    ev = lambda: [torch.cuda.Event() for _ in range(2)]  # noqa: E731
+    x_in, done, y_out = ev(), ev(), ev()
+    for e in done + y_out:
+        e.record(stream)
+
+    def one(s):
+        b = s % 2
+        up.wait_event(done[b])  # the slot's previous compute has read its input
+        with torch.cuda.stream(up):
+            dx[b].copy_(hx, non_blocking=True)
+            x_in[b].record(up)
+        stream.wait_event(x_in[b])
+        stream.wait_event(y_out[b])  # the slot's previous result has been copied out
+        with torch.cuda.stream(stream):
+            st.run(dx[b], dy[b])
+            done[b].record(stream)
+        down.wait_event(done[b])
+        with torch.cuda.stream(down):
+            hy[b].copy_(dy[b], non_blocking=True)
+            y_out[b].record(down)
+
+    steps = max(2, min(args.steps, 4))
+    one(0)
+    torch.cuda.synchronize()
+    barrier(world)
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for s in range(steps):
+        one(s)
+    for e in y_out:
+        stream.wait_event(e)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier(world)
+    secs = e0.elapsed_time(e1) / 1e3
+    units, secs = aggregate(st.input_bytes * steps, secs, world, device)
+    del dx, dy
+    return {"value": round(units / secs / 1e9, 2), "unit": UNIT,
+            "h2d_bytes_per_step": 4 * N, "d2h_bytes_per_step": 4 * N, "steps": steps,
+            "api": "the step's 72 library calls through the Python binding; per step one H2D "
+                   "copy of the input from pinned memory and one D2H copy of a result, on copy "
+                   "streams, pipelined over two slots"}
+
+
+def measure_whole_tensor(mpc, synth, device, stream, peak, log2ns=(27, 28, 29)):
+    """Whole-tensor rows below the headline size: TopK and EF-TopK at K = 10 %, 4-bit
+    quantisation and the decompressions, each call timed between events over 3 calls in a
+    row (inputs of 512 MiB and more, larger than L2)."""
+    out = {}
+
+    def timed(fn, reps=3):
+        with torch.cuda.stream(stream):
+            fn()
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            for _ in range(reps):
+                fn()
+            b.record(stream)
+            stream.synchronize()
+        return a.elapsed_time(b) / reps
+
+    def rec(name, ms, nbytes):
+        gbs = nbytes / (ms / 1e3) / 1e9
+        out[name] = {"us": round(ms * 1e3, 1), "GBps": round(gbs, 1), "frac": round(gbs / peak, 4)}
+
+    for lg in log2ns:
+        N = 1 << lg
+        x = synth.normal((1, N), lg, device)
+        k = synth.k_of(N, 10)
+        ws = torch.empty(mpc.mpc_topk_workspace_bytes(1, N, k), dtype=torch.uint8, device=device)
+        v, i = mpc.mpc_topk_compress(x, k, ws=ws)
+        rec("topk_compress 2^%d K=10%%" % lg, timed(lambda: mpc.mpc_topk_compress(x, k, v, i, ws=ws)),
+            algorithmic_bytes(1, N, k=k, op="topk"))
+        y = torch.empty_like(x)
+        rec("topk_decompress 2^%d K=10%%" % lg, timed(lambda: mpc.mpc_topk_decompress(v, i, N, y=y)),
+            algorithmic_bytes(1, N, k=k, op="topk_decompress"))
+        e = torch.zeros_like(x)
+        rec("ef_topk_compress 2^%d K=10%%" % lg, timed(lambda: mpc.mpc_ef_topk_compress(x, e, k, v, i, ws=ws)),
+            algorithmic_bytes(1, N, k=k, op="ef_topk"))
+        del e, v, i, ws
+        qws = torch.empty(mpc.mpc_quant_workspace_bytes(1, N, 4), dtype=torch.uint8, device=device)
+        c, sc, mn = mpc.mpc_quant_compress(x, 4, ws=qws)
+        rec("quant_compress 2^%d 4-bit" % lg, timed(lambda: mpc.mpc_quant_compress(x, 4, codes=c, scale=sc, minv=mn, ws=qws)),
+            algorithmic_bytes(1, N, bits=4, op="quant"))
+        rec("quant_decompress 2^%d 4-bit" % lg, timed(lambda: mpc.mpc_quant_decompress(c, sc, mn, N, 4, y=y)),
+            algorithmic_bytes(1, N, bits=4, op="dequant"))
+        del x, y, c, qws
+        torch.cuda.empty_cache()
+    st = mpc.mpc_get_status(stream)
+    if st != 0:
+        raise RuntimeError("device status %d: %s" % (st, mpc.mpc_last_error()))
+    return out
+
+
+# ---------------------------------------------------------------------------------------
+# the CNN stage boundary (secondary key)
+# ---------------------------------------------------------------------------------------
 
 class Step:
     """Pre-allocated tensors and the launch sequence of one boundary step."""
@@ -469,46 +832,30 @@ def make_event(external: bool):
     return torch.cuda.Event(enable_timing=True)
 
 
-def run_ours(args, rank, local, world):
-    import paper_2401_07788_gb300 as mpc
-    from paper_2401_07788_gb300 import synth
-
-    device = torch.device("cuda", local)
-    torch.cuda.set_device(device)
-    init_dist(world, "nccl")
-    mpc.lib()
-    seed = rank % 10
-    st = Step(mpc, synth, device, seed)
+def run_cnn_step(args, mpc, synth, device, world):
+    """The CNN stage boundary [128,128,16,16] (the round of every operator that workload
+    sweeps, 18 library calls) as one CUDA graph per step, its nine independent
+    compress+decompress pairs on concurrent branches (--branches); a 256 MiB buffer written
+    then read before each step, outside the timed interval, takes the step's inputs out of
+    L2.  The dominant call is timed over 200 calls in a row on cold input copies."""
+    st = Step(mpc, synth, device, 0)
     n_ops = len(st.ops)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=device)
-    flush_sink = torch.empty((), dtype=torch.int64, device=device)
+    sink = torch.empty((), dtype=torch.int64, device=device)
     stream = torch.cuda.Stream(device)
     side = [torch.cuda.Stream(device) for _ in range(args.branches - 1)]
-    torch.cuda.synchronize()
 
     def flush_l2(i):
-        # write then read a buffer twice the size of L2: the step's inputs leave
-        # L2, and the flush leaves no dirty lines whose write-back the first
-        # launch of the step would pay for
         flush.fill_(i & 0xff)
-        torch.sum(flush.view(torch.int64), dim=0, out=flush_sink)
+        torch.sum(flush.view(torch.int64), dim=0, out=sink)
 
-    # eager warm-up (sets kernel attributes) before capture
     with torch.cuda.stream(stream):
         for w in range(2):
             st.launch(w % POOL, w)
             st.launch(w % POOL, w, side=side)
     stream.synchronize()
     assert mpc.mpc_get_status(stream) == 0, mpc.mpc_last_error()
-
-    # One graph per pool slot.  Event nodes inside a graph cost ~5 us each, so the
-    # headline steps replay event-free graphs; per-launch times come from a second
-    # timed pass with an event after every launch (shares of the step), and the
-    # dominant launch's duration from launches of it in a row on cold inputs
-    # (time_back_to_back).
-    if make_event(external=True) is None:
-        raise RuntimeError("torch.cuda.Event(external=True) is required")
-    keep = []  # events referenced by graph nodes must outlive the graphs
+    keep = []
 
     def capture(slot, **kw):
         g = torch.cuda.CUDAGraph()
@@ -517,49 +864,39 @@ def run_ours(args, rank, local, world):
         return g
 
     plain = [capture(slot, side=side) for slot in range(POOL)]
-    evsets = [[make_event(True) for _ in range(n_ops)] for _ in range(POOL)]
+    evsets = [[torch.cuda.Event(enable_timing=True, external=True) for _ in range(n_ops)]
+              for _ in range(POOL)]
     keep.append(evsets)
     evented = [capture(slot, events=evsets[slot]) for slot in range(POOL)]
     torch.cuda.synchronize()
+    steps = args.cnn_steps
 
-    def timed_pass(graphs, after_step=None, sampler=None):
-        starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-        ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    def timed_pass(graphs, after_step=None):
+        starts = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+        ends = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
         with torch.cuda.stream(stream):
-            for w in range(args.warmup):
+            for w in range(max(3, args.warmup)):
                 flush_l2(w)
                 graphs[w % POOL].replay()
         stream.synchronize()
         barrier(world)
-        torch.cuda.synchronize()
-        if sampler is not None:
-            sampler.__enter__()
-        t0 = time.perf_counter()
         with torch.cuda.stream(stream):
-            for i in range(args.steps):
+            for i in range(steps):
                 flush_l2(i)
                 starts[i].record(stream)
                 graphs[i % POOL].replay()
                 ends[i].record(stream)
-                if after_step is not None and ((i + 1) % POOL == 0 or i == args.steps - 1):
-                    # events inside a graph belong to its slot: read them before reuse
+                if after_step is not None and ((i + 1) % POOL == 0 or i == steps - 1):
                     stream.synchronize()
                     for j in range(i - (i % POOL), i + 1):
                         after_step(j, starts[j], ends[j])
         stream.synchronize()
-        torch.cuda.synchronize()
-        wall = time.perf_counter() - t0
-        if sampler is not None:
-            sampler.__exit__(None, None, None)
         barrier(world)
-        return sum(starts[i].elapsed_time(ends[i]) for i in range(args.steps)) / 1e3, wall
+        return sum(starts[i].elapsed_time(ends[i]) for i in range(steps)) / 1e3
 
     for p in TOPK_PCTS:
         st.errs[p].zero_()
-    sampler = ClockSampler(local)
-    dev_s, wall = timed_pass(plain, sampler=sampler)
-    clocks = sampler.summary()
-
+    dev_s = timed_pass(plain)
     op_ms = [0.0] * n_ops
 
     def read_ops(j, start, end):
@@ -571,74 +908,26 @@ def run_ours(args, rank, local, world):
     timed_pass(evented, read_ops)
     dom = max(range(n_ops), key=lambda j: op_ms[j])
     dom_ms = time_back_to_back(st, dom, stream, flush_l2)
-    alone_ms = time_alone(st, dom, stream, flush_l2, min(args.steps, 300), args.warmup)
     status = mpc.mpc_get_status(stream)
     if status != 0:
         raise RuntimeError("device status %d: %s" % (status, mpc.mpc_last_error()))
-
-    units, secs = aggregate(st.input_bytes * args.steps, dev_s, world, device)
-    value = units / secs / 1e9
-
-    # roofline of the dominant kernel (largest share of the step)
-    peak, peak_kind = hbm_peak()
+    units, secs = aggregate(st.input_bytes * steps, dev_s, world, device)
+    peak, _ = hbm_peak()
     name, nbytes = st.ops[dom]
-    avg_ms = dom_ms
-    achieved = nbytes / (avg_ms / 1e3) / 1e9
-    kern = "topk_cta_kernel" if "topk_compress" in name else (
-        "topk_decompress_rows_kernel" if "decompress K" in name else (
-            "quant_cta_kernel" if "quant_compress" in name else "dequant_rows_kernel"))
-    traffic = recorded_traffic(kern + ":" + name.replace(" ", "_"))
-    roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
-                "frac": round(achieved / peak, 4), "traffic": traffic,
-                "kernel": kern, "op": name, "algorithmic_bytes": nbytes,
-                "avg_launch_us": round(avg_ms * 1e3, 2),
-                "share_of_step": round(op_ms[dom] / max(sum(op_ms), 1e-9), 4),
-                "peak_source": peak_kind,
-                "timing": "200 launches in a row on its stream between two CUDA events, "
-                          "inputs cycling through 8 copies (twice the L2), so every launch "
-                          "reads cold inputs",
-                "alone_us": round(alone_ms * 1e3, 2),
-                "alone_timing": "one launch after an L2 flush between two events behind a "
-                                "GPU-side sleep (median of %d); includes the ~5 us an event "
-                                "pair adds around any launch" % min(args.steps, 300)}
-    per_op = {st.ops[j][0]: {"avg_us": round(op_ms[j] / args.steps * 1e3, 2),
-                             "GBps": round(st.ops[j][1] / (op_ms[j] / args.steps / 1e3) / 1e9, 1)}
-              for j in range(n_ops)}
-
-    # end to end through the Python API: host inputs in, two outputs back, no graphs
-    e2e = run_e2e(args, st, stream, side, world, device)
-
-    operators = None
-    if not args.no_operators and rank == 0:
-        operators = measure_operators(mpc, synth, device, stream, peak)
-
-    cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = cpu_baseline(budget_s=10.0)
-
-    if rank == 0:
-        line = {
-            "metric": METRIC, "value": round(value, 2), "unit": UNIT, "n_gpus": world,
-            "steps": args.steps, "warmup": args.warmup,
-            "ms_per_step": round(secs * 1e3 / args.steps, 4), "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-            "config": {"workload": WORKLOAD, "rows": R, "row_len": L,
-                       "topk_percents": list(TOPK_PCTS), "bits": list(BITS),
-                       "rounding": ["nearest", "stochastic"], "launches_per_step": n_ops,
-                       "step": "one CUDA graph per step (no event nodes inside); " + BRANCH_TEXT[args.branches],
-                       "l2": "256 MiB buffer "
-                       "written then read before each timed step, outside the timed interval "
-                       "(inputs cold, no dirty lines left by the flush)", "parallelism":
-                       "replicas" if world > 1 else "single GPU"},
-            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
-            "gpu_launches": n_ops * args.steps, "clocks": clocks,
-            "wall_s": round(wall, 3), "per_op": per_op,
-            "per_op_timing": "an event after every launch inside a graph of the 18 launches in "
-                             "order on one stream (second pass; each interval includes the ~5 us "
-                             "of an event node)",
-            "operators": operators,
-        }
-        print(json.dumps(line), flush=True)
+    achieved = nbytes / (dom_ms / 1e3) / 1e9
+    del plain, evented, keep, flush
+    return {"workload": "CNN stage boundary [128,128,16,16] fp32, 128 rows x 32768",
+            "value": round(units / secs / 1e9, 2), "unit": UNIT, "steps": steps,
+            "ms_per_step": round(secs * 1e3 / steps, 4), "launches_per_step": n_ops,
+            "step": "one CUDA graph per step (no event nodes inside); " + BRANCH_TEXT[args.branches],
+            "l2": "256 MiB buffer written then read before each timed step, outside the timed "
+                  "interval",
+            "dominant": {"op": name, "avg_launch_us": round(dom_ms * 1e3, 2),
+                         "achieved": round(achieved, 1), "frac": round(achieved / peak, 4),
+                         "algorithmic_bytes": nbytes,
+                         "timing": "200 launches in a row on its stream between two CUDA "
+                                   "events, inputs cycling through 8 copies (twice the L2)"},
+            "per_op_us": {st.ops[j][0]: round(op_ms[j] / steps * 1e3, 2) for j in range(n_ops)}}
 
 
 def time_back_to_back(st, i, stream, flush_l2, rounds=25, n_sets=8):
@@ -669,103 +958,9 @@ def time_back_to_back(st, i, stream, flush_l2, rounds=25, n_sets=8):
     return a.elapsed_time(b) / (rounds * n_sets)
 
 
-def time_alone(st, i, stream, flush_l2, n, warmup):
-    """Median device time (ms) of launch i of the step on its own, on cold inputs: after
-    each L2 flush a GPU-side sleep of ~50 us lets the host enqueue the two events and
-    the launch before the stream reaches them, so the interval holds the launch alone."""
-    with torch.cuda.stream(stream):
-        for w in range(warmup):
-            flush_l2(w)
-            st.launch(w % POOL, w, only=i)
-        stream.synchronize()
-        pairs = []
-        for s in range(n):
-            flush_l2(s)
-            torch.cuda._sleep(100_000)
-            a = torch.cuda.Event(enable_timing=True)
-            b = torch.cuda.Event(enable_timing=True)
-            a.record(stream)
-            st.launch(s % POOL, s, only=i)
-            b.record(stream)
-            pairs.append((a, b))
-        stream.synchronize()
-    ts = [a.elapsed_time(b) for a, b in pairs]
-    return statistics.median(ts)
-
-
-def run_e2e(args, st, stream, side, world, device):
-    """The step end to end through the Python API: every step copies its two inputs from
-    pinned host memory to the device and two of its results back, inside the timed
-    region.  Copies and compute are pipelined over two slots (inputs and read-back
-    outputs double-buffered; step s+1's inputs go up while step s computes and step
-    s-1's results come down), each copy on its own stream; the compute of a slot is the
-    step's API calls captured once into a CUDA graph (its branches as in the headline)."""
-    mpc = st.mpc
-    hx = [t.cpu().pin_memory() for t in st.xs]
-    hg = [t.cpu().pin_memory() for t in st.gs]
-    k10, q8 = 10, (8, True)  # read back: the K=10% activation, the 8-bit stochastic gradient
-    dx = [torch.empty_like(st.xs[0]) for _ in range(2)]
-    dg = [torch.empty_like(st.gs[0]) for _ in range(2)]
-    dy = [torch.empty((R, L), device=device) for _ in range(2)]
-    dgy = [torch.empty((R, L), device=device) for _ in range(2)]
-    hy = [torch.empty((R, L), pin_memory=True) for _ in range(2)]
-    hgy = [torch.empty((R, L), pin_memory=True) for _ in range(2)]
-    up = [torch.cuda.Stream(device) for _ in range(2)]
-    down = [torch.cuda.Stream(device) for _ in range(2)]
-    ev = lambda: [torch.cuda.Event() for _ in range(2)]  # noqa: E731
-    x_in, g_in, done, y_out, g_out = ev(), ev(), ev(), ev(), ev()
-
-    graphs = []
-    for slot in range(2):
-        g = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g, stream=stream):
-            st.launch(slot, slot, x=dx[slot], g=dg[slot], side=side,
-                      y={k10: dy[slot]}, gy={q8: dgy[slot]})
-        graphs.append(g)
-
-    def one(s):
-        b = s % 2
-        for stm, dst, src, e in ((up[0], dx[b], hx[s % POOL], x_in[b]),
-                                 (up[1], dg[b], hg[s % POOL], g_in[b])):
-            stm.wait_event(done[b])  # the slot's previous compute has read it
-            with torch.cuda.stream(stm):
-                dst.copy_(src, non_blocking=True)
-                e.record(stm)
-        for e in (x_in[b], g_in[b], y_out[b], g_out[b]):
-            stream.wait_event(e)
-        with torch.cuda.stream(stream):
-            graphs[b].replay()
-            done[b].record(stream)
-        for stm, dst, src, e in ((down[0], hy[b], dy[b], y_out[b]),
-                                 (down[1], hgy[b], dgy[b], g_out[b])):
-            stm.wait_event(done[b])
-            with torch.cuda.stream(stm):
-                dst.copy_(src, non_blocking=True)
-                e.record(stm)
-
-    steps = max(3, min(args.steps, 50))
-    for s in range(3):
-        one(s)
-    torch.cuda.synchronize()
-    barrier(world)
-    e0 = torch.cuda.Event(enable_timing=True)
-    e1 = torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for s in range(steps):
-        one(s)
-    for e in y_out + g_out:
-        stream.wait_event(e)
-    e1.record(stream)
-    torch.cuda.synchronize()
-    barrier(world)
-    secs = e0.elapsed_time(e1) / 1e3
-    units, secs = aggregate(st.input_bytes * steps, secs, world, device)
-    return {"value": round(units / secs / 1e9, 2), "unit": UNIT,
-            "h2d_bytes_per_step": 2 * 4 * R * L, "d2h_bytes_per_step": 2 * 4 * R * L,
-            "steps": steps, "api": "python binding calls of one step captured into a CUDA "
-            "graph per input slot; per step two H2D copies from pinned memory and two D2H "
-            "copies of results on copy streams, pipelined over two slots"}
-
+# ---------------------------------------------------------------------------------------
+# every operator on its own workload
+# ---------------------------------------------------------------------------------------
 
 def time_op(fn, stream, flush, reps=8):
     """Device time (ms) of one launch of fn on cold inputs, inside a CUDA graph: a graph of
@@ -893,46 +1088,33 @@ def measure_operators(mpc, synth, device, stream, peak):
         algorithmic_bytes(16 * rps, La, bits=4, op="aqsgd_dequant_add"))
     del buf, xa, wsq
     torch.cuda.empty_cache()
-    # bandwidth sweep point: one 1 GiB tensor
+    # sweep point of 2^28 entries: the calls the headline step does not make (index reuse,
+    # stochastic rounding, 6-bit codes) at each row length
     N = 1 << 28
     xs = synth.normal((N,), 28, device)
     for Ls in (768, 4096, 65536):
         Rs = N // Ls
         xv = xs[: Rs * Ls].view(Rs, Ls)
-        for pct in (1, 10, 50):
-            ks = synth.k_of(Ls, pct)
-            vs, is_ = mpc.mpc_topk_compress(xv, ks)
-            rec("topk_compress 2^28 L=%d K=%d%%" % (Ls, pct), time_op(lambda: mpc.mpc_topk_compress(xv, ks, vs, is_), stream, flush),
-                algorithmic_bytes(Rs, Ls, k=ks, op="topk"))
-            if pct == 10:
-                gvs = mpc.mpc_topk_gather(xv, is_)
-                rec("topk_gather 2^28 L=%d K=10%%" % Ls, time_op(lambda: mpc.mpc_topk_gather(xv, is_, vals=gvs), stream, flush),
-                    algorithmic_bytes(Rs, Ls, k=ks, op="topk_gather"))
-                del gvs
-                ys = torch.empty_like(xv)
-                rec("topk_decompress 2^28 L=%d K=10%%" % Ls, time_op(lambda: mpc.mpc_topk_decompress(vs, is_, Ls, y=ys), stream, flush),
-                    algorithmic_bytes(Rs, Ls, k=ks, op="topk_decompress"))
-                es = torch.zeros_like(xv)
-                rec("ef_topk_compress 2^28 L=%d K=10%%" % Ls, time_op(lambda: mpc.mpc_ef_topk_compress(xv, es, ks, vs, is_), stream, flush),
-                    algorithmic_bytes(Rs, Ls, k=ks, op="ef_topk"))
-                del ys, es
-            del vs, is_
-        for b in BITS + (6,):
+        ks = synth.k_of(Ls, 10)
+        vs, is_ = mpc.mpc_topk_compress(xv, ks)
+        gvs = mpc.mpc_topk_gather(xv, is_)
+        rec("topk_gather 2^28 L=%d K=10%%" % Ls, time_op(lambda: mpc.mpc_topk_gather(xv, is_, vals=gvs), stream, flush),
+            algorithmic_bytes(Rs, Ls, k=ks, op="topk_gather"))
+        gs = torch.zeros_like(xv)
+        rec("ef21_topk_compress 2^28 L=%d K=10%%" % Ls, time_op(lambda: mpc.mpc_ef21_topk_compress(xv, gs, ks, vs, is_), stream, flush),
+            algorithmic_bytes(Rs, Ls, k=ks, op="delta_topk"))
+        del gvs, vs, is_, gs
+        for b, sr in ((4, True), (8, True), (6, False)):
             cq, sq, mq = mpc.mpc_quant_compress(xv, b)
-            rec("quant_compress 2^28 L=%d %d-bit" % (Ls, b), time_op(lambda: mpc.mpc_quant_compress(xv, b, codes=cq, scale=sq, minv=mq), stream, flush),
+            rec("quant_compress 2^28 L=%d %d-bit %s" % (Ls, b, "stochastic" if sr else "nearest"),
+                time_op(lambda: mpc.mpc_quant_compress(xv, b, sr, 7, codes=cq, scale=sq, minv=mq), stream, flush),
                 algorithmic_bytes(Rs, Ls, bits=b, op="quant"))
             if b == 6:
                 ys = torch.empty_like(xv)
                 rec("quant_decompress 2^28 L=%d 6-bit" % Ls, time_op(lambda: mpc.mpc_quant_decompress(cq, sq, mq, Ls, 6, y=ys), stream, flush),
                     algorithmic_bytes(Rs, Ls, bits=6, op="dequant"))
                 del ys
-            if b == 4:
-                rec("quant_compress 2^28 L=%d 4-bit stochastic" % Ls, time_op(lambda: mpc.mpc_quant_compress(xv, 4, True, 7, codes=cq, scale=sq, minv=mq), stream, flush),
-                    algorithmic_bytes(Rs, Ls, bits=4, op="quant"))
-                ys = torch.empty_like(xv)
-                rec("quant_decompress 2^28 L=%d 4-bit" % Ls, time_op(lambda: mpc.mpc_quant_decompress(cq, sq, mq, Ls, 4, y=ys), stream, flush),
-                    algorithmic_bytes(Rs, Ls, bits=4, op="dequant"))
-                del ys
+            del cq, sq, mq
     del xs
     torch.cuda.empty_cache()
     st = mpc.mpc_get_status(stream)
@@ -945,8 +1127,15 @@ def measure_operators(mpc, synth, device, stream, peak):
 # CPU oracle (the reference arm and the cpu_baseline key)
 # ---------------------------------------------------------------------------------------
 
+# Bounded sample of the headline step for the single-threaded oracle: entries per row
+# length (whole rows of 768, 4096 and 65536 entries), and one whole-tensor row of 2^20.
+ORACLE_SAMPLE = ((768, 1 << 17), (4096, 1 << 17), (65536, 1 << 17), (None, 1 << 20))
+
+
 class OracleStep:
-    """The same boundary step on SAMPLE_ROWS of the 128 rows, computed by the oracle."""
+    """The headline step on the bounded sample, computed by the oracle: for each row length
+    the same 18 calls (TopK and EF-TopK at 1/10/50 % with decompression, 2/4/8-bit
+    quantisation with dequantisation)."""
 
     def __init__(self, seed: int = 0):
         import oracle
@@ -954,23 +1143,30 @@ class OracleStep:
 
         self.oracle = oracle
         self.lib = oracle.load()
-        x = synth.relu_normal((R, L), seed, "cpu")[:SAMPLE_ROWS].numpy().copy()
-        g = synth.normal((R, L), 1000 + 100 * seed, "cpu", std=1e-3)[:SAMPLE_ROWS].numpy().copy()
-        self.x, self.g = x, g
-        self.ks = {p: synth.k_of(L, p) for p in TOPK_PCTS}
-        self.errs = {p: np.zeros_like(x) for p in TOPK_PCTS}
-        self.seed = seed
-        self.input_bytes = 9 * 4 * SAMPLE_ROWS * L
+        self.parts = []
+        for Ls, n in ORACLE_SAMPLE:
+            Lr = n if Ls is None else Ls
+            Rr = n // Lr
+            x = synth.normal((Rr, Lr), 1000 * seed + 30, "cpu").numpy().copy()
+            ks = {p: synth.k_of(Lr, p) for p in SWEEP_PCTS}
+            errs = {p: np.zeros_like(x) for p in SWEEP_PCTS}
+            self.parts.append((Rr, Lr, x, ks, errs))
+        self.input_bytes = sum(9 * 4 * Rr * Lr for Rr, Lr, _, _, _ in self.parts)  # 9 pairs
+        self.sample = ("per row length, the first %s entries as rows (768, 4096, 65536) and a "
+                       "whole-tensor row of %d entries; every call of the step on them"
+                       % ("/".join(str(n) for _, n in ORACLE_SAMPLE[:3]), ORACLE_SAMPLE[3][1]))
 
     def run(self, step: int):
-        o = self.oracle
-        for p in TOPK_PCTS:
-            v, i = o.ef_topk_compress(self.x, self.errs[p], self.ks[p], self.lib)
-            o.topk_decompress(v, i, L, self.lib)
-        for b in BITS:
-            for sr in (False, True):
-                c, s, m = o.quant_compress(self.g, b, sr, (self.seed << 32) | step, self.lib)
-                o.quant_decompress(c, s, m, L, b, self.lib)
+        o, lib = self.oracle, self.lib
+        for Rr, Lr, x, ks, errs in self.parts:
+            for p in SWEEP_PCTS:
+                v, i = o.topk_compress(x, ks[p], lib)
+                o.topk_decompress(v, i, Lr, lib)
+                v, i = o.ef_topk_compress(x, errs[p], ks[p], lib)
+                o.topk_decompress(v, i, Lr, lib)
+            for b in SWEEP_BITS:
+                c, s, m = o.quant_compress(x, b, False, 0, lib)
+                o.quant_decompress(c, s, m, Lr, b, lib)
 
 
 def cpu_baseline(budget_s: float = 10.0):
@@ -982,8 +1178,8 @@ def cpu_baseline(budget_s: float = 10.0):
         n += 1
     secs = time.perf_counter() - t0
     return {"value": round(st.input_bytes * n / secs / 1e9, 4), "unit": UNIT, "cores": 1,
-            "kind": "oracle", "sample": "%d of %d rows of the step, %d steps in %.1f s"
-            % (SAMPLE_ROWS, R, n, secs), "cpu": cpu_name()}
+            "kind": "oracle", "sample": st.sample + "; %d passes in %.1f s" % (n, secs),
+            "cpu": cpu_name()}
 
 
 def cpu_name():
@@ -1012,77 +1208,17 @@ def run_reference(args, rank, world):
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": round(secs * 1e3 / args.steps, 3), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-        "config": {"workload": WORKLOAD, "rows": R, "row_len": L,
-                   "topk_percents": list(TOPK_PCTS), "bits": list(BITS),
-                   "sample_rows": SAMPLE_ROWS},
+        "config": {"workload": "bandwidth sweep at 2^%d entries: one N(0,1) fp32 tensor of "
+                               "%d entries as rows of 768, 4096, 65536 and one whole-tensor row"
+                               % (LOG2N, 1 << LOG2N),
+                   "topk_percents": list(SWEEP_PCTS), "bits": list(SWEEP_BITS),
+                   "oracle_sample": st.sample},
         "cpu_baseline": {"value": round(value, 4), "unit": UNIT, "cores": 1, "kind": "oracle",
-                         "sample": "%d of %d rows of each step" % (SAMPLE_ROWS, R),
-                         "cpu": cpu_name()},
+                         "sample": st.sample, "cpu": cpu_name()},
         "e2e": {"value": round(value, 4), "unit": UNIT, "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
-
-
-def run_sweep():
-    """The size sweep of the bandwidth study: N = 2^20..2^30 N(0,1) entries as rows of
-    L in {768, 4096, 65536, N} (N itself only up to 2^26, the on-chip row path's reach
-    being 65536 and the grid path's workspace growing with the row); TopK and EF-TopK at
-    K = 1, 10, 50 %, 2/4/8-bit quantisation and 4-bit dequantisation, each launch timed
-    inside a CUDA graph on cold inputs as in `operators`."""
-    import paper_2401_07788_gb300 as mpc
-    from paper_2401_07788_gb300 import synth
-
-    device = torch.device("cuda", 0)
-    torch.cuda.set_device(device)
-    stream = torch.cuda.Stream(device)
-    flush = torch.empty(256 << 20, dtype=torch.uint8, device=device)
-    peak, _ = hbm_peak()
-    table = []
-    for log2n in range(20, 31):
-        N = 1 << log2n
-        xs = synth.normal((N,), log2n, device)
-        for Ls in (768, 4096, 65536) + ((N,) if log2n <= 26 else ()):
-            Rs = N // Ls
-            if Rs < 1:
-                continue
-            xv = xs[: Rs * Ls].view(Rs, Ls)
-            entries = []
-            for pct in (1, 10, 50):
-                ks = synth.k_of(Ls, pct)
-                vs, is_ = mpc.mpc_topk_compress(xv, ks)
-                ws = None
-                need = mpc.mpc_topk_workspace_bytes(Rs, Ls, ks)
-                if need:
-                    ws = torch.empty(need, dtype=torch.uint8, device=device)
-                entries.append(("topk K=%d%%" % pct, time_op(lambda: mpc.mpc_topk_compress(xv, ks, vs, is_, ws=ws), stream, flush),
-                                algorithmic_bytes(Rs, Ls, k=ks, op="topk")))
-                es = torch.zeros_like(xv)
-                entries.append(("ef_topk K=%d%%" % pct, time_op(lambda: mpc.mpc_ef_topk_compress(xv, es, ks, vs, is_, ws=ws), stream, flush),
-                                algorithmic_bytes(Rs, Ls, k=ks, op="ef_topk")))
-                del es, vs, is_, ws
-            for b in ((2, 4, 8) if Ls <= 0x7fffffff // 32 else ()):  # the quantiser's row limit
-                cq, sq, mq = mpc.mpc_quant_compress(xv, b)
-                entries.append(("quant %d-bit" % b, time_op(lambda: mpc.mpc_quant_compress(xv, b, codes=cq, scale=sq, minv=mq), stream, flush),
-                                algorithmic_bytes(Rs, Ls, bits=b, op="quant")))
-                if b == 4:
-                    ys = torch.empty_like(xv)
-                    entries.append(("dequant 4-bit", time_op(lambda: mpc.mpc_quant_decompress(cq, sq, mq, Ls, 4, y=ys), stream, flush),
-                                    algorithmic_bytes(Rs, Ls, bits=4, op="dequant")))
-                    del ys
-                del cq, sq, mq
-            for name, ms, nbytes in entries:
-                gbs = nbytes / (ms / 1e3) / 1e9
-                table.append({"log2n": log2n, "row_len": Ls, "op": name, "us": round(ms * 1e3, 2),
-                              "GBps": round(gbs, 1), "frac": round(gbs / peak, 4)})
-        del xs
-        torch.cuda.empty_cache()
-    st = mpc.mpc_get_status(stream)
-    if st != 0:
-        raise RuntimeError("device status %d: %s" % (st, mpc.mpc_last_error()))
-    print(json.dumps({"sweep": table, "peak": peak, "unit": "GB/s", "timing": "each launch "
-                      "inside a CUDA graph on cold inputs (flush-and-launch graph against a "
-                      "flush-only graph)"}), flush=True)
 
 
 def main():
@@ -1091,11 +1227,7 @@ def main():
     if args.impl == "reference":
         run_reference(args, rank, world)
         return
-    if args.sweep:
-        if rank == 0:
-            run_sweep()
-        return
-    run_ours(args, rank, local, world)
+    run_headline(args, rank, local, world)
     if world > 1:
         import torch.distributed as dist
 

@@ -16,26 +16,36 @@ def _bench():
 
 
 def test_traffic_table_parses():
+    """The table parses, names one source digest, and every entry is a call of the
+    headline step with a positive byte count, not below the bytes the call must read."""
     lines = open(os.path.join(ROOT, "profiles", "dram_traffic.txt")).read().splitlines()
     digests = [ln.split()[1] for ln in lines if ln.startswith("source_digest ")]
     assert len(digests) == 1 and len(digests[0]) == 16
-    entries = {ln.split()[0]: float(ln.split()[1]) for ln in lines
-               if ln.strip() and not ln.startswith("#") and not ln.startswith("source_digest")}
+    entries = {}
+    for ln in lines:
+        if ln.strip() and not ln.startswith("#") and not ln.startswith("source_digest"):
+            name, value = ln.rsplit(None, 1)
+            entries[name] = float(value)
     b = _bench()
-    kern = lambda o: ("topk_cta_kernel" if "topk_compress" in o else  # noqa: E731
-                      "topk_decompress_rows_kernel" if "decompress K" in o else
-                      "quant_cta_kernel" if "quant_compress" in o else "dequant_rows_kernel")
-    ops = ["ef_topk_compress K=%d%%" % p for p in b.TOPK_PCTS]
-    ops += ["topk_decompress K=%d%%" % p for p in b.TOPK_PCTS]
-    for bits in b.BITS:
-        for sr in ("nearest", "stochastic"):
-            ops += ["quant_compress %d-bit %s" % (bits, sr), "quant_decompress %d-bit %s" % (bits, sr)]
-    for o in ops:
-        key = kern(o) + ":" + o.replace(" ", "_")
-        assert key in entries and entries[key] > 0, key
-    # inputs read once: an error-feedback TopK launch reads x and err, 2 x 16.8 MB
-    ef = entries["topk_cta_kernel:ef_topk_compress_K=5%"]
-    assert 2 * 4 * b.R * b.L * 0.99 <= ef <= 2 * 4 * b.R * b.L * 1.05
+    names = set(b.headline_call_names())
+    assert entries, "empty traffic table"
+    N = 1 << b.LOG2N
+    for name, v in entries.items():
+        assert name in names, name
+        # every compress call reads its 4 GiB input at least once
+        if "compress" in name and "decompress" not in name:
+            assert v >= 4 * N * 0.99, (name, v)
+
+
+def test_headline_calls():
+    """36 compress+decompress pairs per headline step: for each of the four row lengths,
+    TopK and EF-TopK at three K and three code widths."""
+    b = _bench()
+    names = b.headline_call_names()
+    assert len(names) == 72 and len(set(names)) == 72
+    assert sum("decompress" in n for n in names) == 36
+    for L in ("768", "4096", "65536", "N"):
+        assert sum(("L=%s " % L) in n for n in names) == 18
 
 
 def test_step_branch_layouts():
