@@ -122,6 +122,8 @@ mpc_status topk_compress_common(int mode, const float* x, float* aux, int64_t ro
   if (use_row_path(row_len)) {
     mpc::TopkRowArgs a = {};
     a.wide_cta = g_topk_path.load() != 3;
+  a.band = g_topk_path.load() != 4;
+    a.band = g_topk_path.load() != 4;
     a.x = x;
     a.aux = aux;
     a.rows = rows;
@@ -306,6 +308,7 @@ mpc_status mpc_aqsgd_compress(const float* x, float* buf, int64_t num_samples,
   MPC_TRY(current_device(&d));
   mpc::TopkRowArgs a = {};
   a.wide_cta = g_topk_path.load() != 3;
+  a.band = g_topk_path.load() != 4;
   a.x = x;
   a.aux = buf;
   a.ids = sample_ids;
@@ -590,7 +593,7 @@ mpc_status mpc_set_knob(mpc_knob knob, int64_t value) {
       g_spin_limit.store(static_cast<uint32_t>(value));
       return ok();
     case MPC_KNOB_TOPK_PATH:
-      if (value < 0 || value > 3) return set_error(MPC_ERR_INVALID_ARG, "topk path");
+      if (value < 0 || value > 4) return set_error(MPC_ERR_INVALID_ARG, "topk path");
       g_topk_path.store(static_cast<int>(value));
       return ok();
     default:

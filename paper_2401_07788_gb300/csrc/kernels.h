@@ -31,6 +31,7 @@ struct TopkRowArgs {
   uint32_t spin_limit;    // polls before a wait gives up
   unsigned* status;       // device status word
   int wide_cta;           // 1: rows of 8193..32768 entries may take one wide CTA each
+  int band;               // 1: rows of 1025..8192 entries take the band kernel
 };
 
 // Largest row the on-chip row path handles (cluster of 8 CTAs x 8192).

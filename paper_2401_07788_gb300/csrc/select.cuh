@@ -43,6 +43,29 @@ __device__ __forceinline__ int bucket_of(int key, float scale, int nb) {
   return min(b, nb - 1);
 }
 
+// The smallest key of bin b (b >= 1) of an |x|-linear histogram (bucket_of, or
+// any bin rule that floors |x| * scale): the least c >= 0 with
+// |x(c)| * scale >= b.  `inv` = 1 / scale, rounded; the start point it gives
+// is a few units off at most and is corrected step by step, with bisection as
+// the bound-free fallback.
+__device__ __forceinline__ int bin_first_key(int b, float scale, float inv) {
+  const float fb = static_cast<float>(b);
+  auto reaches = [&](int c) { return fmul(__int_as_float(c), scale) >= fb; };
+  int c = min(__float_as_int(fmul(fb, inv)), 0x7f800000);
+  for (int i = 0; i < 8 && c > 0 && reaches(c - 1); ++i) --c;
+  for (int i = 0; i < 8 && !reaches(c); ++i) ++c;
+  if (!reaches(c) || (c > 0 && reaches(c - 1))) {
+    int lo = 0, hi = 0x7f800000;  // reaches(hi), !reaches(lo)
+    while (hi - lo > 1) {
+      const int mid = lo + (hi - lo) / 2;
+      if (reaches(mid)) hi = mid;
+      else lo = mid;
+    }
+    c = hi;
+  }
+  return c;
+}
+
 // Shift that maps the key range [lo, hi] (hi > lo) onto at most 256 bins.
 __device__ __forceinline__ int round_shift(int lo, int hi) {
   uint32_t span = static_cast<uint32_t>(hi - lo);

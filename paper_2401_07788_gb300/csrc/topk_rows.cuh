@@ -33,6 +33,7 @@
 #include "kernels.h"
 #include "launch_util.h"
 #include "select.cuh"
+#include "topk_band.cuh"
 
 namespace mpc {
 namespace rows {
@@ -81,28 +82,6 @@ __device__ __forceinline__ void keys4(const float4 v, int base, int n, int k[4])
 __device__ __forceinline__ int lin_bin(int key, float scale) {
   const float p = fminf(fmul(__int_as_float(key), scale), static_cast<float>(kNB - 1));
   return __float_as_int(__fadd_rz(p, 8388608.0f)) & 0x7fffff;
-}
-
-// The smallest key of bin b (1 <= b < kNB): the least c >= 0 with
-// |x(c)| * scale >= b.  `inv` = 1 / scale, rounded; the start point it gives
-// is a few units off at most and is corrected step by step, with bisection as
-// the bound-free fallback.
-__device__ __forceinline__ int bin_first_key(int b, float scale, float inv) {
-  const float fb = static_cast<float>(b);
-  auto reaches = [&](int c) { return fmul(__int_as_float(c), scale) >= fb; };
-  int c = min(__float_as_int(fmul(fb, inv)), 0x7f800000);
-  for (int i = 0; i < 8 && c > 0 && reaches(c - 1); ++i) --c;
-  for (int i = 0; i < 8 && !reaches(c); ++i) ++c;
-  if (!reaches(c) || (c > 0 && reaches(c - 1))) {
-    int lo = 0, hi = 0x7f800000;  // reaches(hi), !reaches(lo)
-    while (hi - lo > 1) {
-      const int mid = lo + (hi - lo) / 2;
-      if (reaches(mid)) hi = mid;
-      else lo = mid;
-    }
-    c = hi;
-  }
-  return c;
 }
 
 // ---------------------------------------------------------------------------
@@ -1288,6 +1267,9 @@ cudaError_t run_mode(const TopkRowArgs& a0, int num_sms, cudaStream_t s) {
   if (L <= 512) return run_warp_any<MODE, 4>(a, num_sms, s);
   if (L <= 768) return run_warp_any<MODE, 6>(a, num_sms, s);
   if (L <= 1024) return run_warp_any<MODE, 8>(a, num_sms, s);
+  // Rows of 1025..8192 entries take the band kernel (topk_band.cuh) unless the
+  // knob keeps the kernels below.
+  if (a.band && band::fits(L)) return band::run_mode<MODE>(a, s);
   // One CTA of 128 threads for rows up to 4096 entries, else clusters of
   // 256-thread CTAs holding up to 8192 entries each, split further (slices of
   // at least 2048 entries) while the grid has fewer than 2 CTAs per SM.

@@ -103,7 +103,7 @@ def test_aqsgd_validation(lib):
 def test_knobs(lib):
     assert lib.mpc_set_knob(99, 0) == 1
     assert lib.mpc_set_knob(2, 5) == 1
-    assert lib.mpc_set_knob(2, 4) == 1
+    assert lib.mpc_set_knob(2, 4) == 0  # rows of 1025..8192 entries without the band kernel
     assert lib.mpc_set_knob(2, 3) == 0  # rows of 8193..32768 entries on clusters only
     assert lib.mpc_set_knob(2, 0) == 0
     assert lib.mpc_set_knob(3, 2) == 1  # programmatic dependent launch: 0 or 1
