@@ -66,6 +66,13 @@ __device__ __forceinline__ int bin_first_key(int b, float scale, float inv) {
   return c;
 }
 
+// w |= bit when |v| >= t: one compare and one predicated OR, no branch.
+__device__ __forceinline__ void or_if_ge(uint32_t& w, float v, float t, uint32_t bit) {
+  asm("{\n .reg .pred p;\n setp.ge.f32 p, %1, %2;\n @p or.b32 %0, %0, %3;\n}"
+      : "+r"(w)
+      : "f"(fabsf(v)), "f"(t), "r"(bit));
+}
+
 // Shift that maps the key range [lo, hi] (hi > lo) onto at most 256 bins.
 __device__ __forceinline__ int round_shift(int lo, int hi) {
   uint32_t span = static_cast<uint32_t>(hi - lo);

@@ -87,13 +87,6 @@ __device__ __forceinline__ float ranked(float x, float a) {
 
 __device__ __forceinline__ uint32_t ukey(float v) { return __float_as_uint(v) & 0x7fffffffu; }
 
-// w |= bit when |v| >= t: one compare and one predicated OR, no branch.
-__device__ __forceinline__ void or_if_ge(uint32_t& w, float v, float t, uint32_t bit) {
-  asm("{\n .reg .pred p;\n setp.ge.f32 p, %1, %2;\n @p or.b32 %0, %0, %3;\n}"
-      : "+r"(w)
-      : "f"(fabsf(v)), "f"(t), "r"(bit));
-}
-
 // Two bins of a 256-bin histogram (bins ranked from high to low) from one scan:
 // the bins holding the r1-th and the r2-th elements (r = 0 or r past the total:
 // bin -1).

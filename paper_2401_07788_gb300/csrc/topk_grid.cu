@@ -1,26 +1,49 @@
 // topk_grid.cu -- exact TopK (§2.3), with error feedback (§2.4) or the EF21
-// buffer update (§2.4), for rows longer than one thread-block cluster holds
-// (up to whole tensors of 2^31-1 entries).  Multi-pass, with the counters and
-// candidates in a caller workspace; one row at a time.
+// buffer update (§2.4), for rows longer than the on-chip row kernels take (up
+// to whole tensors of 2^31-1 entries), with the counters, lists and per-chunk
+// status words in a caller workspace; one row at a time.
 //
-// Per row, a fixed sequence of launches (each kernel returns at once when the
-// device-side state says its step is not needed, so the host never waits):
-//   init     clear the row's counters;
+// Per row, the selection by the band path (one read of the row), else by the
+// multi-pass path where the band path gave up, then the write (one more read).
+// Every kernel returns at once when the device-side state says its step is not
+// needed, so the host never waits.
+//
+// Band path:
+//   w_sample  65536 entries spread over the row give a band of keys
+//             [t_lo, t_hi) that holds the k-th largest magnitude unless the
+//             sample is 4 standard deviations off (as in topk_band.cuh);
+//   w_pass1   one read of the row by persistent CTAs, 8192-entry chunks staged
+//             by double-buffered bulk copies: entries >= t_hi ("sure")
+//             counted; band entries listed in the workspace (a region per CTA)
+//             and counted in a 256-bin histogram of their keys (error feedback:
+//             s = x + err written back into err, which the write reads);
+//   w_pick1   the histogram bin holding the k-th entry (or: the band missed,
+//             and the multi-pass path takes over);
+//   w_bin2    the band entries in that bin, listed;
+//   w_select2 T and `need` among them by integer rounds.
+//
+// Multi-pass path:
+//   init     clear the row's state;
 //   sample   bin scale from a strided sample of the ranked values;
 //   hist     histogram of all entries over bins linear in |x| (error feedback:
-//            s = x + err is written back into err, so later passes read s);
+//            s = x + err is written back into err unless the band path did);
 //   pick     the bin that holds the k-th largest entry, as a key range;
 //   3 x (hist, pick)  refinement rounds with 2048 bins of equal key width over
 //            that range, while it holds more candidates than the list takes;
-//   count    per 8192-entry chunk: entries above the range (or, once T is
-//            known, above / equal to T); entries inside the range are appended
-//            to the candidate list;
-//   select   T and `need` from the candidate list; candidates above / equal to
-//            T join their chunks' counts;
-//   scan     per chunk: kept entries and ties before it;
-//   write    the payload in ascending index order, and the buffer updates.
+//   count    the entries inside the range appended to the candidate list;
+//   select   T and `need` from the candidate list.
+//
+//   (band path) w_mark: band entries above / equal to T join the counts of
+//   their 4096-entry write chunks (pass 1 counted the sure entries there);
+//   (multi-pass) count also counts, per write chunk, the entries above the
+//   range or, once T is known, above / equal to it; select adds the candidates.
+//
+// Write (both paths): w_scan1 / w_scan2, the prefix sums of the per-chunk
+// counts; g_write3, persistent CTAs over 4096-entry chunks, double-buffered:
+// the payload in ascending index order and the buffer updates.
 #include "common.cuh"
 #include "kernels.h"
+#include "launch_util.h"
 #include "select.cuh"
 
 namespace mpc {
@@ -33,6 +56,15 @@ constexpr int kGNB = 2048;               // histogram bins
 constexpr uint32_t kCandCap = 65536;     // candidate list capacity
 constexpr int kSamples = 4096;
 constexpr int kMaxRounds = 3;            // refinement rounds (11 bits each) reach one key
+constexpr int kWSamples = 65536;         // band path: sample entries
+constexpr int kWSBins = 4096;            // band path: sample bins (1/128 octave)
+constexpr int kWSShift = 16;             // band path: sample bin = (key - base) >> 16
+constexpr int kFBins = 256;              // band path: bins of the band histogram
+constexpr uint32_t kCand2Cap = 1u << 21;  // band path: entries of the chosen bin
+constexpr float kWZ = 4.0f;              // band half-width in standard deviations
+constexpr int kWT = 128;                 // write kernel: threads
+constexpr int64_t kWCH = 32 * kWT;       // write kernel: entries of a chunk (4096)
+constexpr uint32_t kWNoSure = 0x7f800001u;  // a t_hi no magnitude reaches (NaN bits)
 
 struct GridMeta {
   float scale;      // |x| bins: nb / sample max (0: integer bins from the start)
@@ -46,40 +78,89 @@ struct GridMeta {
   uint32_t need;
   uint32_t ncand;   // candidates appended by count
   uint32_t nchunks;
+  // band path
+  int band;         // 1 while the band path is on
+  int s_in_aux;     // error feedback: s = x + err has been written into err
+  int counted;      // per-chunk counts are in place (the multi-pass count is skipped)
+  int bin2;         // the chosen band bin needs w_bin2 / w_select2
+  uint32_t t_lo, t_hi;
+  int fsh;          // band histogram: bin = min((key - t_lo) >> fsh, 255)
+  uint32_t sure;    // entries with key >= t_hi
+  uint32_t nband;   // band entries listed (may exceed the capacity: then the path gives up)
+  int b_lo, b_hi;   // the chosen band bin's keys
+  uint32_t b_kr;    // rank of T within it
+  uint32_t ncand2;
 };
 
 struct WsLayout {
   GridMeta* meta;
   uint32_t* hist;   // kGNB
-  uint32_t* cgt;    // nchunks: entries above (later: kept entries before the chunk)
-  uint32_t* ceq;    // nchunks: entries equal to T (later: ties before the chunk)
+  uint32_t* cgt;    // per write chunk (kWCH entries): entries above T; after the scan,
+                    // those of the earlier chunks of its block of 1024 chunks
+  uint32_t* ceq;    // the same for entries equal to T
+  uint32_t* tg;     // per block of 1024 write chunks: entries above T before it
+  uint32_t* te;     // and entries equal to T before it
   int* ckey;        // kCandCap candidate keys
   int64_t* cidx;    // kCandCap candidate positions
+  uint32_t* fhist;  // kFBins: band histogram
+  int* bkey;        // band list: keys
+  uint32_t* bidx;   //            positions in the row
+  int* c2key;       // kCand2Cap: keys of the chosen band bin
+  uint32_t* nbc;    // kMaxBandCtas: band entries listed by each CTA of w_pass1
+  uint32_t bcap;    // band list capacity (G regions of bcap / G entries, G the pass-1 grid)
 };
+
+// CTAs of the persistent band-path kernels at most (each lists its band
+// entries in a region of its own, the band list split evenly among them).
+constexpr int kMaxBandCtas = 4096;
+
+// Band list capacity: a sixteenth of the row and 64K entries (the band of a
+// 16384-entry sample at 4 standard deviations is a few percent of the row).
+uint32_t band_cap(int64_t L) { return static_cast<uint32_t>(L / 16 + 65536); }
 
 size_t align256(size_t b) { return (b + 255) / 256 * 256; }
 
-WsLayout layout(void* ws, int64_t nchunks) {
+WsLayout layout(void* ws, int64_t L, int64_t nchunks) {
   WsLayout w;
   char* p = static_cast<char*>(ws);
   w.meta = reinterpret_cast<GridMeta*>(p);
   p += align256(sizeof(GridMeta));
   w.hist = reinterpret_cast<uint32_t*>(p);
   p += align256(kGNB * 4);
+  const int64_t nwch = (L + kWCH - 1) / kWCH;
   w.cgt = reinterpret_cast<uint32_t*>(p);
-  p += align256(nchunks * 4);
+  p += align256(static_cast<size_t>(nwch) * 4);
   w.ceq = reinterpret_cast<uint32_t*>(p);
-  p += align256(nchunks * 4);
+  p += align256(static_cast<size_t>(nwch) * 4);
+  w.tg = reinterpret_cast<uint32_t*>(p);
+  p += align256(static_cast<size_t>((nwch + 1023) / 1024) * 4);
+  w.te = reinterpret_cast<uint32_t*>(p);
+  p += align256(static_cast<size_t>((nwch + 1023) / 1024) * 4);
   w.cidx = reinterpret_cast<int64_t*>(p);
   p += align256(kCandCap * 8);
   w.ckey = reinterpret_cast<int*>(p);
+  p += align256(kCandCap * 4);
+  w.fhist = reinterpret_cast<uint32_t*>(p);
+  p += align256(kFBins * 4);
+  w.c2key = reinterpret_cast<int*>(p);
+  p += align256(static_cast<size_t>(kCand2Cap) * 4);
+  w.nbc = reinterpret_cast<uint32_t*>(p);
+  p += align256(kMaxBandCtas * 4);
+  w.bcap = band_cap(L);
+  w.bkey = reinterpret_cast<int*>(p);
+  p += align256(static_cast<size_t>(w.bcap) * 4);
+  w.bidx = reinterpret_cast<uint32_t*>(p);
   return w;
 }
 
 size_t ws_bytes_for(int64_t L) {
   const int64_t nchunks = (L + kCH - 1) / kCH;
-  return align256(sizeof(GridMeta)) + align256(kGNB * 4) + 2 * align256(nchunks * 4) +
-         align256(kCandCap * 8) + align256(kCandCap * 4);
+  return align256(sizeof(GridMeta)) + align256(kGNB * 4) +
+         2 * align256(static_cast<size_t>((L + kWCH - 1) / kWCH) * 4) +
+         2 * align256(static_cast<size_t>(((L + kWCH - 1) / kWCH + 1023) / 1024) * 4) +
+         align256(kCandCap * 8) + align256(kCandCap * 4) + align256(kFBins * 4) +
+         align256(static_cast<size_t>(kCand2Cap) * 4) + align256(kMaxBandCtas * 4) +
+         2 * align256(static_cast<size_t>(band_cap(L)) * 4);
 }
 
 template <int MODE>
@@ -162,27 +243,32 @@ __global__ void __launch_bounds__(kGT) g_hist(const float* xr, float* ar, int64_
   __shared__ uint32_t sh[kGNB];
   const GridMeta m = *meta;
   const bool bins = !m.resolved && m.m > kCandCap;
-  const bool write_s = first && MODE == kEF;  // s = x + err goes back into err once
+  // s = x + err goes back into err once (unless the band path already did)
+  const bool write_s = first && MODE == kEF && !m.s_in_aux;
   if (!bins && !write_s) return;
   for (int i = threadIdx.x; i < kGNB; i += kGT) sh[i] = 0;
   __syncthreads();
-  const int64_t c0 = static_cast<int64_t>(blockIdx.x) * kCH;
-  for (int j = 0; j < kGPT; ++j) {
-    const int64_t e = c0 + j * kGT + threadIdx.x;
-    if (e >= L) break;
-    float v;
-    if (write_s) {
-      v = fadd(xr[e], ar[e]);
-      ar[e] = v;
-    } else {
-      v = value_at<MODE>(xr, ar, e);
-    }
-    if (!bins) continue;
-    const int key = mag_key(v);
-    if (m.round == 0) {
-      atomicAdd(&sh[bucket_of(key, m.scale, kGNB)], 1u);
-    } else if (key >= m.lo && key <= m.hi) {
-      atomicAdd(&sh[static_cast<uint32_t>(key - m.lo) >> m.sft], 1u);
+  // chunks c, c + gridDim.x, ... (a fixed grid, so that a launch with nothing to
+  // do costs little)
+  for (int64_t c0 = static_cast<int64_t>(blockIdx.x) * kCH; c0 < L;
+       c0 += static_cast<int64_t>(gridDim.x) * kCH) {
+    for (int j = 0; j < kGPT; ++j) {
+      const int64_t e = c0 + j * kGT + threadIdx.x;
+      if (e >= L) break;
+      float v;
+      if (write_s) {
+        v = fadd(xr[e], ar[e]);
+        ar[e] = v;
+      } else {
+        v = value_at<MODE>(xr, ar, e);
+      }
+      if (!bins) continue;
+      const int key = mag_key(v);
+      if (m.round == 0) {
+        atomicAdd(&sh[bucket_of(key, m.scale, kGNB)], 1u);
+      } else if (key >= m.lo && key <= m.hi) {
+        atomicAdd(&sh[static_cast<uint32_t>(key - m.lo) >> m.sft], 1u);
+      }
     }
   }
   __syncthreads();
@@ -272,8 +358,9 @@ __global__ void __launch_bounds__(kGT) g_pick(GridMeta* meta, uint32_t* hist) {
   for (int i = tid; i < kGNB; i += kGT) hist[i] = 0;  // ready for the next round
 }
 
-// Per chunk: entries above (and equal to) T once it is known; otherwise the
-// entries above [lo, hi], with the entries inside appended to the list.
+// Per write chunk (kWCH entries): once T is known, the entries above and equal
+// to it; otherwise the entries above [lo, hi], with the entries inside appended
+// to the candidate list.  A fixed grid strides over the chunks.
 template <int MODE>
 __global__ void __launch_bounds__(kGT) g_count(const float* xr, const float* ar, int64_t L,
                                                GridMeta* meta, uint32_t* cgt, uint32_t* ceq,
@@ -281,31 +368,34 @@ __global__ void __launch_bounds__(kGT) g_count(const float* xr, const float* ar,
   pdl_begin();
   __shared__ uint32_t red[kGT / 32];
   const GridMeta m = *meta;
-  const int64_t c0 = static_cast<int64_t>(blockIdx.x) * kCH;
-  uint32_t g = 0, q = 0;
-  for (int j = 0; j < kGPT; ++j) {
-    const int64_t e = c0 + j * kGT + threadIdx.x;
-    if (e >= L) break;
-    const int key = mag_key(value_at<MODE>(xr, ar, e));
-    if (m.resolved) {
-      g += key > m.T;
-      q += key == m.T;
-    } else {
-      g += key > m.hi;
-      if (key >= m.lo && key <= m.hi) {
-        const uint32_t at = atomicAdd(&meta->ncand, 1u);
-        if (at < kCandCap) {
-          ckey[at] = key;
-          cidx[at] = e;
+  if (m.counted) return;  // the band path has the counts
+  for (int64_t c = blockIdx.x; c * kWCH < L; c += gridDim.x) {
+    const int64_t c0 = c * kWCH;
+    uint32_t g = 0, q = 0;
+    for (int j = 0; j < kWCH / kGT; ++j) {
+      const int64_t e = c0 + j * kGT + threadIdx.x;
+      if (e >= L) break;
+      const int key = mag_key(value_at<MODE>(xr, ar, e));
+      if (m.resolved) {
+        g += key > m.T;
+        q += key == m.T;
+      } else {
+        g += key > m.hi;
+        if (key >= m.lo && key <= m.hi) {
+          const uint32_t at = atomicAdd(&meta->ncand, 1u);
+          if (at < kCandCap) {
+            ckey[at] = key;
+            cidx[at] = e;
+          }
         }
       }
     }
-  }
-  g = block_sum(g, red);
-  q = block_sum(q, red);
-  if (threadIdx.x == 0) {
-    cgt[blockIdx.x] = g;
-    ceq[blockIdx.x] = q;
+    g = block_sum(g, red);
+    q = block_sum(q, red);
+    if (threadIdx.x == 0) {
+      cgt[c] = g;
+      ceq[c] = q;
+    }
   }
 }
 
@@ -371,7 +461,7 @@ __global__ void __launch_bounds__(1024) g_select(GridMeta* meta, uint32_t* cgt, 
   const int T = s_T;
   for (uint32_t i = tid; i < n; i += 1024) {
     const int key = ckey[i];
-    const int64_t ch = cidx[i] / kCH;
+    const int64_t ch = cidx[i] / kWCH;
     if (key > T) atomicAdd(&cgt[ch], 1u);
     else if (key == T) atomicAdd(&ceq[ch], 1u);
   }
@@ -398,114 +488,693 @@ __device__ __forceinline__ uint32_t excl_scan_1024(uint32_t v, uint32_t* red, ui
   return before + inc - v;
 }
 
-// Per chunk: kept entries before it and ties (entries equal to T) before it,
-// written in place of the chunk's counts.
-__global__ void __launch_bounds__(1024) g_scan(const GridMeta* meta, uint32_t* cgt, uint32_t* ceq,
-                                               int64_t nchunks) {
+// ===========================================================================
+// Band path
+// ===========================================================================
+
+// The band from a sample of the row (one CTA): 65536 entries spread evenly
+// over the row, binned by magnitude key (4096 bins of 1/128 octave below the
+// largest finite sample magnitude); the band reaches 4 standard deviations of
+// the sample count on either side of the k-th entry.
+template <int MODE>
+__global__ void __launch_bounds__(1024) w_sample(const float* xr, const float* ar, int64_t L,
+                                                 int64_t k, GridMeta* meta, uint32_t* fhist) {
   pdl_begin();
+  constexpr int G = kWSBins / 1024;  // bins per thread
+  __shared__ uint32_t hist[kWSBins];
   __shared__ uint32_t red[32];
-  const uint32_t need = meta->need;
-  uint32_t carry_g = 0, carry_e = 0;  // identical in every thread
-  for (int64_t base = 0; base < nchunks; base += 1024) {
-    const int64_t c = base + threadIdx.x;
-    const uint32_t g = c < nchunks ? cgt[c] : 0u;
-    const uint32_t e = c < nchunks ? ceq[c] : 0u;
-    uint32_t te, tk;
-    const uint32_t eb = carry_e + excl_scan_1024(e, red, &te);
-    const uint32_t kept = g + (eb >= need ? 0u : min(e, need - eb));
-    const uint32_t kb = carry_g + excl_scan_1024(kept, red, &tk);
-    if (c < nchunks) {
-      cgt[c] = kb;
-      ceq[c] = eb;
+  __shared__ int pick[2];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  if (meta->resolved) return;  // every entry is kept
+  for (int i = tid; i < kWSBins; i += 1024) hist[i] = 0;
+  for (int i = tid; i < kFBins; i += 1024) fhist[i] = 0;
+  if (tid < 2) pick[tid] = -1;
+  constexpr int PER = kWSamples / 1024;
+  int key[PER];
+  int mx = -1;
+#pragma unroll 16
+  for (int j = 0; j < PER; ++j) {
+    const int64_t e = (static_cast<int64_t>(j) * 1024 + tid) * L / kWSamples;
+    key[j] = mag_key(ranked<MODE>(xr[e], MODE != kPlain ? ar[e] : 0.0f));
+    mx = max(mx, finite_key(key[j]));
+  }
+  mx = __reduce_max_sync(kFull, mx);
+  if (lane == 0) red[warp] = static_cast<uint32_t>(mx);
+  __syncthreads();
+  int smax = -1;
+  for (int w = 0; w < 32; ++w) smax = max(smax, static_cast<int>(red[w]));
+  if (smax <= 0) return;  // no finite non-zero magnitude in the sample: multi-pass path
+  const int base = max(0, smax - ((kWSBins - 1) << kWSShift));
+#pragma unroll 16
+  for (int j = 0; j < PER; ++j)
+    atomicAdd(&hist[min(max(key[j] - base, 0) >> kWSShift, kWSBins - 1)], 1u);
+  __syncthreads();
+  // the bins holding the r_hi-th and the r_lo-th largest sample keys
+  const float mu = __fdividef(static_cast<float>(k) * static_cast<float>(kWSamples),
+                              static_cast<float>(L));
+  const float sd = mu * rsqrtf(mu);
+  const int r_hi = static_cast<int>(floorf(mu - kWZ * sd));
+  const int r_lo = static_cast<int>(ceilf(mu + kWZ * sd)) + 1;
+  uint32_t c[G], tsum = 0;
+#pragma unroll
+  for (int g = 0; g < G; ++g) {
+    c[g] = hist[kWSBins - 1 - (tid * G + g)];
+    tsum += c[g];
+  }
+  uint32_t total;
+  const uint32_t excl = excl_scan_1024(tsum, red, &total);
+  const int rs[2] = {r_hi, r_lo};
+#pragma unroll
+  for (int q = 0; q < 2; ++q) {
+    const int r = rs[q];
+    if (r >= 1 && r <= kWSamples && excl < static_cast<uint32_t>(r) &&
+        static_cast<uint32_t>(r) <= excl + tsum) {
+      uint32_t run = excl;
+#pragma unroll
+      for (int g = 0; g < G; ++g) {
+        if (run + c[g] >= static_cast<uint32_t>(r)) {
+          pick[q] = kWSBins - 1 - (tid * G + g);
+          break;
+        }
+        run += c[g];
+      }
     }
-    carry_g += tk;
-    carry_e += te;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    uint32_t t_lo = 0, t_hi = kWNoSure;
+    if (pick[0] >= 0 && pick[0] < kWSBins - 1)
+      t_hi = static_cast<uint32_t>(base + ((pick[0] + 1) << kWSShift));
+    if (pick[1] > 0) t_lo = static_cast<uint32_t>(base + (pick[1] << kWSShift));
+    if (t_lo > t_hi) t_lo = t_hi;
+    // the band histogram spans [t_lo, t_hi), or, with nothing sure, up to one
+    // octave above the sample's largest magnitude (larger keys share the top bin)
+    const uint32_t fhi = t_hi != kWNoSure ? t_hi - 1u
+                                          : min(static_cast<uint32_t>(smax) + (1u << 23), 0x7f7fffffu);
+    meta->t_lo = t_lo;
+    meta->t_hi = t_hi;
+    meta->fsh = max(0, 24 - __clz(max(fhi, t_lo) - t_lo));  // (key - t_lo) >> fsh < 256
+    meta->sure = 0;
+    meta->nband = 0;
+    meta->ncand2 = 0;
+    meta->bin2 = 0;
+    meta->band = 1;
   }
 }
 
-// Payload of one chunk in ascending index order, and the buffer updates.
+// The chunk loader of the persistent band-path kernels: chunk c's entries of
+// src into buf by bulk copies, part w (1024 entries) completing on bars[w];
+// issued by the first NW lanes of warp 0.  fence.proxy.async first: the buffer
+// was last written by generic stores two chunks before.
+template <int NW, int64_t CH>
+__device__ __forceinline__ void issue_chunk(float* buf, const float* src, const float* pre,
+                                            int64_t L, int64_t c, uint64_t* bars, int lane) {
+  const int64_t c0 = c * CH;
+  const int n = static_cast<int>(min64(CH, L - c0));
+  const int p0 = 1024 * lane;
+  if (lane >= NW || p0 >= n) return;
+  const uint32_t bytes = static_cast<uint32_t>(min(1024, n - p0)) * 4u;
+  fence_proxy_async_smem();
+  if (pre != nullptr) bulk_prefetch_l2(pre + c0 + p0, bytes);
+  mbar_arrive_expect_tx(&bars[lane], bytes);
+  bulk_g2s(buf + p0, src + c0 + p0, bytes, &bars[lane]);
+}
+
+// One read of the row.  Persistent CTAs take chunks c, c + G, ... (G = the grid),
+// double-buffered: the next chunk's bulk copies are in flight while this one
+// is classified.  Thread t owns the 32 consecutive entries [32t, 32t + 32) of a
+// chunk (within its warp's part, so that a warp needs no other warp's data):
+// per entry |x| >= t_hi ("sure") and |x| >= t_lo as bit words.  The sure
+// entries of each write chunk (half a chunk here) go to cgt; the band entries
+// go to this CTA's region of the band list (rcap entries), in index order
+// within each warp's run, and into the CTA's histogram of band keys, added to
+// the row's once at the end.
 template <int MODE>
-__global__ void __launch_bounds__(kGT) g_write(const float* xr, float* ar, int64_t L, int64_t k,
-                                               const GridMeta* meta, const uint32_t* cgt,
-                                               const uint32_t* ceq, float* vals, int32_t* idx) {
+__global__ void __launch_bounds__(kGT) w_pass1(const float* xr, float* ar, int64_t L,
+                                               int64_t nchunks, int aligned, GridMeta* meta,
+                                               uint32_t* cgt, uint32_t* ceq, int* bkey,
+                                               uint32_t* bidx, uint32_t rcap, uint32_t* nbc,
+                                               uint32_t* fhist, uint32_t spin_limit,
+                                               unsigned* status) {
   pdl_begin();
   constexpr int NW = kGT / 32;
-  __shared__ uint32_t ug[kGPT * NW], ue[kGPT * NW];
+  extern __shared__ __align__(16) float wbuf[];  // 2 x kCH
+  __shared__ uint32_t fh[kFBins];
+  __shared__ uint32_t rs[2][NW];  // sure entries per warp, by buffer
+  __shared__ uint32_t s_count, s_fail;
+  __shared__ uint64_t bars[2][NW];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  if (!meta->band || meta->resolved) return;
+  const uint32_t t_lo = meta->t_lo, t_hi = meta->t_hi;
+  const int fsh = meta->fsh;
+  const float f_lo = __uint_as_float(t_lo), f_hi = __uint_as_float(t_hi);
+  for (int i = tid; i < kFBins; i += kGT) fh[i] = 0;
+  if (tid == 0) {
+    s_count = 0;
+    s_fail = 0;
+  }
+  if (aligned && warp == 0 && lane < NW) {
+    mbar_init(&bars[0][lane], 1);
+    mbar_init(&bars[1][lane], 1);
+    fence_mbar_init();
+  }
+  __syncthreads();
+  const uint32_t rbase = blockIdx.x * rcap;  // this CTA's region of the band list
+  const float* pre = MODE != kPlain ? ar : nullptr;
+  int64_t c = blockIdx.x;
+  if (aligned && warp == 0 && c < nchunks) issue_chunk<NW, kCH>(wbuf, xr, pre, L, c, bars[0], lane);
+  uint32_t par = 0;  // bit b: parity of buffer b's next phase
+  uint32_t sure_w = 0;  // sure entries seen by this warp
+  int64_t prev = -1;
+  int b = 0;
+  // the sure counts of chunk c's two write chunks, from the warps' sums in rs[bb]
+  auto put_sure = [&](int64_t cc, int bb) {
+    constexpr int H = NW / 2;  // warps of a write chunk
+    for (int h = 0; h < 2; ++h) {
+      const int64_t wc = 2 * cc + h;
+      if (wc * kWCH >= L) break;
+      uint32_t s = 0;
+#pragma unroll
+      for (int w = 0; w < H; ++w) s += rs[bb][h * H + w];
+      cgt[wc] = s;
+      ceq[wc] = 0;
+    }
+  };
+  static_assert(kCH == 2 * kWCH, "a pass-1 chunk is two write chunks");
+  for (; c < nchunks; c += gridDim.x, b ^= 1) {
+    const int64_t cn = c + gridDim.x;
+    if (aligned && warp == 0 && cn < nchunks)
+      issue_chunk<NW, kCH>(wbuf + (b ^ 1) * kCH, xr, pre, L, cn, bars[b ^ 1], lane);
+    if (tid == 0 && prev >= 0) put_sure(prev, b ^ 1);
+    const int64_t c0 = c * kCH;
+    const int n = static_cast<int>(min64(kCH, L - c0));
+    float* cb = wbuf + b * kCH;
+    const int pb = 1024 * warp;
+    if (pb < n) {
+      if (aligned) {
+        if (!mbar_wait_bounded(&bars[b][warp], (par >> b) & 1u, spin_limit, status)) {
+          mbar_wait_bounded(&bars[b][warp], (par >> b) & 1u, kDrainPolls, nullptr);
+          s_fail = 1;
+        }
+        if (MODE != kPlain) {
+          const int nq = min(1024, n - pb) / 4;
+          float4* c4 = reinterpret_cast<float4*>(cb + pb);
+          float4* a4 = reinterpret_cast<float4*>(ar + c0 + pb);
+          for (int q = lane; q < nq; q += 32) {
+            const float4 xv = c4[q];
+            const float4 av = a4[q];
+            const float4 sv = make_float4(ranked<MODE>(xv.x, av.x), ranked<MODE>(xv.y, av.y),
+                                          ranked<MODE>(xv.z, av.z), ranked<MODE>(xv.w, av.w));
+            c4[q] = sv;
+            if (MODE == kEF) a4[q] = sv;  // s = x + err into err
+          }
+          fence_proxy_async_smem();  // these stores before the buffer's next bulk copy
+        }
+      } else {
+        for (int e = pb + lane; e < min(pb + 1024, n); e += 32) {
+          const float v = ranked<MODE>(xr[c0 + e], MODE != kPlain ? ar[c0 + e] : 0.0f);
+          cb[e] = v;
+          if (MODE == kEF) ar[c0 + e] = v;
+        }
+      }
+      __syncwarp();
+    }
+    par ^= 1u << b;
+    // classification of this thread's 32 entries
+    const int e0 = 32 * tid;
+    const int nv = max(0, min(32, n - e0));
+    const uint32_t vmask = nv >= 32 ? 0xffffffffu : ((1u << nv) - 1u);
+    uint32_t hw = 0, gw = 0;
+    if (nv > 0) {
+      const float4* my4 = reinterpret_cast<const float4*>(cb + e0);
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const float4 v = my4[(u + lane) & 7];  // 8 consecutive lanes on 8 bank groups
+        or_if_ge(hw, v.x, f_hi, 1u << (4 * u + 0));
+        or_if_ge(hw, v.y, f_hi, 1u << (4 * u + 1));
+        or_if_ge(hw, v.z, f_hi, 1u << (4 * u + 2));
+        or_if_ge(hw, v.w, f_hi, 1u << (4 * u + 3));
+        or_if_ge(gw, v.x, f_lo, 1u << (4 * u + 0));
+        or_if_ge(gw, v.y, f_lo, 1u << (4 * u + 1));
+        or_if_ge(gw, v.z, f_lo, 1u << (4 * u + 2));
+        or_if_ge(gw, v.w, f_lo, 1u << (4 * u + 3));
+      }
+      const uint32_t rot = 4u * static_cast<uint32_t>(lane & 7);
+      hw = __funnelshift_l(hw, hw, rot) & vmask;
+      gw = __funnelshift_l(gw, gw, rot) & vmask;
+    }
+    const uint32_t bw = gw & ~hw;
+    const uint32_t nbw = __popc(bw);
+    const uint32_t bi = warp_inclusive_scan(nbw, lane);
+    const uint32_t wtot = __shfl_sync(kFull, bi, 31);
+    uint32_t wb = 0;
+    if (lane == 0 && wtot) wb = atomicAdd(&s_count, wtot);
+    wb = __shfl_sync(kFull, wb, 0);
+    uint32_t pos = wb + bi - nbw;
+    uint32_t w = bw;
+    while (w) {
+      const int j = __ffs(w) - 1;
+      w &= w - 1;
+      const int e = e0 + j;
+      const int key = mag_key(cb[e]);
+      atomicAdd(&fh[min(static_cast<uint32_t>(key - static_cast<int>(t_lo)) >> fsh, kFBins - 1u)],
+                1u);
+      if (pos < rcap) {
+        bkey[rbase + pos] = key;
+        bidx[rbase + pos] = static_cast<uint32_t>(c0 + e);
+      }
+      ++pos;
+    }
+    const uint32_t ws = __reduce_add_sync(kFull, static_cast<uint32_t>(__popc(hw)));
+    sure_w += ws;
+    if (lane == 0) rs[b][warp] = ws;
+    __syncthreads();  // buffer b free for the chunk after next; rs[b] complete
+    prev = c;
+  }
+  if (lane == 0 && sure_w) atomicAdd(&meta->sure, sure_w);
+  if (tid == 0) {
+    if (prev >= 0) put_sure(prev, b ^ 1);
+    const uint32_t cnt = s_count;
+    nbc[blockIdx.x] = min(cnt, rcap);
+    if (cnt) atomicAdd(&meta->nband, cnt);
+    // a full region, or a timed-out copy: the multi-pass path takes over
+    if (cnt > rcap || s_fail) meta->band = 0;
+    if (MODE == kEF && blockIdx.x == 0) meta->s_in_aux = 1;
+  }
+  for (int i = tid; i < kFBins; i += kGT)
+    if (fh[i]) atomicAdd(&fhist[i], fh[i]);
+}
+
+// The band bin holding the k-th entry, or the band path gives up (one warp).
+__global__ void __launch_bounds__(32) w_pick1(GridMeta* meta, const uint32_t* fhist, int64_t k) {
+  pdl_begin();
+  const GridMeta m = *meta;
+  if (!m.band || m.resolved) return;
+  const int lane = threadIdx.x & 31;
+  if (!(static_cast<int64_t>(m.sure) < k && k <= static_cast<int64_t>(m.sure) + m.nband)) {
+    if (lane == 0) meta->band = 0;  // the multi-pass path takes over
+    return;
+  }
+  const uint32_t kr = static_cast<uint32_t>(k - m.sure);
+  const BinPick p = warp_pick_bin(fhist, kr, lane);
+  if (lane == 0) {
+    const int bl = static_cast<int>(m.t_lo) + (p.bin << m.fsh);
+    // the top bin also takes every larger key
+    const int bh = p.bin == kFBins - 1
+                       ? 0x7fffffff
+                       : static_cast<int>(min(static_cast<uint32_t>(bl) + ((1u << m.fsh) - 1u),
+                                              0x7fffffffu));
+    const uint32_t kr2 = kr - p.above;
+    if (p.count == kr2) {  // the bin is kept whole
+      meta->T = bl - 1;
+      meta->need = 0;
+      meta->counted = 1;
+      meta->resolved = 1;
+    } else {
+      meta->b_lo = bl;
+      meta->b_hi = bh;
+      meta->b_kr = kr2;
+      meta->bin2 = 1;
+    }
+  }
+}
+
+// The band entries of the chosen bin, listed: CTA r reads region r of the band
+// list (four loads in flight a thread; one atomic a warp).
+__global__ void __launch_bounds__(256) w_bin2(GridMeta* meta, const int* bkey, const uint32_t* nbc,
+                                              uint32_t rcap, int* c2key) {
+  pdl_begin();
+  const GridMeta m = *meta;
+  if (!m.band || !m.bin2) return;
+  const int lane = threadIdx.x & 31;
+  const unsigned lt = lanemask_lt();
+  const uint32_t nr = nbc[blockIdx.x];
+  const int* rk = bkey + static_cast<size_t>(blockIdx.x) * rcap;
+  for (uint32_t i0 = (threadIdx.x & ~31u) * 4u; i0 < nr; i0 += 256u * 4u) {
+    int key[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const uint32_t i = i0 + 32u * q + lane;
+      key[q] = i < nr ? rk[i] : -1;
+    }
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const bool in = key[q] >= m.b_lo && key[q] <= m.b_hi;
+      const unsigned bb = __ballot_sync(kFull, in);
+      if (!bb) continue;
+      uint32_t base = 0;
+      if (lane == 0) base = atomicAdd(&meta->ncand2, static_cast<uint32_t>(__popc(bb)));
+      base = __shfl_sync(kFull, base, 0);
+      const uint32_t slot = base + __popc(bb & lt);
+      if (in && slot < kCand2Cap) c2key[slot] = key[q];
+    }
+  }
+}
+
+// T and need among the chosen bin's entries, by integer rounds (one CTA).
+__global__ void __launch_bounds__(1024) w_select2(GridMeta* meta, const int* c2key) {
+  pdl_begin();
+  __shared__ uint32_t hist[kRoundBins];
+  __shared__ int s_lo, s_hi, s_T;
+  __shared__ uint32_t s_kr, s_need, s_done;
+  const GridMeta m = *meta;
+  if (!m.band || !m.bin2) return;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  if (m.ncand2 > kCand2Cap) {
+    if (tid == 0) meta->band = 0;  // too crowded: the multi-pass path takes over
+    return;
+  }
+  const uint32_t n = m.ncand2;
+  if (tid == 0) {
+    s_lo = m.b_lo;
+    s_hi = m.b_hi;
+    s_kr = m.b_kr;
+    s_done = 0;
+  }
+  __syncthreads();
+  while (!s_done) {
+    const int lo = s_lo, hi = s_hi;
+    if (lo >= hi) {
+      if (tid == 0) {
+        s_T = lo;
+        s_need = s_kr;
+        s_done = 1;
+      }
+      __syncthreads();
+      break;
+    }
+    const int sft = round_shift(lo, hi);
+    for (int i = tid; i < kRoundBins; i += 1024) hist[i] = 0;
+    __syncthreads();
+    for (uint32_t i = tid; i < n; i += 1024) {
+      const int key = c2key[i];
+      if (key >= lo && key <= hi) atomicAdd(&hist[static_cast<uint32_t>(key - lo) >> sft], 1u);
+    }
+    __syncthreads();
+    if (warp == 0) {
+      const BinPick p = warp_pick_bin(hist, s_kr, lane);
+      if (lane == 0) {
+        const uint32_t kr = s_kr - p.above;
+        const int nlo = lo + (p.bin << sft);
+        const int nhi = static_cast<int>(
+            min(static_cast<uint32_t>(hi), static_cast<uint32_t>(nlo) + ((1u << sft) - 1u)));
+        s_kr = kr;
+        if (p.count == kr) {
+          s_T = nlo - 1;
+          s_need = 0;
+          s_done = 1;
+        } else {
+          s_lo = nlo;
+          s_hi = nhi;
+        }
+      }
+    }
+    __syncthreads();
+  }
+  if (tid == 0) {
+    meta->T = s_T;
+    meta->need = s_need;
+    meta->counted = 1;
+    meta->resolved = 1;
+  }
+}
+
+// Band entries above T, and equal to it, join their write chunks' counts: CTA r
+// reads region r of the band list; lanes of a warp on the same chunk add once.
+__global__ void __launch_bounds__(256) w_mark(const GridMeta* meta, const int* bkey,
+                                              const uint32_t* bidx, const uint32_t* nbc,
+                                              uint32_t rcap, uint32_t* cgt, uint32_t* ceq) {
+  pdl_begin();
+  const GridMeta m = *meta;
+  if (!m.band || !m.resolved) return;
+  const int lane = threadIdx.x & 31;
+  const uint32_t nr = nbc[blockIdx.x];
+  const size_t rb = static_cast<size_t>(blockIdx.x) * rcap;
+  const int T = m.T;
+  for (uint32_t i0 = (threadIdx.x & ~31u) * 4u; i0 < nr; i0 += 256u * 4u) {
+    int key[4];
+    uint32_t ch[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const uint32_t i = i0 + 32u * q + lane;
+      key[q] = i < nr ? bkey[rb + i] : -1;
+      ch[q] = i < nr ? static_cast<uint32_t>(bidx[rb + i] / kWCH) : 0xffffffffu;
+    }
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const unsigned same = __match_any_sync(kFull, ch[q]);
+      const unsigned bg = __ballot_sync(kFull, key[q] > T) & same;
+      const unsigned be = __ballot_sync(kFull, key[q] == T) & same;
+      if (ch[q] != 0xffffffffu && lane == __ffs(same) - 1) {
+        if (bg) atomicAdd(&cgt[ch[q]], static_cast<uint32_t>(__popc(bg)));
+        if (be) atomicAdd(&ceq[ch[q]], static_cast<uint32_t>(__popc(be)));
+      }
+    }
+  }
+}
+
+// Exclusive prefix sums of the per-write-chunk counts, in two steps: each CTA
+// of w_scan1 scans 1024 chunks' counts in place and writes their totals; w_scan2
+// (one CTA) scans the totals.  The counts before chunk c are then
+// cgt[c] + tg[c / 1024] (and ceq[c] + te[c / 1024]).
+__global__ void __launch_bounds__(1024) w_scan1(uint32_t* cgt, uint32_t* ceq, uint32_t* tg,
+                                                uint32_t* te, int64_t nwch) {
+  pdl_begin();
+  __shared__ uint32_t red[32];
+  const int64_t c = static_cast<int64_t>(blockIdx.x) * 1024 + threadIdx.x;
+  const uint32_t g = c < nwch ? cgt[c] : 0u, q = c < nwch ? ceq[c] : 0u;
+  uint32_t sg, sq;
+  const uint32_t xg = excl_scan_1024(g, red, &sg);
+  const uint32_t xq = excl_scan_1024(q, red, &sq);
+  if (c < nwch) {
+    cgt[c] = xg;
+    ceq[c] = xq;
+  }
+  if (threadIdx.x == 0) {
+    tg[blockIdx.x] = sg;
+    te[blockIdx.x] = sq;
+  }
+}
+
+__global__ void __launch_bounds__(1024) w_scan2(uint32_t* tg, uint32_t* te, int nblocks) {
+  pdl_begin();
+  __shared__ uint32_t red[32];
+  uint32_t carry_g = 0, carry_q = 0;
+  for (int b0 = 0; b0 < nblocks; b0 += 1024) {
+    const int b = b0 + threadIdx.x;
+    const uint32_t g = b < nblocks ? tg[b] : 0u, q = b < nblocks ? te[b] : 0u;
+    uint32_t sg, sq;
+    const uint32_t xg = excl_scan_1024(g, red, &sg);
+    const uint32_t xq = excl_scan_1024(q, red, &sq);
+    if (b < nblocks) {
+      tg[b] = carry_g + xg;
+      te[b] = carry_q + xq;
+    }
+    carry_g += sg;
+    carry_q += sq;
+  }
+}
+
+// w |= bit when a > b, or when a == b (one compare and one predicated OR).
+__device__ __forceinline__ void or_if_gt(uint32_t& w, int a, int b, uint32_t bit) {
+  asm("{\n .reg .pred p;\n setp.gt.s32 p, %1, %2;\n @p or.b32 %0, %0, %3;\n}"
+      : "+r"(w)
+      : "r"(a), "r"(b), "r"(bit));
+}
+__device__ __forceinline__ void or_if_eq(uint32_t& w, int a, int b, uint32_t bit) {
+  asm("{\n .reg .pred p;\n setp.eq.s32 p, %1, %2;\n @p or.b32 %0, %0, %3;\n}"
+      : "+r"(w)
+      : "r"(a), "r"(b), "r"(bit));
+}
+
+// The payload in ascending index order, and the buffer updates, once T and
+// need are known and the scan has the counts before each write chunk: one read
+// of the row (x, s from err for error feedback, or x with d = x - g formed here
+// for EF21).  Persistent CTAs over chunks of kWCH entries, double-buffered.
+// Thread t's 32 entries give its words of entries above T and equal to T; ties
+// are kept in index order while their rank in the row is below need; a block
+// scan gives the positions, the kept columns are staged at them, and the
+// payload leaves with coalesced stores.
+template <int MODE>
+__global__ void __launch_bounds__(kWT) g_write3(const float* xr, float* ar, int64_t L,
+                                                int64_t nwch, int64_t k, int aligned,
+                                                const GridMeta* meta, const uint32_t* cgt,
+                                                const uint32_t* ceq, const uint32_t* tg,
+                                                const uint32_t* te, float* vals, int32_t* idx,
+                                                uint32_t spin_limit, unsigned* status) {
+  pdl_begin();
+  constexpr int NW = kWT / 32;
+  extern __shared__ __align__(16) float wbuf[];  // 2 x kWCH values, then kWCH staged columns
+  uint16_t* cols = reinterpret_cast<uint16_t*>(wbuf + 2 * kWCH);
+  __shared__ uint32_t rg[NW], re[NW];
+  __shared__ uint64_t bars[2][NW];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int T = meta->T;
   const uint32_t need = meta->need;
-  const int64_t c0 = static_cast<int64_t>(blockIdx.x) * kCH;
-  const unsigned lt = lanemask_lt();
-  // units of 32 consecutive entries: unit u = j * NW + warp covers
-  // [c0 + j * kGT + 32 * warp, +32)
-  for (int j = 0; j < kGPT; ++j) {
-    const int64_t e = c0 + j * kGT + tid;
-    int key = -1;
-    if (e < L) key = mag_key(value_at<MODE>(xr, ar, e));
-    const unsigned bg = __ballot_sync(kFull, key > T);
-    const unsigned be = __ballot_sync(kFull, key == T);
-    if (lane == 0) {
-      ug[j * NW + warp] = __popc(bg);
-      ue[j * NW + warp] = __popc(be);
-    }
+  if (aligned && warp == 0 && lane < NW) {
+    mbar_init(&bars[0][lane], 1);
+    mbar_init(&bars[1][lane], 1);
+    fence_mbar_init();
   }
   __syncthreads();
-  if (warp == 0) {  // exclusive scans over the chunk's units
-    constexpr int PER = kGPT * NW / 32;
-    uint32_t g[PER], q[PER], tg = 0, te = 0;
-    for (int i = 0; i < PER; ++i) {
-      g[i] = ug[lane * PER + i];
-      q[i] = ue[lane * PER + i];
-      tg += g[i];
-      te += q[i];
+  // the values ranked: s lives in err for error feedback
+  const float* src = MODE == kEF ? ar : xr;
+  const float* pre = MODE == kDelta ? ar : nullptr;
+  int64_t c = blockIdx.x;
+  if (aligned && warp == 0 && c < nwch) issue_chunk<NW, kWCH>(wbuf, src, pre, L, c, bars[0], lane);
+  uint32_t par = 0;
+  int b = 0;
+  for (; c < nwch; c += gridDim.x, b ^= 1) {
+    const int64_t cn = c + gridDim.x;
+    if (aligned && warp == 0 && cn < nwch)
+      issue_chunk<NW, kWCH>(wbuf + (b ^ 1) * kWCH, src, pre, L, cn, bars[b ^ 1], lane);
+    const int64_t c0 = c * kWCH;
+    const int n = static_cast<int>(min64(kWCH, L - c0));
+    float* cb = wbuf + b * kWCH;
+    const int pb = 1024 * warp;
+    if (pb < n) {
+      if (aligned) {
+        if (!mbar_wait_bounded(&bars[b][warp], (par >> b) & 1u, spin_limit, status))
+          mbar_wait_bounded(&bars[b][warp], (par >> b) & 1u, kDrainPolls, nullptr);
+        if (MODE == kDelta) {
+          const int nq = min(1024, n - pb) / 4;
+          float4* c4 = reinterpret_cast<float4*>(cb + pb);
+          const float4* a4 = reinterpret_cast<const float4*>(ar + c0 + pb);
+          for (int q = lane; q < nq; q += 32) {
+            const float4 xv = c4[q];
+            const float4 av = a4[q];
+            c4[q] = make_float4(fsub(xv.x, av.x), fsub(xv.y, av.y), fsub(xv.z, av.z),
+                                fsub(xv.w, av.w));
+          }
+          fence_proxy_async_smem();  // these stores before the buffer's next bulk copy
+        }
+      } else {
+        for (int e = pb + lane; e < min(pb + 1024, n); e += 32)
+          cb[e] = value_at<MODE>(xr, ar, c0 + e);
+      }
+      __syncwarp();
     }
-    uint32_t xg = warp_inclusive_scan(tg, lane) - tg;
-    uint32_t xe = warp_inclusive_scan(te, lane) - te;
-    for (int i = 0; i < PER; ++i) {
-      ug[lane * PER + i] = xg;
-      ue[lane * PER + i] = xe;
-      xg += g[i];
-      xe += q[i];
+    par ^= 1u << b;
+    // words of this thread's 32 entries: above T, and equal to T
+    const int e0 = 32 * tid;
+    const int nv = max(0, min(32, n - e0));
+    const uint32_t vmask = nv >= 32 ? 0xffffffffu : ((1u << nv) - 1u);
+    uint32_t gw = 0, ew = 0;
+    if (nv > 0) {
+      const float4* my4 = reinterpret_cast<const float4*>(cb + e0);
+      if (need == 0) {
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const float4 v = my4[(u + lane) & 7];  // 8 consecutive lanes on 8 bank groups
+          or_if_gt(gw, mag_key(v.x), T, 1u << (4 * u + 0));
+          or_if_gt(gw, mag_key(v.y), T, 1u << (4 * u + 1));
+          or_if_gt(gw, mag_key(v.z), T, 1u << (4 * u + 2));
+          or_if_gt(gw, mag_key(v.w), T, 1u << (4 * u + 3));
+        }
+      } else {
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const float4 v = my4[(u + lane) & 7];
+          const int k0 = mag_key(v.x), k1 = mag_key(v.y), k2 = mag_key(v.z), k3 = mag_key(v.w);
+          or_if_gt(gw, k0, T, 1u << (4 * u + 0));
+          or_if_gt(gw, k1, T, 1u << (4 * u + 1));
+          or_if_gt(gw, k2, T, 1u << (4 * u + 2));
+          or_if_gt(gw, k3, T, 1u << (4 * u + 3));
+          or_if_eq(ew, k0, T, 1u << (4 * u + 0));
+          or_if_eq(ew, k1, T, 1u << (4 * u + 1));
+          or_if_eq(ew, k2, T, 1u << (4 * u + 2));
+          or_if_eq(ew, k3, T, 1u << (4 * u + 3));
+        }
+      }
+      const uint32_t rot = 4u * static_cast<uint32_t>(lane & 7);
+      gw = __funnelshift_l(gw, gw, rot) & vmask;
+      ew = __funnelshift_l(ew, ew, rot) & vmask;
     }
-  }
-  __syncthreads();
-  const uint32_t kbase = cgt[blockIdx.x], ebase = ceq[blockIdx.x];
-  for (int j = 0; j < kGPT; ++j) {
-    const int64_t e = c0 + j * kGT + tid;
-    float v = 0.0f;
-    int key = -1;
-    if (e < L) {
-      v = value_at<MODE>(xr, ar, e);
-      key = mag_key(v);
+    const uint32_t ng = __popc(gw), ne = __popc(ew);
+    const uint32_t gi = warp_inclusive_scan(ng, lane);
+    const uint32_t ei = warp_inclusive_scan(ne, lane);
+    if (lane == 31) {
+      rg[warp] = gi;
+      re[warp] = ei;
     }
-    const int u = j * NW + warp;
-    const bool eq = key == T;
-    const unsigned be = __ballot_sync(kFull, eq);
-    const uint32_t erank = ebase + ue[u] + __popc(be & lt);
-    const bool kp = key > T || (eq && erank < need);
-    const unsigned bk = __ballot_sync(kFull, kp);
-    if (kp) {
-      // kept before it: the chunk's kept predecessors, entries above T in
-      // earlier units, ties taken in earlier units, kept lanes of this unit
-      const uint64_t pos = static_cast<uint64_t>(kbase) + ug[u] +
-                           min(ebase + ue[u], need) - min(ebase, need) + __popc(bk & lt);
+    __syncthreads();
+    uint32_t gp = gi - ng, ep = ei - ne, G = 0, E = 0;
+#pragma unroll
+    for (int w = 0; w < NW; ++w) {
+      gp += (w < warp) ? rg[w] : 0u;
+      ep += (w < warp) ? re[w] : 0u;
+      G += rg[w];
+      E += re[w];
+    }
+    // entries above T and equal to T before this chunk
+    const uint32_t gb = cgt[c] + tg[c >> 10], eb = ceq[c] + te[c >> 10];
+    // ties kept: those whose rank among the row's ties is below need
+    const uint32_t room = need > eb ? need - eb : 0u;  // ties this chunk may still take
+    uint32_t kw = gw;
+    if (ne && room > ep) {
+      uint32_t take = min(room - ep, ne);
+      uint32_t w = ew;
+      while (take--) {
+        kw |= w & (~w + 1u);
+        w &= w - 1;
+      }
+    }
+    // positions: kept entries before this chunk, then before this thread in it
+    const uint64_t base = static_cast<uint64_t>(gb) + min(eb, need);
+    uint32_t p = gp + min(ep, room);
+    const uint32_t total = G + min(E, room);
+    while (kw) {
+      const int j = __ffs(kw) - 1;
+      kw &= kw - 1;
+      cols[p++] = static_cast<uint16_t>(e0 + j);
+    }
+    __syncthreads();
+    for (uint32_t i = tid; i < total; i += kWT) {
+      const int e = cols[i];
+      const float v = cb[e];
+      const uint64_t pos = base + i;
       if (pos < static_cast<uint64_t>(k)) {
         vals[pos] = v;
-        idx[pos] = static_cast<int32_t>(e);
+        idx[pos] = static_cast<int32_t>(c0 + e);
       }
-      if (MODE == kEF) ar[e] = 0.0f;            // err' = s - C(s): +0 where sent
-      if (MODE == kDelta) ar[e] = fadd(ar[e], v);  // g' = g + d where sent
+      if (MODE == kEF) ar[c0 + e] = 0.0f;                    // err' = s - C(s): +0 where sent
+      if (MODE == kDelta) ar[c0 + e] = fadd(ar[c0 + e], v);  // g' = g + d where sent
     }
+    __syncthreads();  // buffer b, the staged columns and rg / re free again
   }
 }
 
+// Persistent grids: the CTAs that fit on the GPU (and no more than the band
+// list has regions).
+template <class K>
+unsigned persistent_grid(K kernel, int threads, int smem, int num_sms, int64_t nchunks) {
+  const int occ = resident_blocks(kernel, threads, smem);
+  const int64_t g = min64(min64(static_cast<int64_t>(num_sms) * occ, kMaxBandCtas), nchunks);
+  return static_cast<unsigned>(max64(g, 1));
+}
+
 template <int MODE>
-cudaError_t run_grid(const TopkGridArgs& a, cudaStream_t s) {
+cudaError_t run_grid(const TopkGridArgs& a, int num_sms, cudaStream_t s) {
   const int64_t L = a.L;
   const int64_t nchunks = (L + kCH - 1) / kCH;
+  const int64_t nwch = (L + kWCH - 1) / kWCH;
+  const int nblk = static_cast<int>((nwch + 1023) / 1024);
   if (nchunks > 0x7fffffffLL) return cudaErrorInvalidValue;
-  const WsLayout w = layout(a.ws, nchunks);
-  const unsigned grid = static_cast<unsigned>(nchunks);
+  const WsLayout w = layout(a.ws, L, nchunks);
+  auto al16 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; };
+  const int aligned = (L % 4 == 0) && al16(a.x) && (MODE == kPlain || al16(a.aux));
+  constexpr int kP1Smem = 2 * kCH * 4;             // two chunk buffers
+  constexpr int kWSmem = 2 * kWCH * 4 + kWCH * 2;  // two chunk buffers and the staged columns
+  auto p1 = w_pass1<MODE>;
+  auto wr = g_write3<MODE>;
+  cudaError_t err = ensure_dynamic_smem(p1, kP1Smem);
+  if (err == cudaSuccess) err = ensure_dynamic_smem(wr, kWSmem);
+  if (err != cudaSuccess) return err;
+  const unsigned g1 = persistent_grid(p1, kGT, kP1Smem, num_sms, nchunks);
+  const unsigned gw = persistent_grid(wr, kWT, kWSmem, num_sms, nwch);
+  const uint32_t rcap = w.bcap / g1;  // band-list region of one pass-1 CTA
+  // the multi-pass kernels: a fixed grid striding over the chunks
+  const unsigned gm = static_cast<unsigned>(min64(nwch, static_cast<int64_t>(num_sms) * 8));
   for (int64_t r = 0; r < a.rows; ++r) {
     const float* xr = a.x + r * L;
     float* ar = (MODE != kPlain) ? a.aux + r * L : nullptr;
@@ -513,16 +1182,28 @@ cudaError_t run_grid(const TopkGridArgs& a, cudaStream_t s) {
     int32_t* ir = a.idx + r * a.k;
     g_init<<<1, 256, 0, s>>>(w.meta, w.hist, nchunks);
     g_sample<MODE><<<1, kGT, 0, s>>>(xr, ar, L, a.k, w.meta);
-    g_hist<MODE><<<grid, kGT, 0, s>>>(xr, ar, L, w.meta, w.hist, 1);
+    // the band path
+    w_sample<MODE><<<1, 1024, 0, s>>>(xr, ar, L, a.k, w.meta, w.fhist);
+    p1<<<g1, kGT, kP1Smem, s>>>(xr, ar, L, nchunks, aligned, w.meta, w.cgt, w.ceq, w.bkey, w.bidx,
+                                rcap, w.nbc, w.fhist, a.spin_limit, a.status);
+    w_pick1<<<1, 32, 0, s>>>(w.meta, w.fhist, a.k);
+    w_bin2<<<g1, 256, 0, s>>>(w.meta, w.bkey, w.nbc, rcap, w.c2key);
+    w_select2<<<1, 1024, 0, s>>>(w.meta, w.c2key);
+    w_mark<<<g1, 256, 0, s>>>(w.meta, w.bkey, w.bidx, w.nbc, rcap, w.cgt, w.ceq);
+    // the multi-pass path (each kernel returns at once when the band path resolved)
+    g_hist<MODE><<<gm, kGT, 0, s>>>(xr, ar, L, w.meta, w.hist, 1);
     g_pick<<<1, kGT, 0, s>>>(w.meta, w.hist);
     for (int i = 0; i < kMaxRounds; ++i) {
-      g_hist<MODE><<<grid, kGT, 0, s>>>(xr, ar, L, w.meta, w.hist, 0);
+      g_hist<MODE><<<gm, kGT, 0, s>>>(xr, ar, L, w.meta, w.hist, 0);
       g_pick<<<1, kGT, 0, s>>>(w.meta, w.hist);
     }
-    g_count<MODE><<<grid, kGT, 0, s>>>(xr, ar, L, w.meta, w.cgt, w.ceq, w.ckey, w.cidx);
+    g_count<MODE><<<gm, kGT, 0, s>>>(xr, ar, L, w.meta, w.cgt, w.ceq, w.ckey, w.cidx);
     g_select<<<1, 1024, 0, s>>>(w.meta, w.cgt, w.ceq, w.ckey, w.cidx);
-    g_scan<<<1, 1024, 0, s>>>(w.meta, w.cgt, w.ceq, nchunks);
-    g_write<MODE><<<grid, kGT, 0, s>>>(xr, ar, L, a.k, w.meta, w.cgt, w.ceq, vr, ir);
+    // both paths: positions per write chunk, then the payload (the second read)
+    w_scan1<<<nblk, 1024, 0, s>>>(w.cgt, w.ceq, w.tg, w.te, nwch);
+    w_scan2<<<1, 1024, 0, s>>>(w.tg, w.te, nblk);
+    wr<<<gw, kWT, kWSmem, s>>>(xr, ar, L, nwch, a.k, aligned, w.meta, w.cgt, w.ceq, w.tg, w.te,
+                               vr, ir, a.spin_limit, a.status);
     const cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
@@ -538,12 +1219,11 @@ size_t topk_grid_workspace_bytes(int64_t rows, int64_t L, int64_t k) {
 }
 
 cudaError_t launch_topk_grid(int mode, const TopkGridArgs& a, int num_sms, cudaStream_t s) {
-  (void)num_sms;
   if (a.rows <= 0) return cudaSuccess;
   switch (mode) {
-    case kPlain: return run_grid<kPlain>(a, s);
-    case kEF: return run_grid<kEF>(a, s);
-    case kDelta: return run_grid<kDelta>(a, s);
+    case kPlain: return run_grid<kPlain>(a, num_sms, s);
+    case kEF: return run_grid<kEF>(a, num_sms, s);
+    case kDelta: return run_grid<kDelta>(a, num_sms, s);
     default: return cudaErrorInvalidValue;
   }
 }

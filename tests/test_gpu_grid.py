@@ -133,3 +133,37 @@ def test_workspace_too_small_is_rejected(mpc):
     with pytest.raises(mpc.MpcError) as e:
         mpc.mpc_topk_compress(x, 10, ws=ws)
     assert e.value.status == 3
+
+
+@pytest.mark.parametrize("L", [131072, 1000003])
+def test_sample_misled(mpc, L):
+    """A row whose sampled positions (16384 evenly spread) hold much larger magnitudes
+    than the rest: the sampled band misses the k-th entry after the first read, and the
+    multi-pass path finishes the selection (error feedback: with s already written into
+    err).  Plain, EF and EF21, against the oracle."""
+    rng = np.random.default_rng(L)
+    R = 1
+    x = (rng.standard_normal((R, L)) * 1e-3).astype(np.float32)
+    pos = (np.arange(16384, dtype=np.int64) * L) // 16384
+    x[0, pos] = (1.0 + rng.random(16384)).astype(np.float32)
+    k = L // 4  # far more than the sampled entries: the threshold is among the small ones
+    v, i = mpc.mpc_topk_compress(dev(x), k)
+    ok(mpc)
+    ov, oi = oracle.topk_compress(x, k)
+    assert_bits_equal(i.cpu().numpy(), oi, "idx")
+    assert_bits_equal(v.cpu().numpy(), ov, "vals")
+    e_host = (rng.standard_normal((R, L)) * 1e-4).astype(np.float32)
+    e_dev = dev(e_host.copy())
+    v, i = mpc.mpc_ef_topk_compress(dev(x), e_dev, k)
+    ok(mpc)
+    ov, oi = oracle.ef_topk_compress(x, e_host, k)
+    assert_bits_equal(i.cpu().numpy(), oi, "EF idx")
+    assert_bits_equal(v.cpu().numpy(), ov, "EF vals")
+    assert_bits_equal(e_dev.cpu().numpy(), e_host, "EF err")
+    g_host = (rng.standard_normal((R, L)) * 1e-4).astype(np.float32)
+    g_dev = dev(g_host.copy())
+    v, i = mpc.mpc_ef21_topk_compress(dev(x), g_dev, k)
+    ok(mpc)
+    ov, oi = oracle.ef21_topk_compress(x, g_host, k)
+    assert_bits_equal(i.cpu().numpy(), oi, "EF21 idx")
+    assert_bits_equal(g_dev.cpu().numpy(), g_host, "EF21 g")

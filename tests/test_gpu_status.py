@@ -83,3 +83,4 @@ def test_results_do_not_depend_on_dependent_launch(mpc):
         assert np.array_equal(p.view(np.uint32) if p.dtype.itemsize == 4 else p,
                               q.view(np.uint32) if q.dtype.itemsize == 4 else q)
     assert mpc.mpc_get_status() == 0
+
