@@ -347,6 +347,7 @@ __global__ void __launch_bounds__(NT) quant_cta_kernel(const QuantArgs a, int sp
   if (!failed) {
 #pragma unroll
     for (int v = 0; v < kQNV; ++v) {
+      if (v >= jmax) break;  // the slice's chunks only (shared memory holds no more)
       const int q = v * NT + tid;
       const int64_t e0 = 4 * q;  // slice-relative
       const float4 f = reinterpret_cast<const float4*>(sx)[q];
@@ -378,26 +379,71 @@ __global__ void __launch_bounds__(NT) quant_cta_kernel(const QuantArgs a, int sp
 }
 
 // Long rows, first pass: per-row min/max keys into the workspace (which the
-// launcher initialises to {0xffffffff, 0}).
-__global__ void __launch_bounds__(kQNT) quant_minmax_kernel(const float* x, int64_t L, int spr,
-                                                            int64_t slice, uint32_t* mm) {
+// launcher initialises to {0xffffffff, 0}).  A fixed grid strides over the
+// rows' slices (slice s of row s / spr); each CTA keeps the extrema of the
+// current row in registers and adds them to the workspace when its row
+// changes, so that the workspace sees few atomics even for one huge row.
+__global__ void __launch_bounds__(kQNT) quant_minmax_kernel(const float* x, int64_t L, int64_t rows,
+                                                            int spr, int64_t slice, int aligned,
+                                                            uint32_t* mm) {
   pdl_begin();
-  const int64_t row = blockIdx.x / spr;
-  const int64_t c0 = (blockIdx.x % spr) * slice;
-  const int64_t n = max64(0, min64(slice, L - c0));
-  const float* xr = x + row * L + c0;
+  __shared__ uint32_t rmin[kQNT / 32], rmax[kQNT / 32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int64_t total = rows * spr;
+  int64_t cur = -1;
   uint32_t kmin = 0xffffffffu, kmax = 0u;
-  for (int64_t e = threadIdx.x; e < n; e += kQNT) {
-    const uint32_t ok = ord_key(xr[e]);
-    kmin = min(kmin, ok);
-    kmax = max(kmax, ok);
+  auto flush = [&]() {
+    uint32_t a = __reduce_min_sync(kFull, kmin), b = __reduce_max_sync(kFull, kmax);
+    if (lane == 0) {
+      rmin[warp] = a;
+      rmax[warp] = b;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0 && cur >= 0) {
+      for (int w = 0; w < kQNT / 32; ++w) {
+        a = min(a, rmin[w]);
+        b = max(b, rmax[w]);
+      }
+      atomicMin(mm + 2 * cur, a);
+      atomicMax(mm + 2 * cur + 1, b);
+    }
+    __syncthreads();
+    kmin = 0xffffffffu;
+    kmax = 0u;
+  };
+  for (int64_t s = blockIdx.x; s < total; s += gridDim.x) {
+    const int64_t row = s / spr;
+    if (row != cur) {  // uniform: every thread sees the same s
+      if (cur >= 0) flush();
+      cur = row;
+    }
+    const int64_t c0 = (s % spr) * slice;
+    const int64_t n = max64(0, min64(slice, L - c0));
+    const float* xr = x + row * L + c0;
+    if (aligned) {
+      const float4* x4 = reinterpret_cast<const float4*>(xr);
+      const int64_t n4 = n / 4;
+#pragma unroll 4
+      for (int64_t q = threadIdx.x; q < n4; q += kQNT) {
+        const float4 f = x4[q];
+        const uint32_t a0 = ord_key(f.x), a1 = ord_key(f.y), a2 = ord_key(f.z), a3 = ord_key(f.w);
+        kmin = min(kmin, min(min(a0, a1), min(a2, a3)));
+        kmax = max(kmax, max(max(a0, a1), max(a2, a3)));
+      }
+      for (int64_t e = 4 * n4 + threadIdx.x; e < n; e += kQNT) {
+        const uint32_t ok = ord_key(xr[e]);
+        kmin = min(kmin, ok);
+        kmax = max(kmax, ok);
+      }
+    } else {
+      for (int64_t e = threadIdx.x; e < n; e += kQNT) {
+        const uint32_t ok = ord_key(xr[e]);
+        kmin = min(kmin, ok);
+        kmax = max(kmax, ok);
+      }
+    }
   }
-  kmin = __reduce_min_sync(kFull, kmin);
-  kmax = __reduce_max_sync(kFull, kmax);
-  if ((threadIdx.x & 31) == 0) {
-    atomicMin(mm + 2 * row, kmin);
-    atomicMax(mm + 2 * row + 1, kmax);
-  }
+  flush();
 }
 
 __global__ void minmax_init_kernel(uint32_t* mm, int64_t rows) {
@@ -674,8 +720,7 @@ cudaError_t run_quant_bits(const QuantArgs& a0, int num_sms, cudaStream_t s) {
       a.rows <= num_sms)
     return run_quant_wide<BITS, SR, 4 * kQNT>(a, s);
   auto kernel = quant_cta_kernel<BITS, SR, kQNT>;
-  const int smem = kQSCAP * 4;
-  cudaError_t err = ensure_dynamic_smem(kernel, smem);
+  cudaError_t err = ensure_dynamic_smem(kernel, kQSCAP * 4);
   if (err != cudaSuccess) return err;
   int64_t spr;
   if (a.ws == nullptr) {
@@ -689,12 +734,18 @@ cudaError_t run_quant_bits(const QuantArgs& a0, int num_sms, cudaStream_t s) {
     if (a.rows > 0x7fffffffLL / spr) return cudaErrorInvalidValue;  // before any launch
     uint32_t* mm = static_cast<uint32_t*>(a.ws);
     minmax_init_kernel<<<static_cast<unsigned>(min64((a.rows + 255) / 256, 1024)), 256, 0, s>>>(mm, a.rows);
-    quant_minmax_kernel<<<static_cast<unsigned>(a.rows * spr), kQNT, 0, s>>>(a.x, L, static_cast<int>(spr), a.slice, mm);
+    const int occ = resident_blocks(quant_minmax_kernel, kQNT, 0);
+    const int64_t mgrid = min64(a.rows * spr, static_cast<int64_t>(num_sms) * occ);
+    quant_minmax_kernel<<<static_cast<unsigned>(mgrid), kQNT, 0, s>>>(
+        a.x, L, a.rows, static_cast<int>(spr), a.slice, a.aligned, mm);
     err = cudaGetLastError();
     if (err != cudaSuccess) return err;
   }
   const int64_t blocks = a.rows * spr;
   if (blocks > 0x7fffffffLL) return cudaErrorInvalidValue;
+  // shared memory for the slice's chunks only (4 x kQNT entries each), so that
+  // short slices leave room for more CTAs per SM
+  const int smem = static_cast<int>((a.slice + 4 * kQNT - 1) / (4 * kQNT)) * 4 * kQNT * 4;
   return launch_kernel(kernel, dim3(static_cast<unsigned>(blocks)), dim3(kQNT), smem, s,
                        (a.ws == nullptr) ? static_cast<unsigned>(spr) : 1u, a,
                        static_cast<int>(spr));

@@ -1129,16 +1129,30 @@ __global__ void __launch_bounds__(kWT) g_write3(const float* xr, float* ar, int6
       cols[p++] = static_cast<uint16_t>(e0 + j);
     }
     __syncthreads();
-    for (uint32_t i = tid; i < total; i += kWT) {
-      const int e = cols[i];
-      const float v = cb[e];
-      const uint64_t pos = base + i;
-      if (pos < static_cast<uint64_t>(k)) {
-        vals[pos] = v;
-        idx[pos] = static_cast<int32_t>(c0 + e);
+    // four kept entries a thread at a time: the state loads of EF21 go out
+    // together (the kept columns are distinct, so no store aliases a load)
+    for (uint32_t i0 = tid; i0 < total; i0 += 4 * kWT) {
+      int e[4];
+      float v[4], g[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const uint32_t i = i0 + q * kWT;
+        e[q] = i < total ? cols[i] : 0;
+        v[q] = cb[e[q]];
+        g[q] = (MODE == kDelta && i < total) ? ar[c0 + e[q]] : 0.0f;
       }
-      if (MODE == kEF) ar[c0 + e] = 0.0f;                    // err' = s - C(s): +0 where sent
-      if (MODE == kDelta) ar[c0 + e] = fadd(ar[c0 + e], v);  // g' = g + d where sent
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const uint32_t i = i0 + q * kWT;
+        if (i >= total) break;
+        const uint64_t pos = base + i;
+        if (pos < static_cast<uint64_t>(k)) {
+          vals[pos] = v[q];
+          idx[pos] = static_cast<int32_t>(c0 + e[q]);
+        }
+        if (MODE == kEF) ar[c0 + e[q]] = 0.0f;               // err' = s - C(s): +0 where sent
+        if (MODE == kDelta) ar[c0 + e[q]] = fadd(g[q], v[q]);  // g' = g + d where sent
+      }
     }
     __syncthreads();  // buffer b, the staged columns and rg / re free again
   }
