@@ -315,12 +315,15 @@ def kernels_of(op: str, L_: int) -> list:
     if op in ("topk", "ef_topk"):
         if L_ <= 1024:
             return ["topk_warp_kernel"]
+        if L_ <= 8192:
+            return ["topk_band_kernel"]
         if L_ <= ROW_PATH_MAX:
             return ["topk_cta_kernel"]
-        return ["g_init", "g_sample"] + ["g_hist", "g_pick"] * 4 + ["g_count", "g_select",
-                                                                   "g_scan", "g_write"]
+        return (["g_init", "g_sample", "w_sample", "w_pass1", "w_pick1", "w_bin2", "w_select2",
+                 "w_mark"] + ["g_hist", "g_pick"] * 4
+                + ["g_count", "g_select", "w_scan1", "w_scan2", "g_write3"])
     if op == "topk_decompress":
-        return ["topk_decompress_rows_kernel" if L_ <= ROW_PATH_MAX else "topk_decompress_kernel"]
+        return ["topk_decompress_tiles_kernel"]
     if op == "quant":
         if L_ <= 2048:
             return ["quant_warp_kernel"]

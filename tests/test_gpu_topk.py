@@ -175,6 +175,22 @@ def test_long_row_decompress_tiles(mpc):
         assert_bits_equal(y.cpu().numpy(), oracle.topk_decompress(vals, idx, L), "k=%d" % k)
 
 
+@pytest.mark.parametrize("R,L", [(4096, 768), (3000, 8192), (5, 8193), (3, 3000001),
+                                 (2, 1 << 22)])
+def test_decompress_tiles_cross_rows(mpc, R, L):
+    """Output tiles of whole short rows (the row of a payload entry found by a high
+    product), rows of exactly one tile, and long rows split into more tiles than there are
+    CTAs, so that a CTA starts inside a row and carries on across row boundaries."""
+    rng = np.random.default_rng(L)
+    for k in sorted({1, 3, L // 100 + 1, L // 2, L}):
+        idx = np.sort(np.stack([rng.choice(L, k, replace=False) for _ in range(R)]),
+                      axis=1).astype(np.int32) if k < L else np.tile(np.arange(L, dtype=np.int32), (R, 1))
+        vals = rng.standard_normal((R, k)).astype(np.float32)
+        y = mpc.mpc_topk_decompress(dev(vals), dev(idx), L)
+        assert_bits_equal(y.cpu().numpy(), oracle.topk_decompress(vals, idx, L),
+                          "R=%d L=%d k=%d" % (R, L, k))
+
+
 # Rows of 8193..32768 entries with enough rows to fill the GPU take one wide CTA each
 # (512 threads up to 16384 entries, else 1024); the knob value 3 keeps them on clusters.
 WIDE = [(160, 8192), (160, 8193), (160, 12345), (160, 16384), (120, 16385), (116, 20000),
