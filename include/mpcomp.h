@@ -303,10 +303,12 @@ const char* mpc_last_error(void);
  *                         up, which tests the timeout report without a fault);
  *   MPC_KNOB_TOPK_PATH    0 = automatic, 1 = force the on-chip row path when
  *                         it fits, 2 = force the multi-pass (workspace) path,
- *                         3 = automatic but rows of 8193..32768 entries always
- *                         split over a cluster of CTAs (never one wide CTA),
- *                         4 = automatic but rows of 1025..8192 entries take
- *                         the cluster / CTA kernels instead of the band kernel;
+ *                         3 = automatic but rows of 8193..65536 entries always
+ *                         split over a cluster of CTAs (never one wide CTA nor
+ *                         the two-pass row kernel),
+ *                         4 = automatic but rows of 1025..65536 entries take
+ *                         the cluster / CTA kernels instead of the band and
+ *                         two-pass row kernels;
  *   MPC_KNOB_PDL          1 (default) = launch the hot kernels with
  *                         programmatic dependent launch, so that a launch
  *                         overlaps the end of the previous one in the stream

@@ -73,6 +73,18 @@ __device__ __forceinline__ void or_if_ge(uint32_t& w, float v, float t, uint32_t
       : "f"(fabsf(v)), "f"(t), "r"(bit));
 }
 
+// w |= bit when |v| > t, and when |v| == t: as or_if_ge.
+__device__ __forceinline__ void or_if_gt(uint32_t& w, float v, float t, uint32_t bit) {
+  asm("{\n .reg .pred p;\n setp.gt.f32 p, %1, %2;\n @p or.b32 %0, %0, %3;\n}"
+      : "+r"(w)
+      : "f"(fabsf(v)), "f"(t), "r"(bit));
+}
+__device__ __forceinline__ void or_if_eq(uint32_t& w, float v, float t, uint32_t bit) {
+  asm("{\n .reg .pred p;\n setp.eq.f32 p, %1, %2;\n @p or.b32 %0, %0, %3;\n}"
+      : "+r"(w)
+      : "f"(fabsf(v)), "f"(t), "r"(bit));
+}
+
 // Shift that maps the key range [lo, hi] (hi > lo) onto at most 256 bins.
 __device__ __forceinline__ int round_shift(int lo, int hi) {
   uint32_t span = static_cast<uint32_t>(hi - lo);

@@ -126,8 +126,8 @@ __device__ __forceinline__ void warp_pick_two(const uint32_t* hist, uint32_t r1,
 // Block sums of a and b, and the exclusive prefix and sum of c, through the
 // scratch set `set` (alternate the set between consecutive calls: the next
 // call's writes then never meet this call's reads, so one barrier suffices).
-template <int NT>
-__device__ __forceinline__ void block_sums(uint32_t a, uint32_t b, uint32_t c, Shared<NT>& sh,
+template <int NT, class SH>
+__device__ __forceinline__ void block_sums(uint32_t a, uint32_t b, uint32_t c, SH& sh,
                                            int set, int lane, int warp, uint32_t* sa,
                                            uint32_t* sb, uint32_t* pc, uint32_t* sc) {
   constexpr int NW = NT / 32;
@@ -160,9 +160,9 @@ __device__ __forceinline__ void block_sums(uint32_t a, uint32_t b, uint32_t c, S
 // Each round a 256-bin histogram of the keys still in the range, the bin
 // holding the kr-th, until one key remains or a bin is taken whole.  Every
 // thread of the block calls it.
-template <int NT, class KeyAt>
-__device__ Threshold select_rounds(KeyAt key_at, int count, int lo, int hi, uint32_t kr,
-                                   Shared<NT>& sh, int tid, int lane, int warp) {
+template <int NT, class SH, class KeyAt>
+__device__ Threshold select_rounds(KeyAt key_at, int count, int lo, int hi, uint32_t kr, SH& sh,
+                                   int tid, int lane, int warp) {
   for (;;) {
     if (lo >= hi) return Threshold{lo, kr};
     const int sft = round_shift(lo, hi);
@@ -192,6 +192,41 @@ __device__ Threshold select_rounds(KeyAt key_at, int count, int lo, int hi, uint
     if (cnt == kr) return Threshold{nlo - 1, 0u};
     lo = nlo;
     hi = nhi;
+  }
+}
+
+// The kr-th largest (1 <= kr <= cnt) of the cnt keys cand[] as a threshold:
+// each key ranked against all others by P threads, partial counts joined by
+// shuffles.  The thread that finds it writes *T (keep keys above it) and *need
+// (how many keys equal to T are kept as well, in index order; 0 when the
+// threshold sits just below a key taken with all its copies).
+template <int NT>
+__device__ void rank_block(const int* cand, uint32_t cnt, uint32_t kr, int* T, uint32_t* need,
+                           int tid) {
+  uint32_t P = 1;
+  while (P < 32 && cnt * P * 2 <= static_cast<uint32_t>(NT)) P *= 2;
+  const uint32_t part = static_cast<uint32_t>(tid) & (P - 1);
+  for (uint32_t c0 = 0; c0 < cnt; c0 += NT / P) {
+    const uint32_t ci = c0 + static_cast<uint32_t>(tid) / P;
+    uint32_t gt = 0, ge = 0;
+    int ki = 0;
+    if (ci < cnt) {
+      ki = cand[ci];
+      for (uint32_t j = part; j < cnt; j += P) {
+        const int aj = cand[j];
+        gt += aj > ki;
+        ge += aj >= ki;
+      }
+    }
+    for (uint32_t o = P >> 1; o > 0; o >>= 1) {
+      gt += __shfl_xor_sync(kFull, gt, o);
+      ge += __shfl_xor_sync(kFull, ge, o);
+    }
+    if (ci < cnt && part == 0 && gt < kr && kr <= ge) {
+      const uint32_t nd = kr - gt;
+      *T = (nd == ge - gt) ? ki - 1 : ki;
+      *need = (nd == ge - gt) ? 0u : nd;
+    }
   }
 }
 
@@ -511,37 +546,13 @@ __global__ void __launch_bounds__(NT, NT == 64 ? 16 : (NT == 128 ? 10 : 5))
         T = th.T;
         need = th.need;
       } else {
-        // the bin's entries ranked against each other on the block (P threads each)
+        // the bin's entries ranked against each other on the block
         for (uint32_t i = tid; i < m; i += NT) {
           const int key = key_at(static_cast<int>(i));
           if (key >= bl && key <= bh) sh.u.cand[atomicAdd(&sh.ccount, 1u)] = key;
         }
         __syncthreads();
-        uint32_t P = 1;
-        while (P < 32 && cnt * P * 2 <= static_cast<uint32_t>(NT)) P *= 2;
-        const uint32_t part = static_cast<uint32_t>(tid) & (P - 1);
-        for (uint32_t c0 = 0; c0 < cnt; c0 += NT / P) {
-          const uint32_t ci = c0 + static_cast<uint32_t>(tid) / P;
-          uint32_t gt = 0, ge = 0;
-          int ki = 0;
-          if (ci < cnt) {
-            ki = sh.u.cand[ci];
-            for (uint32_t j = part; j < cnt; j += P) {
-              const int aj = sh.u.cand[j];
-              gt += aj > ki;
-              ge += aj >= ki;
-            }
-          }
-          for (uint32_t o = P >> 1; o > 0; o >>= 1) {
-            gt += __shfl_xor_sync(kFull, gt, o);
-            ge += __shfl_xor_sync(kFull, ge, o);
-          }
-          if (ci < cnt && part == 0 && gt < kr2 && kr2 <= ge) {
-            const uint32_t nd = kr2 - gt;
-            sh.T = (nd == ge - gt) ? ki - 1 : ki;
-            sh.need = (nd == ge - gt) ? 0u : nd;
-          }
-        }
+        rank_block<NT>(sh.u.cand, cnt, kr2, &sh.T, &sh.need, tid);
         __syncthreads();
         T = sh.T;
         need = sh.need;

@@ -34,6 +34,7 @@
 #include "launch_util.h"
 #include "select.cuh"
 #include "topk_band.cuh"
+#include "topk_lrow.cuh"
 
 namespace mpc {
 namespace rows {
@@ -1270,6 +1271,10 @@ cudaError_t run_mode(const TopkRowArgs& a0, int num_sms, cudaStream_t s) {
   // Rows of 1025..8192 entries take the band kernel (topk_band.cuh) unless the
   // knob keeps the kernels below.
   if (a.band && band::fits(L)) return band::run_mode<MODE>(a, s);
+  // Aligned rows of 8193..65536 entries: one 512-thread CTA per row reading the
+  // row twice, the second time from L2 (topk_lrow.cuh), unless the knob keeps
+  // the kernels below.
+  if (a.band && a.wide_cta && lrow::fits(a)) return lrow::run_mode<MODE>(a, s);
   // One CTA of 128 threads for rows up to 4096 entries, else clusters of
   // 256-thread CTAs holding up to 8192 entries each, split further (slices of
   // at least 2048 entries) while the grid has fewer than 2 CTAs per SM.
@@ -1294,7 +1299,7 @@ cudaError_t run_mode(const TopkRowArgs& a0, int num_sms, cudaStream_t s) {
     return run_cta_any<MODE, 1024, 32768>(a, 1, s);
   }
   int64_t C = (L + 8191) / 8192;
-  while (a.rows * C < 2 * num_sms && C < kMaxCluster && L / (2 * C) >= 2048) C *= 2;
+  while (a.rows * C < 2 * num_sms && 2 * C <= kMaxCluster && L / (2 * C) >= 2048) C *= 2;
   if (C > kMaxCluster) return cudaErrorInvalidValue;
   a.slice = ((L + C - 1) / C + 3) / 4 * 4;
   return run_cta_any<MODE, 256, 8192>(a, static_cast<int>(C), s);

@@ -26,10 +26,14 @@ def mpc():
     m.mpc_set_knob(m.MPC_KNOB_SPIN_LIMIT, DEFAULT_SPIN)
 
 
-@pytest.mark.parametrize("op,L", [("ef", 4096), ("ef", 32768), ("plain", 768), ("quant", 32768)])
-def test_timeout_is_reported_and_context_survives(mpc, op, L):
+# (op, row length, TopK path knob): the band kernel, the cluster kernels (knob 3: the
+# two-pass row kernel, which waits on no copy, stays out), the warp kernel, quantisation
+@pytest.mark.parametrize("op,L,path", [("ef", 4096, 0), ("ef", 32768, 3), ("plain", 768, 0),
+                                       ("quant", 32768, 0)])
+def test_timeout_is_reported_and_context_survives(mpc, op, L, path):
     x = torch.from_numpy(rows_of("normal", 6, L, seed=1)).cuda()
     err = torch.zeros_like(x)
+    mpc.mpc_set_knob(mpc.MPC_KNOB_TOPK_PATH, path)
     mpc.mpc_set_knob(mpc.MPC_KNOB_SPIN_LIMIT, 0)
     try:
         if op == "ef":
@@ -42,6 +46,7 @@ def test_timeout_is_reported_and_context_survives(mpc, op, L):
         assert "wait" in mpc.mpc_last_error()
     finally:
         mpc.mpc_set_knob(mpc.MPC_KNOB_SPIN_LIMIT, DEFAULT_SPIN)
+        mpc.mpc_set_knob(mpc.MPC_KNOB_TOPK_PATH, 0)
     assert mpc.mpc_get_status() == 0
     # the same call now succeeds and matches the oracle
     xn = x.cpu().numpy()
