@@ -34,7 +34,16 @@ constexpr int kQSCAP = 4 * kQNT * kQNV;  // 8192 entries per CTA slice
 // reversed.  Its inverse recovers the exact float.
 __device__ __forceinline__ uint32_t ord_key(float v) {
   const uint32_t u = __float_as_uint(v);
-  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+  // negative: all bits flipped; else the sign bit set (an arithmetic shift and
+  // one three-input logic operation)
+  return u ^ (static_cast<uint32_t>(static_cast<int32_t>(u) >> 31) | 0x80000000u);
+}
+
+// Extrema keys of a 4-entry group, folded into (kmin, kmax).
+__device__ __forceinline__ void fold_keys4(const float4 f, uint32_t& kmin, uint32_t& kmax) {
+  const uint32_t k0 = ord_key(f.x), k1 = ord_key(f.y), k2 = ord_key(f.z), k3 = ord_key(f.w);
+  kmin = min(kmin, min(min(k0, k1), min(k2, k3)));
+  kmax = max(kmax, max(max(k0, k1), max(k2, k3)));
 }
 __device__ __forceinline__ float ord_value(uint32_t k) {
   return __uint_as_float((k & 0x80000000u) ? (k & 0x7fffffffu) : ~k);
@@ -102,6 +111,30 @@ __device__ __forceinline__ uint32_t code_of(float x, const RowParams& p, float u
   return __float_as_uint(fadd(q, 8388608.0f)) & 0x7fffffu;
 }
 
+// The 4 codes of a whole group as one 4*BITS-bit piece.  Each code leaves the
+// FP32 pipe as the bit pattern of q + 2^23 (= 0x4b000000 + q); the patterns are
+// combined by multiply-adds (p3 * S + p2) * S ... with S = 2^BITS, and the
+// constant 0x4b000000 * (1 + S + S^2 + S^3) taken off once (all mod 2^32, exact
+// as the result is below 2^32).  Nearest rounding needs no clamp: for finite x
+// in [mn, mx], t = (x - mn) * inv stays in [0, levels * (1 + 2^-23)], so
+// round-half-even of t lies in [0, levels].  Stochastic rounding keeps the upper
+// clamp (t + u may round up to levels + 1).
+template <int BITS, bool SR>
+__device__ __forceinline__ uint32_t pack4(const float xs[4], const RowParams& p, const float u[4]) {
+  uint32_t b[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float t = fmul(fsub(xs[i], p.mn), p.inv);
+    float q;
+    if (SR) q = fminf(floorf(fadd(t, u[i])), p.levels);
+    else q = rintf(t);
+    b[i] = __float_as_uint(fadd(q, 8388608.0f));
+  }
+  constexpr uint32_t S = 1u << BITS;
+  constexpr uint32_t kBias = 0x4b000000u * (1u + S + S * S + S * S * S);
+  return ((b[3] * S + b[2]) * S + b[1]) * S + b[0] - kBias;
+}
+
 // Codes of the 4 entries e0..e0+3 of a row (entries at or past n give 0).
 // u: the stochastic rounding offsets of the 4 entries (unused for nearest).
 template <int BITS, bool SR>
@@ -110,8 +143,7 @@ __device__ __forceinline__ uint32_t codes4(const float xs[4], int64_t e0, int64_
   uint32_t packed = 0;
   if (p.degenerate) return 0;
   if (e0 + 4 <= n) {
-#pragma unroll
-    for (int t = 0; t < 4; ++t) packed |= code_of<SR>(xs[t], p, u[t]) << (BITS * t);
+    packed = pack4<BITS, SR>(xs, p, u);
   } else {
 #pragma unroll
     for (int t = 0; t < 4; ++t)
@@ -178,36 +210,65 @@ __device__ __forceinline__ void store_codes_any(uint64_t piece, int bits, int la
 // ---------------------------------------------------------------------------
 // One warp per row
 // ---------------------------------------------------------------------------
+// Rows of up to 768 entries hold the warp's next row in registers while this
+// one is coded, so that its loads are in flight meanwhile (three CTAs per SM;
+// longer rows would spill).
 template <int BITS, int NVW, bool SR>
-__global__ void __launch_bounds__(32 * kQWarps, NVW <= 8 ? 4 : 2) quant_warp_kernel(const QuantArgs a) {
+__global__ void __launch_bounds__(32 * kQWarps, NVW <= 6 ? 3 : (NVW <= 8 ? 4 : 2))
+    quant_warp_kernel(const QuantArgs a) {
   pdl_begin();
   __shared__ uint32_t gbuf[BITS == 0 ? kQWarps * 64 : 1];  // width-b packing, per warp
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int64_t L = a.L;
   const int bits = BITS == 0 ? a.bits : BITS;
   const int64_t data_words = (L * bits + 31) / 32;
-  for (int64_t row = static_cast<int64_t>(blockIdx.x) * kQWarps + warp; row < a.rows;
-       row += static_cast<int64_t>(gridDim.x) * kQWarps) {
-    const float* xr = a.x + row * L;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * kQWarps;
+  constexpr bool kPre = NVW <= 6;
+  // this lane's groups of row r (+0 past the row's end)
+  auto fetch = [&](int64_t r, float4* f) {
+    const float* xr = a.x + r * L;
+#pragma unroll
+    for (int v = 0; v < NVW; ++v) {
+      const int64_t e0 = 4 * (v * 32 + lane);
+      if (a.aligned && e0 + 4 <= L) {
+        f[v] = *reinterpret_cast<const float4*>(xr + e0);
+      } else {
+        float s[4];
+#pragma unroll
+        for (int t = 0; t < 4; ++t) s[t] = (e0 + t < L) ? xr[e0 + t] : 0.0f;
+        f[v] = make_float4(s[0], s[1], s[2], s[3]);
+      }
+    }
+  };
+  float4 nxt[kPre ? NVW : 1];
+  int64_t row = static_cast<int64_t>(blockIdx.x) * kQWarps + warp;
+  if (kPre && row < a.rows) fetch(row, nxt);
+  for (; row < a.rows; row += stride) {
+    float4 cur[NVW];
+    if (kPre) {
+#pragma unroll
+      for (int v = 0; v < NVW; ++v) cur[v] = nxt[v];
+      if (row + stride < a.rows) fetch(row + stride, nxt);
+    } else {
+      fetch(row, cur);
+    }
     float xs[NVW][4];
     uint32_t kmin = 0xffffffffu, kmax = 0u;
 #pragma unroll
     for (int v = 0; v < NVW; ++v) {
       const int64_t e0 = 4 * (v * 32 + lane);
-      if (a.aligned && e0 + 4 <= L) {
-        const float4 f = *reinterpret_cast<const float4*>(xr + e0);
-        xs[v][0] = f.x; xs[v][1] = f.y; xs[v][2] = f.z; xs[v][3] = f.w;
+      xs[v][0] = cur[v].x; xs[v][1] = cur[v].y; xs[v][2] = cur[v].z; xs[v][3] = cur[v].w;
+      if (e0 + 4 <= L) {
+        fold_keys4(cur[v], kmin, kmax);
       } else {
 #pragma unroll
-        for (int t = 0; t < 4; ++t) xs[v][t] = (e0 + t < L) ? xr[e0 + t] : 0.0f;
+        for (int t = 0; t < 4; ++t)
+          if (e0 + t < L) {
+            const uint32_t ok = ord_key(xs[v][t]);
+            kmin = min(kmin, ok);
+            kmax = max(kmax, ok);
+          }
       }
-#pragma unroll
-      for (int t = 0; t < 4; ++t)
-        if (e0 + t < L) {
-          const uint32_t ok = ord_key(xs[v][t]);
-          kmin = min(kmin, ok);
-          kmax = max(kmax, ok);
-        }
     }
     kmin = __reduce_min_sync(kFull, kmin);
     kmax = __reduce_max_sync(kFull, kmax);
@@ -289,14 +350,18 @@ __global__ void __launch_bounds__(NT) quant_cta_kernel(const QuantArgs a, int sp
       }
       const int q = v * NT + tid;
       const float4 f = reinterpret_cast<const float4*>(sx)[q];
-      const float xs[4] = {f.x, f.y, f.z, f.w};
+      if (4 * q + 4 <= n) {
+        fold_keys4(f, kmin, kmax);
+      } else {
+        const float xs[4] = {f.x, f.y, f.z, f.w};
 #pragma unroll
-      for (int t = 0; t < 4; ++t)
-        if (4 * q + t < n) {
-          const uint32_t ok = ord_key(xs[t]);
-          kmin = min(kmin, ok);
-          kmax = max(kmax, ok);
-        }
+        for (int t = 0; t < 4; ++t)
+          if (4 * q + t < n) {
+            const uint32_t ok = ord_key(xs[t]);
+            kmin = min(kmin, ok);
+            kmax = max(kmax, ok);
+          }
+      }
     }
   }
   failed = __syncthreads_or(failed);
@@ -710,6 +775,9 @@ cudaError_t run_quant_bits(const QuantArgs& a0, int num_sms, cudaStream_t s) {
     if (L <= 1024) return run_quant_warp<BITS, 8, SR>(a, num_sms, s);
     return run_quant_warp<BITS, 16, SR>(a, num_sms, s);
   }
+  // Rows of 2049..4096 entries: one CTA of 128 threads each (32 entries a
+  // thread, so that the per-row work of a thread is spread over more entries).
+  if (a.ws == nullptr && L <= 4 * 128 * kQNV) return run_quant_wide<BITS, SR, 128>(a, s);
   // Rows of 8193..32768 entries take one wide CTA each (512 threads and two
   // CTAs per SM up to 16384, else 1024 threads and one per SM) when that
   // fills the GPU in one wave: the row's extrema then need no cluster barrier.
