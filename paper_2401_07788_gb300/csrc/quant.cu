@@ -297,6 +297,101 @@ __global__ void __launch_bounds__(32 * kQWarps, NVW <= 6 ? 3 : (NVW <= 8 ? 4 : 2
 }
 
 // ---------------------------------------------------------------------------
+// Rows of 2049..4096 entries: four warps per row, row in registers
+// ---------------------------------------------------------------------------
+// Thread t of the CTA holds the groups q = 128 v + t (v < 8) of its row, and
+// the same groups of the CTA's next row (loads in flight while this row is
+// coded).  Extrema by warp reductions and one CTA barrier per row (the
+// per-warp partials alternate between two slots).
+constexpr int kR4NVW = 8;
+
+template <int BITS, bool SR>
+__global__ void __launch_bounds__(128, 5) quant_rows4_kernel(const QuantArgs a) {
+  pdl_begin();
+  __shared__ uint32_t red[2][2][4];
+  __shared__ uint32_t gbuf[BITS == 0 ? 4 * 64 : 1];  // width-b packing, per warp
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int64_t L = a.L;
+  const int bits = BITS == 0 ? a.bits : BITS;
+  const int64_t data_words = (L * bits + 31) / 32;
+  auto fetch = [&](int64_t r, float4* f) {
+    const float* xr = a.x + r * L;
+#pragma unroll
+    for (int v = 0; v < kR4NVW; ++v) {
+      const int64_t e0 = 4 * (v * 128 + tid);
+      if (a.aligned && e0 + 4 <= L) {
+        f[v] = *reinterpret_cast<const float4*>(xr + e0);
+      } else {
+        float s[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) s[i] = (e0 + i < L) ? xr[e0 + i] : 0.0f;
+        f[v] = make_float4(s[0], s[1], s[2], s[3]);
+      }
+    }
+  };
+  float4 nxt[kR4NVW];
+  int64_t row = blockIdx.x;
+  if (row < a.rows) fetch(row, nxt);
+  for (int it = 0; row < a.rows; row += gridDim.x, ++it) {
+    float4 cur[kR4NVW];
+#pragma unroll
+    for (int v = 0; v < kR4NVW; ++v) cur[v] = nxt[v];
+    if (row + gridDim.x < a.rows) fetch(row + gridDim.x, nxt);
+    uint32_t kmin = 0xffffffffu, kmax = 0u;
+#pragma unroll
+    for (int v = 0; v < kR4NVW; ++v) {
+      const int64_t e0 = 4 * (v * 128 + tid);
+      if (e0 + 4 <= L) {
+        fold_keys4(cur[v], kmin, kmax);
+      } else {
+        const float xs[4] = {cur[v].x, cur[v].y, cur[v].z, cur[v].w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+          if (e0 + i < L) {
+            const uint32_t ok = ord_key(xs[i]);
+            kmin = min(kmin, ok);
+            kmax = max(kmax, ok);
+          }
+      }
+    }
+    kmin = __reduce_min_sync(kFull, kmin);
+    kmax = __reduce_max_sync(kFull, kmax);
+    const int sl = it & 1;
+    if (lane == 0) {
+      red[sl][0][warp] = kmin;
+      red[sl][1][warp] = kmax;
+    }
+    __syncthreads();
+    kmin = min(min(red[sl][0][0], red[sl][0][1]), min(red[sl][0][2], red[sl][0][3]));
+    kmax = max(max(red[sl][1][0], red[sl][1][1]), max(red[sl][1][2], red[sl][1][3]));
+    const RowParams p = row_params(kmin, kmax, bits, tid == 0 ? a.scale + row : nullptr,
+                                   tid == 0 ? a.minv + row : nullptr);
+    uint32_t* cr = a.codes + row * a.W;
+#pragma unroll
+    for (int v = 0; v < kR4NVW; ++v) {
+      const int64_t e0 = 4 * (v * 128 + tid);
+      const float xs[4] = {cur[v].x, cur[v].y, cur[v].z, cur[v].w};
+      float u[4] = {0.f, 0.f, 0.f, 0.f};
+      if constexpr (BITS == 0) {
+        const int64_t chunk = 128 * (v * 4 + warp);  // the warp's 128 entries
+        if (chunk < L) {
+          if (SR) uniform4(a.seed, static_cast<uint64_t>(row * L + e0), u);
+          const uint64_t piece = codes4_any<SR>(xs, e0, L, p, u, bits);
+          store_codes_any(piece, bits, lane, gbuf + warp * 64, cr, chunk * bits / 32, data_words);
+        }
+      } else {
+        if (SR) uniform4(a.seed, static_cast<uint64_t>(row * L + e0), u);
+        uint32_t piece = codes4<BITS, SR>(xs, e0, L, p, u);
+        const bool store = assemble_word<BITS>(piece, lane);
+        const int64_t w = e0 * BITS / 32;
+        if (store && w < data_words) cr[w] = piece;
+      }
+    }
+    if (tid < a.W - data_words) cr[data_words + tid] = 0u;  // row padding
+  }
+}
+
+// ---------------------------------------------------------------------------
 // Cluster of CTAs per row (or, with a workspace, CTAs over one row's chunks)
 // ---------------------------------------------------------------------------
 template <int NT>
@@ -775,9 +870,14 @@ cudaError_t run_quant_bits(const QuantArgs& a0, int num_sms, cudaStream_t s) {
     if (L <= 1024) return run_quant_warp<BITS, 8, SR>(a, num_sms, s);
     return run_quant_warp<BITS, 16, SR>(a, num_sms, s);
   }
-  // Rows of 2049..4096 entries: one CTA of 128 threads each (32 entries a
-  // thread, so that the per-row work of a thread is spread over more entries).
-  if (a.ws == nullptr && L <= 4 * 128 * kQNV) return run_quant_wide<BITS, SR, 128>(a, s);
+  // Rows of 2049..4096 entries: four warps per row, rows in registers
+  if (a.ws == nullptr && L <= 4 * 128 * kR4NVW) {
+    auto kernel = quant_rows4_kernel<BITS, SR>;
+    const int occ = resident_blocks(kernel, 128, 0);
+    const int64_t cap = static_cast<int64_t>(num_sms) * (occ > 0 ? occ : 1);
+    return launch_kernel(kernel, dim3(static_cast<unsigned>(a.rows < cap ? a.rows : cap)), dim3(128),
+                         0, s, 0u, a);
+  }
   // Rows of 8193..32768 entries take one wide CTA each (512 threads and two
   // CTAs per SM up to 16384, else 1024 threads and one per SM) when that
   // fills the GPU in one wave: the row's extrema then need no cluster barrier.
