@@ -319,9 +319,9 @@ def kernels_of(op: str, L_: int) -> list:
             return ["topk_band_kernel"]
         if L_ <= ROW_PATH_MAX:
             return ["topk_lrow_kernel"]  # 16-byte aligned rows (the sweep's are)
-        return (["g_init", "g_sample", "w_sample", "w_pass1", "w_pick1", "w_bin2", "w_select2",
-                 "w_mark"] + ["g_hist", "g_pick"] * 4
-                + ["g_count", "g_select", "w_scan1", "w_scan2", "g_write3"])
+        return (["g_init", "w_sample", "w_spick", "w_pass1", "w_pick1", "w_bin2", "w_select2",
+                 "w_mark", "g_sample"] + ["g_hist", "g_pick"] * 4
+                + ["g_count", "g_select", "w_scan1", "w_scan2", "g_write3", "g_wlist"])
     if op == "topk_decompress":
         return ["topk_decompress_tiles_kernel"]
     if op == "quant":

@@ -4,26 +4,30 @@
 // status words in a caller workspace; one row at a time.
 //
 // Per row, the selection by the band path (one read of the row), else by the
-// multi-pass path where the band path gave up, then the write (one more read).
+// multi-pass path where the band path gave up, then the write: one more read
+// of the row, or, in list mode (k up to a thirty-second of the row), the
+// payload from the list of every entry >= t_lo that the band path's read made.
 // Every kernel returns at once when the device-side state says its step is not
 // needed, so the host never waits.
 //
 // Band path:
-//   w_sample  65536 entries spread over the row give a band of keys
-//             [t_lo, t_hi) that holds the k-th largest magnitude unless the
-//             sample is 4 standard deviations off (as in topk_band.cuh);
+//   w_sample, w_spick  65536 entries spread over the row (one a thread over 64
+//             CTAs) give a band of keys [t_lo, t_hi) that holds the k-th
+//             largest magnitude unless the sample is 4 standard deviations
+//             off (as in topk_band.cuh);
 //   w_pass1   one read of the row by persistent CTAs, 8192-entry chunks staged
 //             by double-buffered bulk copies: entries >= t_hi ("sure")
-//             counted; band entries listed in the workspace (a region per CTA)
-//             and counted in a 256-bin histogram of their keys (error feedback:
-//             s = x + err written back into err, which the write reads);
+//             counted; band entries (list mode: every entry >= t_lo) listed in
+//             the workspace (a region per CTA, each chunk's entries one segment
+//             in index order) and the band's counted in a 256-bin histogram of
+//             their keys (error feedback: s = x + err written back into err);
 //   w_pick1   the histogram bin holding the k-th entry (or: the band missed,
 //             and the multi-pass path takes over);
 //   w_bin2    the band entries in that bin, listed;
 //   w_select2 T and `need` among them by integer rounds.
 //
 // Multi-pass path:
-//   init     clear the row's state;
+//   init     clear the row's state (before the band path);
 //   sample   bin scale from a strided sample of the ranked values;
 //   hist     histogram of all entries over bins linear in |x| (error feedback:
 //            s = x + err is written back into err unless the band path did);
@@ -40,7 +44,8 @@
 //
 // Write (both paths): w_scan1 / w_scan2, the prefix sums of the per-chunk
 // counts; g_write3, persistent CTAs over 4096-entry chunks, double-buffered:
-// the payload in ascending index order and the buffer updates.
+// the payload in ascending index order and the buffer updates; or, in list
+// mode, g_wlist: the same from the list's segments.
 #include "common.cuh"
 #include "kernels.h"
 #include "launch_util.h"
@@ -57,8 +62,9 @@ constexpr uint32_t kCandCap = 65536;     // candidate list capacity
 constexpr int kSamples = 4096;
 constexpr int kMaxRounds = 3;            // refinement rounds (11 bits each) reach one key
 constexpr int kWSamples = 65536;         // band path: sample entries
-constexpr int kWSBins = 4096;            // band path: sample bins (1/128 octave)
-constexpr int kWSShift = 16;             // band path: sample bin = (key - base) >> 16
+constexpr int kWSCtas = kWSamples / 1024;  // band path: sampling CTAs (one entry a thread)
+constexpr int kWSBins = 32768;           // band path: sample bins, key >> 16 (1/128 octave)
+constexpr int kWSShift = 16;
 constexpr int kFBins = 256;              // band path: bins of the band histogram
 constexpr uint32_t kCand2Cap = 1u << 21;  // band path: entries of the chosen bin
 constexpr float kWZ = 4.0f;              // band half-width in standard deviations
@@ -90,6 +96,8 @@ struct GridMeta {
   int b_lo, b_hi;   // the chosen band bin's keys
   uint32_t b_kr;    // rank of T within it
   uint32_t ncand2;
+  int lmode;        // list mode: every entry >= t_lo listed (the payload comes from the list)
+  int smax;         // largest finite sample key (band path)
 };
 
 struct WsLayout {
@@ -103,8 +111,11 @@ struct WsLayout {
   int* ckey;        // kCandCap candidate keys
   int64_t* cidx;    // kCandCap candidate positions
   uint32_t* fhist;  // kFBins: band histogram
-  int* bkey;        // band list: keys
+  uint32_t* shist;  // kWSBins: sample histogram
+  int* bkey;        // band list: value bits (magnitude key = bits & 0x7fffffff)
   uint32_t* bidx;   //            positions in the row
+  uint32_t* seg;    // per pass-1 chunk: start of its entries in its CTA's region
+  uint32_t* segn;   //                   and their number
   int* c2key;       // kCand2Cap: keys of the chosen band bin
   uint32_t* nbc;    // kMaxBandCtas: band entries listed by each CTA of w_pass1
   uint32_t bcap;    // band list capacity (G regions of bcap / G entries, G the pass-1 grid)
@@ -115,12 +126,20 @@ struct WsLayout {
 constexpr int kMaxBandCtas = 4096;
 
 // Band list capacity: a sixteenth of the row and 64K entries (the band of a
-// 16384-entry sample at 4 standard deviations is a few percent of the row).
-uint32_t band_cap(int64_t L) { return static_cast<uint32_t>(L / 16 + 65536); }
+// 65536-entry sample at 4 standard deviations is a few percent of the row);
+// for k up to a thirty-second of the row, room for list mode too: k, a quarter
+// more, a sixty-fourth of the row and 64K entries.  (Beyond that the list costs
+// more to build and read back than the second read of the row it saves.)
+bool list_eligible(int64_t L, int64_t k) { return k <= L / 32; }
+uint32_t band_cap(int64_t L, int64_t k) {
+  int64_t c = L / 16 + 65536;
+  if (list_eligible(L, k)) c = max64(c, k + k / 4 + L / 64 + 65536);
+  return static_cast<uint32_t>(min64(c, 0xffffffffLL));
+}
 
 size_t align256(size_t b) { return (b + 255) / 256 * 256; }
 
-WsLayout layout(void* ws, int64_t L, int64_t nchunks) {
+WsLayout layout(void* ws, int64_t L, int64_t k, int64_t nchunks) {
   WsLayout w;
   char* p = static_cast<char*>(ws);
   w.meta = reinterpret_cast<GridMeta*>(p);
@@ -142,25 +161,33 @@ WsLayout layout(void* ws, int64_t L, int64_t nchunks) {
   p += align256(kCandCap * 4);
   w.fhist = reinterpret_cast<uint32_t*>(p);
   p += align256(kFBins * 4);
+  w.shist = reinterpret_cast<uint32_t*>(p);
+  p += align256(kWSBins * 4);
   w.c2key = reinterpret_cast<int*>(p);
   p += align256(static_cast<size_t>(kCand2Cap) * 4);
   w.nbc = reinterpret_cast<uint32_t*>(p);
   p += align256(kMaxBandCtas * 4);
-  w.bcap = band_cap(L);
+  w.bcap = band_cap(L, k);
   w.bkey = reinterpret_cast<int*>(p);
   p += align256(static_cast<size_t>(w.bcap) * 4);
   w.bidx = reinterpret_cast<uint32_t*>(p);
+  p += align256(static_cast<size_t>(w.bcap) * 4);
+  w.seg = reinterpret_cast<uint32_t*>(p);
+  p += align256(static_cast<size_t>(nchunks) * 4);
+  w.segn = reinterpret_cast<uint32_t*>(p);
   return w;
 }
 
-size_t ws_bytes_for(int64_t L) {
+size_t ws_bytes_for(int64_t L, int64_t k) {
   const int64_t nchunks = (L + kCH - 1) / kCH;
-  return align256(sizeof(GridMeta)) + align256(kGNB * 4) +
+  return 2 * align256(static_cast<size_t>(nchunks) * 4) + align256(sizeof(GridMeta)) +
+         align256(kGNB * 4) +
          2 * align256(static_cast<size_t>((L + kWCH - 1) / kWCH) * 4) +
          2 * align256(static_cast<size_t>(((L + kWCH - 1) / kWCH + 1023) / 1024) * 4) +
          align256(kCandCap * 8) + align256(kCandCap * 4) + align256(kFBins * 4) +
+         align256(kWSBins * 4) +
          align256(static_cast<size_t>(kCand2Cap) * 4) + align256(kMaxBandCtas * 4) +
-         2 * align256(static_cast<size_t>(band_cap(L)) * 4);
+         2 * align256(static_cast<size_t>(band_cap(L, k)) * 4);
 }
 
 template <int MODE>
@@ -190,14 +217,23 @@ __device__ __forceinline__ uint32_t block_sum(uint32_t v, uint32_t* red) {
   return s;
 }
 
-__global__ void g_init(GridMeta* meta, uint32_t* hist, int64_t nchunks) {
+__global__ void g_init(GridMeta* meta, uint32_t* hist, uint32_t* shist, uint32_t* fhist,
+                       int64_t nchunks, int64_t L, int64_t k) {
   pdl_begin();
   for (int i = threadIdx.x; i < kGNB; i += blockDim.x) hist[i] = 0;
+  for (int i = threadIdx.x; i < kWSBins; i += blockDim.x) shist[i] = 0;
+  for (int i = threadIdx.x; i < kFBins; i += blockDim.x) fhist[i] = 0;
   if (threadIdx.x == 0) {
     GridMeta m = {};
     m.lo = 0;
     m.hi = 0x7fffffff;
     m.nchunks = static_cast<uint32_t>(nchunks);
+    m.smax = -1;
+    if (k >= L) {  // every entry is kept
+      m.resolved = 1;
+      m.T = -1;
+      m.need = 0;
+    }
     *meta = m;
   }
 }
@@ -207,6 +243,7 @@ __global__ void __launch_bounds__(kGT) g_sample(const float* xr, const float* ar
                                                 int64_t k, GridMeta* meta) {
   pdl_begin();
   __shared__ uint32_t red[kGT / 32];
+  if (meta->resolved) return;  // the band path found T (or every entry is kept)
   int mx = -1;
   for (int s = threadIdx.x; s < kSamples; s += kGT) {
     const int64_t e = (L / kSamples) * s;
@@ -221,11 +258,6 @@ __global__ void __launch_bounds__(kGT) g_sample(const float* xr, const float* ar
     meta->scale = bucket_scale(m, kGNB);
     meta->kr = static_cast<uint32_t>(k);
     meta->m = static_cast<uint32_t>(L);
-    if (k >= L) {  // every entry is kept
-      meta->resolved = 1;
-      meta->T = -1;
-      meta->need = 0;
-    }
     if (meta->scale == 0.0f) {
       meta->round = 1;  // integer bins over the whole key range, 2048 of them
       meta->sft = 21 - __clz(0x7fffffff);
@@ -492,71 +524,79 @@ __device__ __forceinline__ uint32_t excl_scan_1024(uint32_t v, uint32_t* red, ui
 // Band path
 // ===========================================================================
 
-// The band from a sample of the row (one CTA): 65536 entries spread evenly
-// over the row, binned by magnitude key (4096 bins of 1/128 octave below the
-// largest finite sample magnitude); the band reaches 4 standard deviations of
-// the sample count on either side of the k-th entry.
+// The band from a sample of the row.  w_sample: 65536 entries spread evenly
+// over the row, one a thread over kWSCtas CTAs, binned by magnitude key into
+// 32768 bins of 1/128 octave (key >> 16), and the largest finite sample key.
+// w_spick (one CTA): the band reaches 4 standard deviations of the sample count
+// on either side of the k-th entry; list mode when the sample's count at or
+// above t_lo, scaled to the row with a margin, fits the list.
 template <int MODE>
 __global__ void __launch_bounds__(1024) w_sample(const float* xr, const float* ar, int64_t L,
-                                                 int64_t k, GridMeta* meta, uint32_t* fhist) {
+                                                 GridMeta* meta, uint32_t* shist) {
   pdl_begin();
-  constexpr int G = kWSBins / 1024;  // bins per thread
-  __shared__ uint32_t hist[kWSBins];
-  __shared__ uint32_t red[32];
-  __shared__ int pick[2];
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   if (meta->resolved) return;  // every entry is kept
-  for (int i = tid; i < kWSBins; i += 1024) hist[i] = 0;
-  for (int i = tid; i < kFBins; i += 1024) fhist[i] = 0;
-  if (tid < 2) pick[tid] = -1;
-  constexpr int PER = kWSamples / 1024;
-  int key[PER];
-  int mx = -1;
-#pragma unroll 16
-  for (int j = 0; j < PER; ++j) {
-    const int64_t e = (static_cast<int64_t>(j) * 1024 + tid) * L / kWSamples;
-    key[j] = mag_key(ranked<MODE>(xr[e], MODE != kPlain ? ar[e] : 0.0f));
-    mx = max(mx, finite_key(key[j]));
-  }
-  mx = __reduce_max_sync(kFull, mx);
-  if (lane == 0) red[warp] = static_cast<uint32_t>(mx);
-  __syncthreads();
-  int smax = -1;
-  for (int w = 0; w < 32; ++w) smax = max(smax, static_cast<int>(red[w]));
+  const int64_t s = static_cast<int64_t>(blockIdx.x) * 1024 + threadIdx.x;
+  const int64_t e = s * L / kWSamples;
+  const int key = mag_key(ranked<MODE>(xr[e], MODE != kPlain ? ar[e] : 0.0f));
+  // lanes with the same bin add once
+  const uint32_t bin = static_cast<uint32_t>(key) >> kWSShift;
+  const unsigned same = __match_any_sync(kFull, bin);
+  if ((threadIdx.x & 31) == __ffs(same) - 1) atomicAdd(&shist[bin], static_cast<uint32_t>(__popc(same)));
+  const int mx = __reduce_max_sync(kFull, finite_key(key));
+  if ((threadIdx.x & 31) == 0 && mx > 0) atomicMax(&meta->smax, mx);
+}
+
+__global__ void __launch_bounds__(1024) w_spick(int64_t L, int64_t k, GridMeta* meta,
+                                                const uint32_t* shist, int list_ok, uint32_t bcap) {
+  pdl_begin();
+  // bins in rank order (largest keys first): warp w reads ranks [1024 w, 1024 w + 1024),
+  // lane l the ranks 1024 w + 32 j + l (coalesced)
+  constexpr int J = kWSBins / 1024;
+  __shared__ uint32_t wsum[32];
+  __shared__ int pick[2];
+  __shared__ uint32_t s_ge;  // sample entries in the bins down to t_lo's
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  if (meta->resolved) return;
+  const int smax = meta->smax;
   if (smax <= 0) return;  // no finite non-zero magnitude in the sample: multi-pass path
-  const int base = max(0, smax - ((kWSBins - 1) << kWSShift));
-#pragma unroll 16
-  for (int j = 0; j < PER; ++j)
-    atomicAdd(&hist[min(max(key[j] - base, 0) >> kWSShift, kWSBins - 1)], 1u);
-  __syncthreads();
-  // the bins holding the r_hi-th and the r_lo-th largest sample keys
+  if (tid < 2) pick[tid] = -1;
+  if (tid == 0) s_ge = kWSamples;
   const float mu = __fdividef(static_cast<float>(k) * static_cast<float>(kWSamples),
                               static_cast<float>(L));
   const float sd = mu * rsqrtf(mu);
   const int r_hi = static_cast<int>(floorf(mu - kWZ * sd));
   const int r_lo = static_cast<int>(ceilf(mu + kWZ * sd)) + 1;
-  uint32_t c[G], tsum = 0;
+  uint32_t v[J], s = 0;
 #pragma unroll
-  for (int g = 0; g < G; ++g) {
-    c[g] = hist[kWSBins - 1 - (tid * G + g)];
-    tsum += c[g];
+  for (int j = 0; j < J; ++j) {
+    v[j] = shist[kWSBins - 1 - (1024 * warp + 32 * j + lane)];
+    s += v[j];
   }
-  uint32_t total;
-  const uint32_t excl = excl_scan_1024(tsum, red, &total);
+  s = __reduce_add_sync(kFull, s);
+  if (lane == 0) wsum[warp] = s;
+  __syncthreads();
+  uint32_t before = 0;  // sample entries in the warps' blocks before this one
+  for (int w = 0; w < warp; ++w) before += wsum[w];
   const int rs[2] = {r_hi, r_lo};
 #pragma unroll
   for (int q = 0; q < 2; ++q) {
     const int r = rs[q];
-    if (r >= 1 && r <= kWSamples && excl < static_cast<uint32_t>(r) &&
-        static_cast<uint32_t>(r) <= excl + tsum) {
-      uint32_t run = excl;
-#pragma unroll
-      for (int g = 0; g < G; ++g) {
-        if (run + c[g] >= static_cast<uint32_t>(r)) {
-          pick[q] = kWSBins - 1 - (tid * G + g);
+    if (r >= 1 && r <= kWSamples && before < static_cast<uint32_t>(r) &&
+        static_cast<uint32_t>(r) <= before + s) {
+      // this warp's block holds the r-th largest: 32 bins at a time
+      uint32_t run = before;
+      for (int j = 0; j < J; ++j) {
+        const uint32_t incl = run + warp_inclusive_scan(v[j], lane);
+        const bool hit = incl >= static_cast<uint32_t>(r) && incl - v[j] < static_cast<uint32_t>(r);
+        const unsigned who = __ballot_sync(kFull, hit);
+        if (who) {
+          if (lane == __ffs(who) - 1) {
+            pick[q] = kWSBins - 1 - (1024 * warp + 32 * j + lane);
+            if (q == 1) s_ge = incl;
+          }
           break;
         }
-        run += c[g];
+        run = __shfl_sync(kFull, incl, 31);
       }
     }
   }
@@ -564,8 +604,8 @@ __global__ void __launch_bounds__(1024) w_sample(const float* xr, const float* a
   if (tid == 0) {
     uint32_t t_lo = 0, t_hi = kWNoSure;
     if (pick[0] >= 0 && pick[0] < kWSBins - 1)
-      t_hi = static_cast<uint32_t>(base + ((pick[0] + 1) << kWSShift));
-    if (pick[1] > 0) t_lo = static_cast<uint32_t>(base + (pick[1] << kWSShift));
+      t_hi = min(static_cast<uint32_t>(pick[0] + 1) << kWSShift, kWNoSure);
+    if (pick[1] > 0) t_lo = static_cast<uint32_t>(pick[1]) << kWSShift;
     if (t_lo > t_hi) t_lo = t_hi;
     // the band histogram spans [t_lo, t_hi), or, with nothing sure, up to one
     // octave above the sample's largest magnitude (larger keys share the top bin)
@@ -579,6 +619,9 @@ __global__ void __launch_bounds__(1024) w_sample(const float* xr, const float* a
     meta->ncand2 = 0;
     meta->bin2 = 0;
     meta->band = 1;
+    const float est = static_cast<float>(pick[1] > 0 ? s_ge : kWSamples) *
+                      (static_cast<float>(L) / static_cast<float>(kWSamples));
+    meta->lmode = list_ok && pick[1] > 0 && est * 1.25f + 65536.0f <= static_cast<float>(bcap);
   }
 }
 
@@ -614,25 +657,25 @@ __global__ void __launch_bounds__(kGT) w_pass1(const float* xr, float* ar, int64
                                                int64_t nchunks, int aligned, GridMeta* meta,
                                                uint32_t* cgt, uint32_t* ceq, int* bkey,
                                                uint32_t* bidx, uint32_t rcap, uint32_t* nbc,
-                                               uint32_t* fhist, uint32_t spin_limit,
-                                               unsigned* status) {
+                                               uint32_t* seg, uint32_t* segn, uint32_t* fhist,
+                                               uint32_t spin_limit, unsigned* status) {
   pdl_begin();
   constexpr int NW = kGT / 32;
   extern __shared__ __align__(16) float wbuf[];  // 2 x kCH
   __shared__ uint32_t fh[kFBins];
   __shared__ uint32_t rs[2][NW];  // sure entries per warp, by buffer
-  __shared__ uint32_t s_count, s_fail;
+  __shared__ uint32_t wl[NW];     // listed entries per warp of the current chunk
+  __shared__ uint32_t s_fail;
   __shared__ uint64_t bars[2][NW];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   if (!meta->band || meta->resolved) return;
   const uint32_t t_lo = meta->t_lo, t_hi = meta->t_hi;
   const int fsh = meta->fsh;
+  const bool lmode = meta->lmode != 0;
   const float f_lo = __uint_as_float(t_lo), f_hi = __uint_as_float(t_hi);
   for (int i = tid; i < kFBins; i += kGT) fh[i] = 0;
-  if (tid == 0) {
-    s_count = 0;
-    s_fail = 0;
-  }
+  if (tid == 0) s_fail = 0;
+  uint32_t cnt = 0;  // entries this CTA listed (the same in every thread)
   if (aligned && warp == 0 && lane < NW) {
     mbar_init(&bars[0][lane], 1);
     mbar_init(&bars[1][lane], 1);
@@ -656,7 +699,7 @@ __global__ void __launch_bounds__(kGT) w_pass1(const float* xr, float* ar, int64
       uint32_t s = 0;
 #pragma unroll
       for (int w = 0; w < H; ++w) s += rs[bb][h * H + w];
-      cgt[wc] = s;
+      cgt[wc] = lmode ? 0u : s;  // list mode: the sure entries are counted from the list
       ceq[wc] = 0;
     }
   };
@@ -723,24 +766,38 @@ __global__ void __launch_bounds__(kGT) w_pass1(const float* xr, float* ar, int64
       hw = __funnelshift_l(hw, hw, rot) & vmask;
       gw = __funnelshift_l(gw, gw, rot) & vmask;
     }
+    // the listed entries (the band; list mode: every entry >= t_lo) of this chunk
+    // as one segment of the CTA's region, in index order
     const uint32_t bw = gw & ~hw;
-    const uint32_t nbw = __popc(bw);
-    const uint32_t bi = warp_inclusive_scan(nbw, lane);
-    const uint32_t wtot = __shfl_sync(kFull, bi, 31);
-    uint32_t wb = 0;
-    if (lane == 0 && wtot) wb = atomicAdd(&s_count, wtot);
-    wb = __shfl_sync(kFull, wb, 0);
-    uint32_t pos = wb + bi - nbw;
-    uint32_t w = bw;
+    const uint32_t lw = lmode ? gw : bw;
+    const uint32_t nlw = __popc(lw);
+    const uint32_t bi = warp_inclusive_scan(nlw, lane);
+    if (lane == 31) wl[warp] = bi;
+    __syncthreads();
+    uint32_t wb = 0, ctot = 0;
+#pragma unroll
+    for (int w2 = 0; w2 < NW; ++w2) {
+      wb += w2 < warp ? wl[w2] : 0u;
+      ctot += wl[w2];
+    }
+    if (tid == 0) {
+      seg[c] = cnt;
+      segn[c] = ctot;
+    }
+    uint32_t pos = cnt + wb + bi - nlw;
+    cnt += ctot;
+    uint32_t w = lw;
     while (w) {
       const int j = __ffs(w) - 1;
       w &= w - 1;
       const int e = e0 + j;
-      const int key = mag_key(cb[e]);
-      atomicAdd(&fh[min(static_cast<uint32_t>(key - static_cast<int>(t_lo)) >> fsh, kFBins - 1u)],
-                1u);
+      const int bits = __float_as_int(cb[e]);
+      if ((bw >> j) & 1u)
+        atomicAdd(&fh[min(static_cast<uint32_t>((bits & 0x7fffffff) - static_cast<int>(t_lo)) >> fsh,
+                          kFBins - 1u)],
+                  1u);
       if (pos < rcap) {
-        bkey[rbase + pos] = key;
+        bkey[rbase + pos] = bits;
         bidx[rbase + pos] = static_cast<uint32_t>(c0 + e);
       }
       ++pos;
@@ -754,7 +811,6 @@ __global__ void __launch_bounds__(kGT) w_pass1(const float* xr, float* ar, int64
   if (lane == 0 && sure_w) atomicAdd(&meta->sure, sure_w);
   if (tid == 0) {
     if (prev >= 0) put_sure(prev, b ^ 1);
-    const uint32_t cnt = s_count;
     nbc[blockIdx.x] = min(cnt, rcap);
     if (cnt) atomicAdd(&meta->nband, cnt);
     // a full region, or a timed-out copy: the multi-pass path takes over
@@ -771,7 +827,8 @@ __global__ void __launch_bounds__(32) w_pick1(GridMeta* meta, const uint32_t* fh
   const GridMeta m = *meta;
   if (!m.band || m.resolved) return;
   const int lane = threadIdx.x & 31;
-  if (!(static_cast<int64_t>(m.sure) < k && k <= static_cast<int64_t>(m.sure) + m.nband)) {
+  const int64_t ge = m.lmode ? static_cast<int64_t>(m.nband) : static_cast<int64_t>(m.sure) + m.nband;
+  if (!(static_cast<int64_t>(m.sure) < k && k <= ge)) {
     if (lane == 0) meta->band = 0;  // the multi-pass path takes over
     return;
   }
@@ -779,11 +836,12 @@ __global__ void __launch_bounds__(32) w_pick1(GridMeta* meta, const uint32_t* fh
   const BinPick p = warp_pick_bin(fhist, kr, lane);
   if (lane == 0) {
     const int bl = static_cast<int>(m.t_lo) + (p.bin << m.fsh);
-    // the top bin also takes every larger key
-    const int bh = p.bin == kFBins - 1
-                       ? 0x7fffffff
-                       : static_cast<int>(min(static_cast<uint32_t>(bl) + ((1u << m.fsh) - 1u),
-                                              0x7fffffffu));
+    // the top bin also takes every larger band key (none reaches t_hi; the
+    // list of list mode holds the sure entries too)
+    int bh = p.bin == kFBins - 1
+                 ? 0x7fffffff
+                 : static_cast<int>(min(static_cast<uint32_t>(bl) + ((1u << m.fsh) - 1u), 0x7fffffffu));
+    if (m.t_hi != kWNoSure) bh = min(bh, static_cast<int>(m.t_hi) - 1);
     const uint32_t kr2 = kr - p.above;
     if (p.count == kr2) {  // the bin is kept whole
       meta->T = bl - 1;
@@ -815,7 +873,7 @@ __global__ void __launch_bounds__(256) w_bin2(GridMeta* meta, const int* bkey, c
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
       const uint32_t i = i0 + 32u * q + lane;
-      key[q] = i < nr ? rk[i] : -1;
+      key[q] = i < nr ? (rk[i] & 0x7fffffff) : -1;
     }
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
@@ -917,7 +975,7 @@ __global__ void __launch_bounds__(256) w_mark(const GridMeta* meta, const int* b
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
       const uint32_t i = i0 + 32u * q + lane;
-      key[q] = i < nr ? bkey[rb + i] : -1;
+      key[q] = i < nr ? (bkey[rb + i] & 0x7fffffff) : -1;
       ch[q] = i < nr ? static_cast<uint32_t>(bidx[rb + i] / kWCH) : 0xffffffffu;
     }
 #pragma unroll
@@ -1009,6 +1067,7 @@ __global__ void __launch_bounds__(kWT) g_write3(const float* xr, float* ar, int6
   __shared__ uint32_t rg[NW], re[NW];
   __shared__ uint64_t bars[2][NW];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  if (meta->band && meta->lmode) return;  // g_wlist writes the payload from the list
   const int T = meta->T;
   const uint32_t need = meta->need;
   if (aligned && warp == 0 && lane < NW) {
@@ -1158,6 +1217,62 @@ __global__ void __launch_bounds__(kWT) g_write3(const float* xr, float* ar, int6
   }
 }
 
+// List mode: the payload from the list instead of a second read of the row.
+// Warp w takes pass-1 chunks c = w, w + W, ...; chunk c's entries (every entry
+// >= t_lo, in index order) are the segment of region c % G1 that pass 1
+// recorded.  Kept: above T, and ties while their rank among the row's ties is
+// below need; positions from the scanned per-write-chunk counts (a pass-1 chunk
+// is write chunks 2c and 2c + 1).  Error feedback: +0 into err at the kept
+// entries (err holds s); EF21: state + d there.
+template <int MODE>
+__global__ void __launch_bounds__(256) g_wlist(float* ar, int64_t nchunks, uint32_t g1,
+                                               uint32_t rcap, int64_t k, const GridMeta* meta,
+                                               const int* bkey, const uint32_t* bidx,
+                                               const uint32_t* seg, const uint32_t* segn,
+                                               const uint32_t* cgt, const uint32_t* ceq,
+                                               const uint32_t* tg, const uint32_t* te,
+                                               float* vals, int32_t* idx) {
+  pdl_begin();
+  if (!(meta->band && meta->lmode)) return;
+  const int T = meta->T;
+  const uint32_t need = meta->need;
+  const int lane = threadIdx.x & 31;
+  const unsigned lt = lanemask_lt();
+  const int64_t nw = static_cast<int64_t>(gridDim.x) * (blockDim.x / 32);
+  for (int64_t c = static_cast<int64_t>(blockIdx.x) * (blockDim.x / 32) + (threadIdx.x >> 5);
+       c < nchunks; c += nw) {
+    const int64_t wc = 2 * c;
+    const uint32_t gb = cgt[wc] + tg[wc >> 10], eb = ceq[wc] + te[wc >> 10];
+    uint64_t pos = static_cast<uint64_t>(gb) + min(eb, need);
+    uint32_t eq_seen = eb;
+    const size_t rb = static_cast<size_t>(c % g1) * rcap + seg[c];
+    const uint32_t n = segn[c];
+    for (uint32_t i0 = 0; i0 < n; i0 += 32) {
+      const uint32_t i = i0 + lane;
+      const bool in = i < n;
+      const int bits = in ? bkey[rb + i] : 0;
+      const uint32_t col = in ? bidx[rb + i] : 0u;
+      const int key = bits & 0x7fffffff;
+      const bool eq = in && key == T;
+      const unsigned be = __ballot_sync(kFull, eq);
+      const bool kp = (in && key > T) || (eq && eq_seen + __popc(be & lt) < need);
+      eq_seen += __popc(be);
+      const unsigned bk = __ballot_sync(kFull, kp);
+      if (kp) {
+        const uint64_t p = pos + __popc(bk & lt);
+        const float v = __int_as_float(bits);
+        if (p < static_cast<uint64_t>(k)) {
+          vals[p] = v;
+          idx[p] = static_cast<int32_t>(col);
+        }
+        if (MODE == kEF) ar[col] = 0.0f;                   // err' = s - C(s): +0 where sent
+        if (MODE == kDelta) ar[col] = fadd(ar[col], v);   // g' = g + d where sent
+      }
+      pos += __popc(bk);
+    }
+  }
+}
+
 // Persistent grids: the CTAs that fit on the GPU (and no more than the band
 // list has regions).
 template <class K>
@@ -1174,7 +1289,7 @@ cudaError_t run_grid(const TopkGridArgs& a, int num_sms, cudaStream_t s) {
   const int64_t nwch = (L + kWCH - 1) / kWCH;
   const int nblk = static_cast<int>((nwch + 1023) / 1024);
   if (nchunks > 0x7fffffffLL) return cudaErrorInvalidValue;
-  const WsLayout w = layout(a.ws, L, nchunks);
+  const WsLayout w = layout(a.ws, L, a.k, nchunks);
   auto al16 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; };
   const int aligned = (L % 4 == 0) && al16(a.x) && (MODE == kPlain || al16(a.aux));
   constexpr int kP1Smem = 2 * kCH * 4;             // two chunk buffers
@@ -1187,6 +1302,8 @@ cudaError_t run_grid(const TopkGridArgs& a, int num_sms, cudaStream_t s) {
   const unsigned g1 = persistent_grid(p1, kGT, kP1Smem, num_sms, nchunks);
   const unsigned gw = persistent_grid(wr, kWT, kWSmem, num_sms, nwch);
   const uint32_t rcap = w.bcap / g1;  // band-list region of one pass-1 CTA
+  // the list-mode write: a warp per pass-1 chunk
+  const unsigned gl = static_cast<unsigned>(min64((nchunks + 7) / 8, static_cast<int64_t>(num_sms) * 8));
   // the multi-pass kernels: a fixed grid striding over the chunks
   const unsigned gm = static_cast<unsigned>(min64(nwch, static_cast<int64_t>(num_sms) * 8));
   for (int64_t r = 0; r < a.rows; ++r) {
@@ -1194,17 +1311,18 @@ cudaError_t run_grid(const TopkGridArgs& a, int num_sms, cudaStream_t s) {
     float* ar = (MODE != kPlain) ? a.aux + r * L : nullptr;
     float* vr = a.vals + r * a.k;
     int32_t* ir = a.idx + r * a.k;
-    g_init<<<1, 256, 0, s>>>(w.meta, w.hist, nchunks);
-    g_sample<MODE><<<1, kGT, 0, s>>>(xr, ar, L, a.k, w.meta);
+    g_init<<<1, 1024, 0, s>>>(w.meta, w.hist, w.shist, w.fhist, nchunks, L, a.k);
     // the band path
-    w_sample<MODE><<<1, 1024, 0, s>>>(xr, ar, L, a.k, w.meta, w.fhist);
+    w_sample<MODE><<<kWSCtas, 1024, 0, s>>>(xr, ar, L, w.meta, w.shist);
+    w_spick<<<1, 1024, 0, s>>>(L, a.k, w.meta, w.shist, list_eligible(L, a.k) ? 1 : 0, w.bcap);
     p1<<<g1, kGT, kP1Smem, s>>>(xr, ar, L, nchunks, aligned, w.meta, w.cgt, w.ceq, w.bkey, w.bidx,
-                                rcap, w.nbc, w.fhist, a.spin_limit, a.status);
+                                rcap, w.nbc, w.seg, w.segn, w.fhist, a.spin_limit, a.status);
     w_pick1<<<1, 32, 0, s>>>(w.meta, w.fhist, a.k);
     w_bin2<<<g1, 256, 0, s>>>(w.meta, w.bkey, w.nbc, rcap, w.c2key);
     w_select2<<<1, 1024, 0, s>>>(w.meta, w.c2key);
     w_mark<<<g1, 256, 0, s>>>(w.meta, w.bkey, w.bidx, w.nbc, rcap, w.cgt, w.ceq);
     // the multi-pass path (each kernel returns at once when the band path resolved)
+    g_sample<MODE><<<1, kGT, 0, s>>>(xr, ar, L, a.k, w.meta);
     g_hist<MODE><<<gm, kGT, 0, s>>>(xr, ar, L, w.meta, w.hist, 1);
     g_pick<<<1, kGT, 0, s>>>(w.meta, w.hist);
     for (int i = 0; i < kMaxRounds; ++i) {
@@ -1218,6 +1336,8 @@ cudaError_t run_grid(const TopkGridArgs& a, int num_sms, cudaStream_t s) {
     w_scan2<<<1, 1024, 0, s>>>(w.tg, w.te, nblk);
     wr<<<gw, kWT, kWSmem, s>>>(xr, ar, L, nwch, a.k, aligned, w.meta, w.cgt, w.ceq, w.tg, w.te,
                                vr, ir, a.spin_limit, a.status);
+    g_wlist<MODE><<<gl, 256, 0, s>>>(ar, nchunks, g1, rcap, a.k, w.meta, w.bkey, w.bidx, w.seg,
+                                     w.segn, w.cgt, w.ceq, w.tg, w.te, vr, ir);
     const cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
@@ -1228,8 +1348,7 @@ cudaError_t run_grid(const TopkGridArgs& a, int num_sms, cudaStream_t s) {
 
 size_t topk_grid_workspace_bytes(int64_t rows, int64_t L, int64_t k) {
   (void)rows;
-  (void)k;
-  return ws_bytes_for(L);
+  return ws_bytes_for(L, k);
 }
 
 cudaError_t launch_topk_grid(int mode, const TopkGridArgs& a, int num_sms, cudaStream_t s) {
