@@ -239,7 +239,10 @@ mpc_status mpc_quant_decompress(const uint32_t* codes, const float* scale,
  *   bits, mode as mpc_quant_compress; codes, scale, minv out as there.
  *   ws         device workspace of mpc_aqsgd_quant_workspace_bytes() bytes,
  *              8-byte aligned (always needed: it holds d).
- * Three launches (d, the quantiser, the buffer update), stream-ordered. */
+ * One launch for 2/4/8-bit codes on rows of up to 4096 entries (d formed,
+ * quantised and the buffer updated in the same pass; the workspace is then
+ * unused); otherwise three (d, the quantiser, the buffer update),
+ * stream-ordered. */
 size_t mpc_aqsgd_quant_workspace_bytes(int64_t n_ids, int64_t rows_per_sample,
                                        int64_t row_len, int bits);
 mpc_status mpc_aqsgd_quant_compress(const float* x, float* buf, int64_t num_samples,

@@ -524,6 +524,31 @@ mpc_status mpc_aqsgd_quant_compress(const float* x, float* buf, int64_t num_samp
   Device d;
   MPC_TRY(current_device(&d));
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  // one pass where the shape allows it (2/4/8-bit codes, rows of up to 4096)
+  if (mpc::quant_workspace_bytes(rows, row_len, bits) == 0) {
+    mpc::QuantArgs a = {};
+    a.x = x;
+    a.rows = rows;
+    a.L = row_len;
+    a.bits = bits;
+    a.stochastic = (mode == MPC_ROUND_STOCHASTIC);
+    a.seed = seed;
+    a.codes = codes;
+    a.scale = scale;
+    a.minv = minv;
+    a.W = static_cast<int64_t>(mpc_quant_codes_words(1, row_len, bits));
+    a.aligned = (row_len % 4 == 0) && aligned_to(x, 16) && aligned_to(buf, 16);
+    a.spin_limit = g_spin_limit.load();
+    a.status = d.status;
+    a.aq_buf = buf;
+    a.aq_ids = sample_ids;
+    a.aq_rps = rows_per_sample;
+    a.aq_num_samples = num_samples;
+    const cudaError_t f = mpc::launch_aqsgd_quant_fused(a, d.num_sms, s);
+    if (f == cudaSuccess) return ok();
+    if (f != cudaErrorNotSupported) return cuda_error(f, "aqsgd_quant launch");
+  }
+  // else: d into the workspace, the quantiser on it, then the buffer update
   float* delta = static_cast<float*>(ws);
   const size_t dbytes = aqsgd_delta_bytes(rows, row_len);
   cudaError_t e = mpc::launch_aqsgd_delta(x, buf, sample_ids, n_ids, rows_per_sample, row_len,

@@ -2,9 +2,12 @@
 // activations of each training sample is sent, here compressed by the min-max
 // quantiser of §2.2 as in the cited work):
 //   d = x - buf[id, r];  message = Quant(d);  buf[id, r] += Dequant(message).
-// The abi runs: aqsgd_delta_kernel (d into a workspace, one row per logical
-// row i * rows_per_sample + r), the quantiser on d, aqsgd_dequant_add_kernel
-// (also the receiver's update of its copy of the buffer).  All HBM-bound.
+// For 2/4/8-bit codes on rows of up to 4096 entries the sender runs in one pass
+// (aqsgd_quant_fused_kernel, quant.cu).  Otherwise the abi runs:
+// aqsgd_delta_kernel (d into a workspace, one row per logical row
+// i * rows_per_sample + r), the quantiser on d, aqsgd_dequant_add_kernel.  The
+// receiver's update of its copy of the buffer is aqsgd_dequant_add_kernel.
+// All HBM-bound.
 #include <cstdint>
 
 #include "common.cuh"

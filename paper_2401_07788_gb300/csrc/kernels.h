@@ -98,8 +98,18 @@ struct QuantArgs {
   void* ws;         // multi-pass path: [rows] x {min key, max key}
   uint32_t spin_limit;
   unsigned* status;
+  // quantised AQ-SGD in one pass (aq_buf != nullptr): the rows quantised are
+  // d = x - aq_buf[id, r] (id = aq_ids[row / aq_rps], r = row % aq_rps), and
+  // aq_buf[id, r] += dequant(codes) is written in the same pass
+  float* aq_buf = nullptr;
+  const int64_t* aq_ids = nullptr;
+  int64_t aq_rps = 1;
+  int64_t aq_num_samples = 0;
 };
 constexpr int64_t kQuantRowPathMaxLen = 65536;
+// Quantised AQ-SGD in one pass where the shape allows (2/4/8-bit codes, rows of
+// up to 4096 entries); cudaErrorNotSupported otherwise (nothing launched).
+cudaError_t launch_aqsgd_quant_fused(const QuantArgs& a, int num_sms, cudaStream_t s);
 size_t quant_workspace_bytes(int64_t rows, int64_t L, int bits);
 cudaError_t launch_quant_compress(const QuantArgs& a, int num_sms, cudaStream_t s);
 // Allocation-free variant: the min/max scratch is a static device array.

@@ -83,6 +83,7 @@ struct RowParams {
   float mn;
   float inv;
   float levels;
+  float scale;  // (mx - mn) / levels, 0 for a degenerate row
   bool degenerate;
 };
 
@@ -95,7 +96,8 @@ __device__ __forceinline__ RowParams row_params(uint32_t kmin, uint32_t kmax, in
   const float range = fsub(mx, p.mn);
   p.inv = fdiv(p.levels, range);
   p.degenerate = (range == 0.0f) || isinf(range) || isinf(p.inv);
-  if (scale_out) *scale_out = p.degenerate ? 0.0f : fdiv(range, p.levels);
+  p.scale = p.degenerate ? 0.0f : fdiv(range, p.levels);
+  if (scale_out) *scale_out = p.scale;
   if (minv_out) *minv_out = p.mn;
   return p;
 }
@@ -128,6 +130,25 @@ __device__ __forceinline__ uint32_t pack4(const float xs[4], const RowParams& p,
     float q;
     if (SR) q = fminf(floorf(fadd(t, u[i])), p.levels);
     else q = rintf(t);
+    b[i] = __float_as_uint(fadd(q, 8388608.0f));
+  }
+  constexpr uint32_t S = 1u << BITS;
+  constexpr uint32_t kBias = 0x4b000000u * (1u + S + S * S + S * S * S);
+  return ((b[3] * S + b[2]) * S + b[1]) * S + b[0] - kBias;
+}
+
+// pack4 that also returns the 4 codes as floats (for the dequantised values).
+template <int BITS, bool SR>
+__device__ __forceinline__ uint32_t pack4q(const float xs[4], const RowParams& p, const float u[4],
+                                           float qf[4]) {
+  uint32_t b[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float t = fmul(fsub(xs[i], p.mn), p.inv);
+    float q;
+    if (SR) q = fminf(floorf(fadd(t, u[i])), p.levels);
+    else q = rintf(t);
+    qf[i] = q;
     b[i] = __float_as_uint(fadd(q, 8388608.0f));
   }
   constexpr uint32_t S = 1u << BITS;
@@ -389,6 +410,146 @@ __global__ void __launch_bounds__(128, 5) quant_rows4_kernel(const QuantArgs a) 
     }
     if (tid < a.W - data_words) cr[data_words + tid] = 0u;  // row padding
   }
+}
+
+// ---------------------------------------------------------------------------
+// Quantised AQ-SGD in one pass (rows of up to 4096 entries, 2/4/8-bit codes)
+// ---------------------------------------------------------------------------
+// NT threads per row (one warp up to 1024 entries, four warps up to 4096),
+// thread t holding the groups q = NT v + t (v < NV): d = x - buf[id, r] formed
+// as the groups load, the row's extrema of d, its codes, and buf[id, r] +=
+// minv + code * scale written back in the same pass (the receiver's update,
+// the same arithmetic).  A row whose sample id is out of range is skipped and
+// reported.
+template <int BITS, bool SR, int NT, int NV>
+__global__ void __launch_bounds__(NT == 32 ? 256 : NT) aqsgd_quant_fused_kernel(const QuantArgs a) {
+  pdl_begin();
+  constexpr int RPC = NT == 32 ? 8 : 1;  // rows in flight per CTA (a warp each, or the CTA)
+  constexpr int NWR = NT / 32;           // warps of a row
+  __shared__ uint32_t red[2][2][NWR > 1 ? NWR : 1];
+  const int tid = threadIdx.x % NT, lane = threadIdx.x & 31, wr = tid >> 5;
+  const int slot = threadIdx.x / NT;  // this thread's row slot in the CTA
+  const int64_t L = a.L;
+  const int64_t data_words = (L * BITS + 31) / 32;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * RPC;
+  int it = 0;
+  for (int64_t row = static_cast<int64_t>(blockIdx.x) * RPC + slot; row < a.rows; row += stride, ++it) {
+    const int64_t sid = a.aq_ids[row / a.aq_rps];
+    const bool ok = sid >= 0 && sid < a.aq_num_samples;
+    if (!ok && tid == 0) set_status(a.status, STATUS_BAD_SAMPLE);
+    float* br = ok ? a.aq_buf + (sid * a.aq_rps + row % a.aq_rps) * L : nullptr;
+    const float* xr = a.x + row * L;
+    float4 d[NV], g[NV];
+    uint32_t kmin = 0xffffffffu, kmax = 0u;
+#pragma unroll
+    for (int v = 0; v < NV; ++v) {
+      const int64_t e0 = 4 * (v * NT + tid);
+      float xs[4] = {0.f, 0.f, 0.f, 0.f}, gs[4] = {0.f, 0.f, 0.f, 0.f};
+      if (ok) {
+        if (a.aligned && e0 + 4 <= L) {
+          const float4 xv = *reinterpret_cast<const float4*>(xr + e0);
+          const float4 gv = *reinterpret_cast<const float4*>(br + e0);
+          xs[0] = xv.x; xs[1] = xv.y; xs[2] = xv.z; xs[3] = xv.w;
+          gs[0] = gv.x; gs[1] = gv.y; gs[2] = gv.z; gs[3] = gv.w;
+        } else {
+#pragma unroll
+          for (int i = 0; i < 4; ++i)
+            if (e0 + i < L) {
+              xs[i] = xr[e0 + i];
+              gs[i] = br[e0 + i];
+            }
+        }
+      }
+      d[v] = make_float4(fsub(xs[0], gs[0]), fsub(xs[1], gs[1]), fsub(xs[2], gs[2]), fsub(xs[3], gs[3]));
+      g[v] = make_float4(gs[0], gs[1], gs[2], gs[3]);
+      if (e0 + 4 <= L) {
+        fold_keys4(d[v], kmin, kmax);
+      } else {
+        const float ds[4] = {d[v].x, d[v].y, d[v].z, d[v].w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+          if (e0 + i < L) {
+            const uint32_t okk = ord_key(ds[i]);
+            kmin = min(kmin, okk);
+            kmax = max(kmax, okk);
+          }
+      }
+    }
+    kmin = __reduce_min_sync(kFull, kmin);
+    kmax = __reduce_max_sync(kFull, kmax);
+    if (NWR > 1) {
+      const int sl = it & 1;
+      if (lane == 0) {
+        red[sl][0][wr] = kmin;
+        red[sl][1][wr] = kmax;
+      }
+      __syncthreads();
+#pragma unroll
+      for (int w = 0; w < NWR; ++w) {
+        kmin = min(kmin, red[sl][0][w]);
+        kmax = max(kmax, red[sl][1][w]);
+      }
+    }
+    if (!ok) continue;  // uniform over the row's threads (after the CTA barrier)
+    const RowParams p = row_params(kmin, kmax, BITS, tid == 0 ? a.scale + row : nullptr,
+                                   tid == 0 ? a.minv + row : nullptr);
+    uint32_t* cr = a.codes + row * a.W;
+#pragma unroll
+    for (int v = 0; v < NV; ++v) {
+      const int64_t e0 = 4 * (v * NT + tid);
+      const float xs[4] = {d[v].x, d[v].y, d[v].z, d[v].w};
+      float u[4] = {0.f, 0.f, 0.f, 0.f};
+      if (SR) uniform4(a.seed, static_cast<uint64_t>(row * L + e0), u);
+      float qf[4] = {0.f, 0.f, 0.f, 0.f};
+      uint32_t piece = 0;
+      if (!p.degenerate) {
+        if (e0 + 4 <= L) {
+          piece = pack4q<BITS, SR>(xs, p, u, qf);
+        } else {
+#pragma unroll
+          for (int i = 0; i < 4; ++i)
+            if (e0 + i < L) {
+              const uint32_t c = code_of<SR>(xs[i], p, u[i]);
+              qf[i] = static_cast<float>(c);
+              piece |= c << (BITS * i);
+            }
+        }
+      }
+      const bool store = assemble_word<BITS>(piece, lane);
+      const int64_t w = e0 * BITS / 32;
+      if (store && w < data_words) cr[w] = piece;
+      // the buffer: state + minv + code * scale
+      const float gs[4] = {g[v].x, g[v].y, g[v].z, g[v].w};
+      float nb[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) nb[i] = fadd(gs[i], fadd(p.mn, fmul(qf[i], p.scale)));
+      if (a.aligned && e0 + 4 <= L) {
+        *reinterpret_cast<float4*>(br + e0) = make_float4(nb[0], nb[1], nb[2], nb[3]);
+      } else {
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+          if (e0 + i < L) br[e0 + i] = nb[i];
+      }
+    }
+    if (tid < a.W - data_words) cr[data_words + tid] = 0u;  // row padding
+  }
+}
+
+template <int BITS, bool SR>
+cudaError_t run_aqsgd_fused(const QuantArgs& a, int num_sms, cudaStream_t s) {
+  auto go = [&](auto kernel, int threads, int rpc) {
+    const int occ = resident_blocks(kernel, threads, 0);
+    const int64_t want = (a.rows + rpc - 1) / rpc;
+    const int64_t cap = static_cast<int64_t>(num_sms) * (occ > 0 ? occ : 1);
+    return launch_kernel(kernel, dim3(static_cast<unsigned>(want < cap ? want : cap)), dim3(threads),
+                         0, s, 0u, a);
+  };
+  const int64_t L = a.L;
+  if (L <= 256) return go(aqsgd_quant_fused_kernel<BITS, SR, 32, 2>, 256, 8);
+  if (L <= 512) return go(aqsgd_quant_fused_kernel<BITS, SR, 32, 4>, 256, 8);
+  if (L <= 1024) return go(aqsgd_quant_fused_kernel<BITS, SR, 32, 8>, 256, 8);
+  if (L <= 2048) return go(aqsgd_quant_fused_kernel<BITS, SR, 128, 4>, 128, 1);
+  return go(aqsgd_quant_fused_kernel<BITS, SR, 128, 8>, 128, 1);
 }
 
 // ---------------------------------------------------------------------------
@@ -930,6 +1091,20 @@ unsigned grid_for(int64_t work, int num_sms) {
 size_t quant_workspace_bytes(int64_t rows, int64_t L, int bits) {
   if (bits == 32 || L <= kQuantRowPathMaxLen) return 0;
   return static_cast<size_t>(rows) * 8u;
+}
+
+cudaError_t launch_aqsgd_quant_fused(const QuantArgs& a, int num_sms, cudaStream_t s) {
+  if (a.rows <= 0) return cudaSuccess;
+  if (a.aq_buf == nullptr || a.L > 4096 || a.ws != nullptr) return cudaErrorNotSupported;
+  switch (a.bits) {
+    case 2: return a.stochastic ? run_aqsgd_fused<2, true>(a, num_sms, s)
+                                : run_aqsgd_fused<2, false>(a, num_sms, s);
+    case 4: return a.stochastic ? run_aqsgd_fused<4, true>(a, num_sms, s)
+                                : run_aqsgd_fused<4, false>(a, num_sms, s);
+    case 8: return a.stochastic ? run_aqsgd_fused<8, true>(a, num_sms, s)
+                                : run_aqsgd_fused<8, false>(a, num_sms, s);
+    default: return cudaErrorNotSupported;
+  }
 }
 
 cudaError_t launch_quant_compress(const QuantArgs& a, int num_sms, cudaStream_t s) {

@@ -66,6 +66,15 @@ def test_aqsgd_quant_lengths(mpc, L):
     run_steps(mpc, S=9, rps=3, L=L, n=4, bits=4, stochastic=True, steps=2, seed=L % 977)
 
 
+@pytest.mark.parametrize("L", [1, 7, 128, 256, 300, 768, 1024, 1025, 2048, 2049, 3000, 4095, 4096])
+@pytest.mark.parametrize("bits,stochastic", [(2, False), (8, True), (4, False)])
+def test_aqsgd_quant_one_pass_shapes(mpc, L, bits, stochastic):
+    """The one-pass sender (2/4/8-bit codes, rows of up to 4096 entries: a warp per row,
+    four warps from 1025 on), ragged lengths included, against the oracle."""
+    run_steps(mpc, S=11, rps=3, L=L, n=5, bits=bits, stochastic=stochastic, steps=2,
+              seed=L + bits)
+
+
 def test_aqsgd_quant_cnn_boundary_shape(mpc):
     """The CNN stage boundary: 128 samples of [128, 16, 16] activations, one row per sample,
     drawn from a 512-sample set."""
