@@ -94,12 +94,23 @@ __global__ void __launch_bounds__(kDecThreads)
       const uint32_t n = static_cast<uint32_t>(nrows * k);  // <= kDT
       const uint32_t magic = static_cast<uint32_t>(0xffffffffu / static_cast<uint32_t>(k)) + 1u;
       const uint32_t Lu = static_cast<uint32_t>(L);
-#pragma unroll 4
-      for (uint32_t j = tid; j < n; j += kDecThreads) {
-        const uint32_t lr = k == 1 ? j : __umulhi(j, magic);
-        const int32_t col = idx[e0 + j];
-        const float v = vals[e0 + j];
-        if (col >= 0 && static_cast<uint32_t>(col) < Lu) tile[lr * Lu + col] = v;
+      // batches of kB entries a thread: all of a batch's loads in flight together
+      constexpr int kB = 8;
+      for (uint32_t j0 = tid; j0 < n; j0 += kB * kDecThreads) {
+        int32_t col[kB];
+        float v[kB];
+#pragma unroll
+        for (int b = 0; b < kB; ++b) {
+          const uint32_t j = j0 + b * kDecThreads;
+          col[b] = j < n ? idx[e0 + j] : -1;
+          v[b] = j < n ? vals[e0 + j] : 0.0f;
+        }
+#pragma unroll
+        for (int b = 0; b < kB; ++b) {
+          const uint32_t j = j0 + b * kDecThreads;
+          const uint32_t lr = k == 1 ? j : __umulhi(j, magic);
+          if (col[b] >= 0 && static_cast<uint32_t>(col[b]) < Lu) tile[lr * Lu + col[b]] = v[b];
+        }
       }
     } else {
       // a column tile of a long row: the row's next payload entries below c0 + ncols
