@@ -74,6 +74,10 @@ def parse_args():
     p.add_argument("--no-secondary", action="store_true",
                    help="skip the CNN-boundary step and the whole-tensor table")
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--profile-call", default="",
+                   help="for ncu captures: run only these calls of the sweep step (comma-separated "
+                        "names as in the per_op table, in order), warm-up and timed steps alike, "
+                        "and print one line saying what ran instead of the benchmark line")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cnn-steps", type=int, default=200)
     p.add_argument("--branches", type=int, default=6, choices=(1, 2, 3, 5, 6, 9),
@@ -327,6 +331,8 @@ def kernels_of(op: str, L_: int) -> list:
     if op == "quant":
         if L_ <= 2048:
             return ["quant_warp_kernel"]
+        if L_ <= 4096:
+            return ["quant_rows4_kernel"]
         if L_ <= ROW_PATH_MAX:
             return ["quant_cta_kernel"]
         return ["minmax_init_kernel", "quant_minmax_kernel", "quant_cta_kernel"]
@@ -446,6 +452,28 @@ class SweepStep:
                 events[j].record()
 
 
+def run_profile_calls(args, st, mpc, device):
+    """Only the named calls of the sweep step, in the given order, for warm-up + timed steps
+    (a profiler then picks the launches it wants); no timing is reported."""
+    by_name = {c.name: c for c in st.calls}
+    names = [s.strip() for s in args.profile_call.split(",") if s.strip()]
+    missing = [s for s in names if s not in by_name]
+    if missing:
+        raise SystemExit("unknown call(s): %s" % ", ".join(missing))
+    stream = torch.cuda.Stream(device)
+    with torch.cuda.stream(stream):
+        for s in range(max(1, args.warmup) + args.steps):
+            for n in names:
+                by_name[n].fn(st.xs[s % 2], st.y)
+    stream.synchronize()
+    status = mpc.mpc_get_status(stream)
+    if status != 0:
+        raise RuntimeError("device status %d: %s" % (status, mpc.mpc_last_error()))
+    print(json.dumps({"profile_call": names, "log2n": args.log2n,
+                      "runs": max(1, args.warmup) + args.steps,
+                      "launches_per_run": sum(len(by_name[n].kernels) for n in names)}), flush=True)
+
+
 def run_headline(args, rank, local, world):
     import paper_2401_07788_gb300 as mpc
     from paper_2401_07788_gb300 import synth
@@ -455,6 +483,9 @@ def run_headline(args, rank, local, world):
     init_dist(world, "nccl")
     mpc.lib()
     st = SweepStep(mpc, synth, device, args.log2n, rank % 10)
+    if args.profile_call:
+        run_profile_calls(args, st, mpc, device)
+        return
     n_calls = len(st.calls)
     stream = torch.cuda.Stream(device)
     with torch.cuda.stream(stream):
