@@ -46,6 +46,7 @@ __device__ int64_t warp_lower_bound(const int32_t* a, int64_t n, int64_t target,
 // of the row's ascending indices below the tile's end.  Persistent CTAs each
 // take a contiguous range of tiles and carry the payload position from tile to
 // tile, so only a CTA whose first tile starts inside a row searches for it.
+template <bool SHORT>
 __global__ void __launch_bounds__(kDecThreads)
     topk_decompress_tiles_kernel(const float* __restrict__ vals, const int32_t* __restrict__ idx,
                                  int64_t rows, int64_t L, int64_t k, float* __restrict__ y,
@@ -58,10 +59,41 @@ __global__ void __launch_bounds__(kDecThreads)
   const int64_t per = (ntiles + gridDim.x - 1) / gridDim.x;
   const int64_t t0 = static_cast<int64_t>(blockIdx.x) * per;
   const int64_t t1 = min64(ntiles, t0 + per);
+  constexpr int kB = 8;  // short rows: payload entries a thread per batch
+  constexpr int kU = 4;  // long rows: payload entries a thread per round
+  const uint32_t Lu = static_cast<uint32_t>(L);
+  const uint32_t magic = static_cast<uint32_t>(0xffffffffu / static_cast<uint32_t>(k)) + 1u;
+  // Short rows: the first batch of a tile's payload is loaded while the previous
+  // tile is copied out (pcol, pv: those loads).
+  int32_t pcol[kB];
+  float pv[kB];
+  auto fetch_short = [&](int64_t t, uint32_t j0, int32_t* col, float* v) {
+    const int64_t r0 = t * rpt;
+    const uint32_t n = static_cast<uint32_t>(min64(rpt, rows - r0) * k);
+    const int64_t e0 = r0 * k;
+#pragma unroll
+    for (int b = 0; b < kB; ++b) {
+      const uint32_t j = j0 + b * kDecThreads;
+      col[b] = j < n ? idx[e0 + j] : -1;
+      v[b] = j < n ? vals[e0 + j] : 0.0f;
+    }
+  };
+  // long rows: entries pos .. of row r0, columns relative to c0
+  auto fetch_long = [&](int64_t r0, int64_t c0, int64_t pos, int64_t* col, float* v) {
+    const int32_t* ir = idx + r0 * k;
+    const float* vr = vals + r0 * k;
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      const int64_t e = pos + u * kDecThreads + tid;
+      col[u] = e < k ? static_cast<int64_t>(ir[e]) - c0 : -1;
+      v[u] = e < k ? vr[e] : 0.0f;
+    }
+  };
   int64_t pos = 0;  // payload entry of the row where the current tile's entries start
+  bool have = false;  // the current tile's first batch is in pcol, pv
   for (int64_t t = t0; t < t1; ++t) {
     int64_t r0, nrows, c0, ncols;
-    if (tpr == 1) {
+    if (SHORT) {
       r0 = t * rpt;
       nrows = min64(rpt, rows - r0);
       c0 = 0;
@@ -86,24 +118,23 @@ __global__ void __launch_bounds__(kDecThreads)
     for (int64_t i = tid; i < (cells + 3) / 4; i += kDecThreads)
       reinterpret_cast<float4*>(tile)[i] = make_float4(0.f, 0.f, 0.f, 0.f);
     __syncthreads();
-    if (tpr == 1) {
+    if (SHORT) {
       // whole rows: the payload range of rows r0 .. r0 + nrows - 1; the local row of
       // entry j is j / k, taken as the high half of j * ceil(2^32 / k) (exact for j and
-      // k up to 2^13; k = 1 needs no division)
-      const int64_t e0 = r0 * k;
+      // k up to 2^13; k = 1 needs no division).  Batches of kB entries a thread, all of
+      // a batch's loads in flight together.
       const uint32_t n = static_cast<uint32_t>(nrows * k);  // <= kDT
-      const uint32_t magic = static_cast<uint32_t>(0xffffffffu / static_cast<uint32_t>(k)) + 1u;
-      const uint32_t Lu = static_cast<uint32_t>(L);
-      // batches of kB entries a thread: all of a batch's loads in flight together
-      constexpr int kB = 8;
       for (uint32_t j0 = tid; j0 < n; j0 += kB * kDecThreads) {
         int32_t col[kB];
         float v[kB];
+        if (have && j0 == static_cast<uint32_t>(tid)) {
 #pragma unroll
-        for (int b = 0; b < kB; ++b) {
-          const uint32_t j = j0 + b * kDecThreads;
-          col[b] = j < n ? idx[e0 + j] : -1;
-          v[b] = j < n ? vals[e0 + j] : 0.0f;
+          for (int b = 0; b < kB; ++b) {
+            col[b] = pcol[b];
+            v[b] = pv[b];
+          }
+        } else {
+          fetch_short(t, j0, col, v);
         }
 #pragma unroll
         for (int b = 0; b < kB; ++b) {
@@ -115,25 +146,17 @@ __global__ void __launch_bounds__(kDecThreads)
     } else {
       // a column tile of a long row: the row's next payload entries below c0 + ncols
       // (ascending indices, so they are a prefix of the entries read from pos on)
-      const int32_t* ir = idx + r0 * k;
-      const float* vr = vals + r0 * k;
       for (int it = 0;; ++it) {
-        constexpr int kU = 4;
         int64_t col[kU];
         float v[kU];
-        bool in[kU];
-#pragma unroll
-        for (int u = 0; u < kU; ++u) {
-          const int64_t e = pos + u * kDecThreads + tid;
-          col[u] = e < k ? static_cast<int64_t>(ir[e]) - c0 : -1;
-          v[u] = e < k ? vr[e] : 0.0f;
-          in[u] = e < k && col[u] < ncols;
-        }
+        fetch_long(r0, c0, pos, col, v);
         int cnt = 0;
 #pragma unroll
         for (int u = 0; u < kU; ++u) {
-          if (in[u] && col[u] >= 0) tile[col[u]] = v[u];
-          cnt += __popc(__ballot_sync(kFull, in[u]));
+          const int64_t e = pos + u * kDecThreads + tid;
+          const bool in = e < k && col[u] < ncols;
+          if (in && col[u] >= 0) tile[col[u]] = v[u];
+          cnt += __popc(__ballot_sync(kFull, in));
         }
         if (lane == 0) s_cnt[it & 1][warp] = cnt;
         __syncthreads();
@@ -145,6 +168,14 @@ __global__ void __launch_bounds__(kDecThreads)
       }
     }
     __syncthreads();
+    // short rows: the next tile's first payload loads go out before this tile's copy
+    // (for long rows this measured slower: the extra registers cost more occupancy
+    // than the overlap gains)
+    have = false;
+    if (SHORT && t + 1 < t1) {
+      fetch_short(t + 1, tid, pcol, pv);
+      have = true;
+    }
     float* dst = y + r0 * L + c0;
     if (aligned) {
       const int64_t n4 = cells / 4;
@@ -253,7 +284,7 @@ cudaError_t launch_topk_decompress(const float* vals, const int32_t* idx, int64_
     ntiles = rows * tpr;
   }
   constexpr int smem = kDT * 4;
-  auto kernel = topk_decompress_tiles_kernel;
+  auto kernel = tpr == 1 ? topk_decompress_tiles_kernel<true> : topk_decompress_tiles_kernel<false>;
   cudaError_t err = ensure_dynamic_smem(kernel, smem);
   if (err != cudaSuccess) return err;
   const int occ = resident_blocks(kernel, kDecThreads, smem);
