@@ -5,7 +5,7 @@
 //
 // Two kernels share the selection of select.cuh.  Both read x (and the error
 // or state row) from HBM once, keep the ranked values (x, x + err or
-// x - state) in shared memory, write the payload once, write err once (error
+// x - state) on chip, write the payload once, write err once (error
 // feedback) or the state at the kept entries only (EF21 / AQ-SGD).
 //
 //  * topk_cta_kernel: rows longer than 1024 entries.  One thread-block cluster
@@ -24,6 +24,12 @@
 //  * topk_warp_kernel: one warp per row for rows of at most 1024 entries,
 //    persistent over rows; each warp double-buffers its rows with its own bulk
 //    copies and mbarriers, so the next row loads while this one is selected.
+//    The row stays in registers (plain TopK: the keys; the fused variants: the
+//    ranked values), the selection's histogram and candidates in the warp's
+//    scratch.  The write marks the kept entries, places each group of 128 by one
+//    packed warp scan, stages the kept (value, column) pairs of two groups at a
+//    time in the scratch with predicated stores, and copies them out with
+//    coalesced stores.
 //
 // FULL instantiations drop the per-entry end-of-slice checks; they run when
 // every 4-entry slot a thread processes lies inside the slice.
@@ -880,11 +886,41 @@ __global__ void __launch_bounds__(NT, (NT == 128 ? 6 : NT == 256 ? 4 : NT == 512
 // Warp-per-row kernel (rows of at most 128 * NVW entries, WPC warps per CTA)
 // ---------------------------------------------------------------------------
 struct WarpShared {
-  uint32_t hist[kRoundBins + 64];  // + 32 zero spill counters, + 32 past-the-end ones
-  int lkey[kLCAPW];
+  union {
+    struct {
+      uint32_t hist[kRoundBins + 64];  // + 32 zero spill counters, + 32 past-the-end ones
+      int lkey[kLCAPW];
+    } sel;
+    uint2 out[(kRoundBins + 64 + kLCAPW) / 2];  // the write stage: (value, column) pairs
+  } u;
   uint32_t lcount;
   uint64_t bar[2];
 };
+
+// w |= bit when key > t: one compare and one predicated OR.
+__device__ __forceinline__ void or_if_key_gt(uint32_t& w, int key, int t, uint32_t bit) {
+  asm("{\n .reg .pred p;\n setp.gt.s32 p, %1, %2;\n @p or.b32 %0, %0, %3;\n}" : "+r"(w) : "r"(key), "r"(t), "r"(bit));
+}
+
+// Appends the kept ones of four entries (bits of nib) to a warp's write stage
+// as (value bits, column) pairs from shared byte address `at` on, and advances
+// it: predicated stores, no branch.
+__device__ __forceinline__ void stage_kept4(uint32_t nib, uint32_t& at, float4 v, int col0) {
+  asm volatile(
+      "{\n .reg .pred p;\n .reg .b32 t;\n"
+      " and.b32 t, %1, 1;\n setp.ne.b32 p, t, 0;\n"
+      " @p st.shared.v2.b32 [%0], {%2, %6};\n @p add.u32 %0, %0, 8;\n"
+      " and.b32 t, %1, 2;\n setp.ne.b32 p, t, 0;\n"
+      " @p st.shared.v2.b32 [%0], {%3, %7};\n @p add.u32 %0, %0, 8;\n"
+      " and.b32 t, %1, 4;\n setp.ne.b32 p, t, 0;\n"
+      " @p st.shared.v2.b32 [%0], {%4, %8};\n @p add.u32 %0, %0, 8;\n"
+      " and.b32 t, %1, 8;\n setp.ne.b32 p, t, 0;\n"
+      " @p st.shared.v2.b32 [%0], {%5, %9};\n @p add.u32 %0, %0, 8;\n}"
+      : "+r"(at)
+      : "r"(nib), "r"(__float_as_uint(v.x)), "r"(__float_as_uint(v.y)), "r"(__float_as_uint(v.z)),
+        "r"(__float_as_uint(v.w)), "r"(col0), "r"(col0 + 1), "r"(col0 + 2), "r"(col0 + 3)
+      : "memory");
+}
 
 // Row of the error / state buffer for a logical row (nullptr for plain TopK);
 // *ok = false for an AQ-SGD sample id out of range.
@@ -910,8 +946,25 @@ __device__ __forceinline__ float* state_row(const TopkRowArgs& a, int64_t row, b
 // slower; for other lengths the staged row is faster).
 __host__ __device__ constexpr int warp_row_buffers(int mode, int nvw) { return (mode == kPlain || nvw == 6) ? 1 : 2; }
 
+// Warps per CTA: eight, four when a warp's two row buffers exceed 12 KiB.
+__host__ __device__ constexpr int warp_wpc(int mode, int nvw) {
+  return 2 * 128 * nvw * 4 * warp_row_buffers(mode, nvw) > 12 * 1024 ? 4 : 8;
+}
+
+// CTAs per SM the registers are held to: as many as the shared memory admits
+// (row buffers and WarpShared), at most four; two for the fused variants on
+// rows of 513..768 entries, which hold 24 ranked values a thread (measured: at
+// three they spill and run ~5 % slower).
+__host__ __device__ constexpr int warp_min_blocks(int mode, int nvw) {
+  return (nvw == 6 && mode != kPlain) ? 2 : 227 * 1024 / (warp_wpc(mode, nvw) * (2 * 128 * nvw * 4 * warp_row_buffers(mode, nvw) +
+                                              static_cast<int>(sizeof(WarpShared)))) < 4
+             ? 227 * 1024 / (warp_wpc(mode, nvw) * (2 * 128 * nvw * 4 * warp_row_buffers(mode, nvw) +
+                                                    static_cast<int>(sizeof(WarpShared))))
+             : 4;
+}
+
 template <int MODE, int NVW, int WPC, bool FULL>
-__global__ void __launch_bounds__(32 * WPC) topk_warp_kernel(const TopkRowArgs a) {
+__global__ void __launch_bounds__(32 * WPC, warp_min_blocks(MODE, NVW)) topk_warp_kernel(const TopkRowArgs a) {
   pdl_begin();
   constexpr int RCAP = 128 * NVW;
   // x, and the err / state row, are staged per row in the warp's buffers;
@@ -1006,25 +1059,57 @@ __global__ void __launch_bounds__(32 * WPC) topk_warp_kernel(const TopkRowArgs a
       return make_float4(t[0], t[1], t[2], t[3]);
     };
 
-    // ---- ranked values (in place), the largest finite magnitude, any NaN -------
-    int kmax = -1, kall = -1;
+    // ---- ranked values and their keys; the largest key --------------------------
+    // Plain TopK holds the keys in registers and reads the values again from the
+    // row buffer; the fused variants hold the ranked values (x + err, x - state)
+    // and derive the keys.
+    constexpr bool kHoldKeys = MODE == kPlain;
+    int kv[kHoldKeys ? NVW : 1][4];
+    float4 sv[kHoldKeys ? 1 : NVW];
+    auto keys_of = [&](int v, int kk[4]) {
+      if constexpr (kHoldKeys) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) kk[i] = kv[v][i];
+      } else {
+        keys4<FULL>(sv[v], 4 * (v * 32 + lane), n, kk);
+      }
+    };
+    auto value_of = [&](int v) -> float4 {
+      if constexpr (kHoldKeys) return x4[v * 32 + lane];
+      else return sv[v];
+    };
+    int kall = -1;
 #pragma unroll
     for (int v = 0; v < NVW; ++v) {
       const int q = v * 32 + lane;
-      float4 val = x4[q];
-      if (MODE != kPlain) {
-        val = ranked4<MODE>(val, aux4(q));
-        x4[q] = val;
-      }
       int kk[4];
-      keys4<FULL>(val, 4 * q, n, kk);
-      kmax = max(kmax, max(max(finite_key(kk[0]), finite_key(kk[1])),
-                           max(finite_key(kk[2]), finite_key(kk[3]))));
+      if constexpr (kHoldKeys) {
+        keys4<FULL>(x4[q], 4 * q, n, kv[v]);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) kk[i] = kv[v][i];
+      } else {
+        sv[v] = ranked4<MODE>(x4[q], aux4(q));
+        keys4<FULL>(sv[v], 4 * q, n, kk);
+      }
       kall = max(kall, max(max(kk[0], kk[1]), max(kk[2], kk[3])));
     }
-    kmax = __reduce_max_sync(kFull, kmax);
-    // a NaN row (outside the finite-input contract) takes the integer rounds
-    if (__reduce_max_sync(kFull, kall) > 0x7f800000) kmax = 0;
+    kall = __reduce_max_sync(kFull, kall);
+    // the bin scale comes from the largest finite magnitude (TopK marks entries
+    // with +inf); a row with a NaN (outside the finite-input contract) takes the
+    // integer rounds
+    int kmax = kall;
+    if (kall >= 0x7f800000) {
+      kmax = -1;
+#pragma unroll
+      for (int v = 0; v < NVW; ++v) {
+        int kk[4];
+        keys_of(v, kk);
+        kmax = max(kmax, max(max(finite_key(kk[0]), finite_key(kk[1])),
+                             max(finite_key(kk[2]), finite_key(kk[3]))));
+      }
+      kmax = __reduce_max_sync(kFull, kmax);
+      if (kall > 0x7f800000) kmax = 0;
+    }
 
     // ---- select ---------------------------------------------------------------
     Threshold t;
@@ -1038,16 +1123,16 @@ __global__ void __launch_bounds__(32 * WPC) topk_warp_kernel(const TopkRowArgs a
       uint32_t m = static_cast<uint32_t>(n);  // with scale 0 every entry is a candidate
       if (scale > 0.0f) {
 #pragma unroll
-        for (int j = 0; j < 8; ++j) sh.hist[lane * 8 + j] = 0;
-        sh.hist[kRoundBins + lane] = 0;
-        sh.hist[kRoundBins + 32 + lane] = 0;
+        for (int j = 0; j < 8; ++j) sh.u.sel.hist[lane * 8 + j] = 0;
+        sh.u.sel.hist[kRoundBins + lane] = 0;
+        sh.u.sel.hist[kRoundBins + 32 + lane] = 0;
         if (lane == 0) sh.lcount = 0;
         __syncwarp();
 #pragma unroll
         for (int v = 0; v < NVW; ++v) {
           const int q = v * 32 + lane;
           int kk[4];
-          keys4<FULL>(x4[q], 4 * q, n, kk);
+          keys_of(v, kk);
 #pragma unroll
           for (int i = 0; i < 4; ++i) {
             // one atomic per entry and no branch: zeros to this lane's spill
@@ -1056,14 +1141,14 @@ __global__ void __launch_bounds__(32 * WPC) topk_warp_kernel(const TopkRowArgs a
             const int slot = kk[i] > 0 ? b
                                        : ((FULL || kk[i] == 0) ? kRoundBins + lane
                                                                : kRoundBins + 32 + lane);
-            atomicAdd(&sh.hist[slot], 1u);
+            atomicAdd(&sh.u.sel.hist[slot], 1u);
           }
         }
         __syncwarp();
-        const uint32_t zc = __reduce_add_sync(kFull, sh.hist[kRoundBins + lane]);
-        if (lane == 0) sh.hist[0] += zc;
+        const uint32_t zc = __reduce_add_sync(kFull, sh.u.sel.hist[kRoundBins + lane]);
+        if (lane == 0) sh.u.sel.hist[0] += zc;
         __syncwarp();
-        const BinPick p = warp_pick_bin(sh.hist, kr, lane);
+        const BinPick p = warp_pick_bin(sh.u.sel.hist, kr, lane);
         __syncwarp();
         B = p.bin;
         kr -= p.above;
@@ -1075,23 +1160,23 @@ __global__ void __launch_bounds__(32 * WPC) topk_warp_kernel(const TopkRowArgs a
         for (int v = 0; v < NVW; ++v) {
           const int q = v * 32 + lane;
           int kk[4];
-          keys4<FULL>(x4[q], 4 * q, n, kk);
+          keys_of(v, kk);
 #pragma unroll
           for (int i = 0; i < 4; ++i)
             if ((FULL || kk[i] >= 0) && bucket_of(kk[i], scale, kRoundBins) == B) {
               const uint32_t at = atomicAdd(&sh.lcount, 1u);
-              if (at < kLCAPW) sh.lkey[at] = kk[i];
+              if (at < kLCAPW) sh.u.sel.lkey[at] = kk[i];
             }
         }
         __syncwarp();
-        t = warp_select(sh.lkey, min(sh.lcount, static_cast<uint32_t>(kLCAPW)), kr, sh.hist, lane);
+        t = warp_select(sh.u.sel.lkey, min(sh.lcount, static_cast<uint32_t>(kLCAPW)), kr, sh.u.sel.hist, lane);
       } else {
         int lo = 0x7fffffff, hi = -1;
 #pragma unroll
         for (int v = 0; v < NVW; ++v) {
           const int q = v * 32 + lane;
           int kk[4];
-          keys4<FULL>(x4[q], 4 * q, n, kk);
+          keys_of(v, kk);
 #pragma unroll
           for (int i = 0; i < 4; ++i)
             if (kk[i] >= 0 && (scale == 0.0f || bucket_of(kk[i], scale, kRoundBins) == B)) {
@@ -1109,20 +1194,20 @@ __global__ void __launch_bounds__(32 * WPC) topk_warp_kernel(const TopkRowArgs a
           }
           const int sft = round_shift(lo, hi);
 #pragma unroll
-          for (int j = 0; j < 8; ++j) sh.hist[lane * 8 + j] = 0;
+          for (int j = 0; j < 8; ++j) sh.u.sel.hist[lane * 8 + j] = 0;
           __syncwarp();
 #pragma unroll
           for (int v = 0; v < NVW; ++v) {
             const int q = v * 32 + lane;
             int kk[4];
-            keys4<FULL>(x4[q], 4 * q, n, kk);
+            keys_of(v, kk);
 #pragma unroll
             for (int i = 0; i < 4; ++i)
               if (kk[i] >= lo && kk[i] <= hi)
-                atomicAdd(&sh.hist[static_cast<uint32_t>(kk[i] - lo) >> sft], 1u);
+                atomicAdd(&sh.u.sel.hist[static_cast<uint32_t>(kk[i] - lo) >> sft], 1u);
           }
           __syncwarp();
-          const BinPick q = warp_pick_bin(sh.hist, kr, lane);
+          const BinPick q = warp_pick_bin(sh.u.sel.hist, kr, lane);
           __syncwarp();
           kr -= q.above;
           const int nlo = lo + (q.bin << sft);
@@ -1142,72 +1227,106 @@ __global__ void __launch_bounds__(32 * WPC) topk_warp_kernel(const TopkRowArgs a
     const uint32_t need = t.need;
 
     // ---- write (one pass: the warp owns the whole row) ------------------------
-    float* vrow = a.vals + row * k;
-    int32_t* irow = a.idx + row * k;
-    uint32_t pos = 0, eq_seen = 0;
+    // kept entries: bit 4v + i of km for entry 4 (32 v + lane) + i
+    uint32_t km = 0;
 #pragma unroll
     for (int v = 0; v < NVW; ++v) {
-      const int q = v * 32 + lane;
-      const float4 v4 = x4[q];
       int kk[4];
-      keys4<FULL>(v4, 4 * q, n, kk);
-      bool kp[4];
-      if (need) {
-        uint32_t r = eq_seen;
+      keys_of(v, kk);
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const unsigned be = __ballot_sync(kFull, kk[i] == T);
-          r += __popc(be & lt);
-          eq_seen += __popc(be);
-        }
+      for (int i = 0; i < 4; ++i) or_if_key_gt(km, kk[i], T, 1u << (4 * v + i));
+    }
+    if (need) {
+      // the first `need` entries with key T, in index order
+      uint32_t seen = 0;
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const bool e = kk[i] == T;
-          kp[i] = kk[i] > T || (e && r < need);
-          r += e;
-        }
-      } else {
+      for (int v = 0; v < NVW; ++v) {
+        int kk[4];
+        keys_of(v, kk);
+        uint32_t em = 0;
 #pragma unroll
-        for (int i = 0; i < 4; ++i) kp[i] = kk[i] > T;
-      }
-      uint32_t p = pos;
+        for (int i = 0; i < 4; ++i) em |= static_cast<uint32_t>(kk[i] == T) << i;
+        const uint32_t c = __popc(em);
+        const uint32_t inc = warp_inclusive_scan(c, lane);
+        uint32_t r = seen + inc - c;
 #pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const unsigned bk = __ballot_sync(kFull, kp[i]);
-        p += __popc(bk & lt);
-        pos += __popc(bk);
-      }
-      const int e0 = 4 * q;
-      if (FULL || e0 < n) {
-        const float val[4] = {v4.x, v4.y, v4.z, v4.w};
-        float st[4] = {0.f, 0.f, 0.f, 0.f};
-        if (MODE == kDelta) {
-          const float4 sv = aux4(q);
-          st[0] = sv.x;
-          st[1] = sv.y;
-          st[2] = sv.z;
-          st[3] = sv.w;
-        }
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          if (kp[i]) {
-            if (p < static_cast<uint64_t>(k)) {
-              vrow[p] = val[i];
-              irow[p] = e0 + i;
-            }
-            if (MODE == kDelta) arow[e0 + i] = fadd(st[i], val[i]);
-            ++p;
+        for (int i = 0; i < 4; ++i)
+          if ((em >> i) & 1u) {
+            if (r < need) km |= 1u << (4 * v + i);
+            ++r;
           }
+        seen += __shfl_sync(kFull, inc, 31);
+      }
+    }
+    float* vrow = a.vals + row * k;
+    int32_t* irow = a.idx + row * k;
+    // The kept entries of two groups at a time go to the warp's write stage (the
+    // selection's scratch, free again) in index order, then out with coalesced
+    // stores.
+    auto fld = [](uint32_t w, int j) { return (w >> (8 * j)) & 0xffu; };
+    const uint32_t out_s = static_cast<uint32_t>(__cvta_generic_to_shared(sh.u.out));
+    uint32_t pos = 0;  // entries kept by the groups before
+    __syncwarp();      // every lane is done with the selection's scratch
+#pragma unroll
+    for (int v0 = 0; v0 < NVW; v0 += 4) {
+      // this lane's kept counts of four groups, a byte each (a group keeps at
+      // most 128 entries of the warp): one scan gives all four offsets
+      uint32_t pc = 0;
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        if (v0 + j < NVW) pc |= static_cast<uint32_t>(__popc((km >> (4 * (v0 + j))) & 0xfu)) << (8 * j);
+      const uint32_t inc = warp_inclusive_scan(pc, lane);
+      const uint32_t tot = __shfl_sync(kFull, inc, 31);
+      const uint32_t exc = inc - pc;
+#pragma unroll
+      for (int j = 0; j < 4 && v0 + j < NVW; j += 2) {  // NVW is even
+        const int va = v0 + j;
+        const uint32_t ta = fld(tot, j), tr = ta + fld(tot, j + 1);
+        uint32_t at = out_s + 8u * fld(exc, j);
+        stage_kept4((km >> (4 * va)) & 0xfu, at, value_of(va), 4 * (va * 32 + lane));
+        at = out_s + 8u * (ta + fld(exc, j + 1));
+        stage_kept4((km >> (4 * (va + 1))) & 0xfu, at, value_of((va + 1)), 4 * ((va + 1) * 32 + lane));
+        __syncwarp();
+        const uint32_t lim = pos < static_cast<uint64_t>(k)
+                                 ? static_cast<uint32_t>(min(static_cast<int64_t>(tr), k - pos))
+                                 : 0u;
+        float* vp = vrow + pos;
+        int32_t* ip = irow + pos;
+        for (uint32_t i = lane; i < lim; i += 32) {
+          const uint2 e = sh.u.out[i];
+          vp[i] = __uint_as_float(e.x);
+          ip[i] = static_cast<int32_t>(e.y);
         }
-        if (MODE == kEF) {
-          const float ne[4] = {kp[0] ? 0.0f : val[0], kp[1] ? 0.0f : val[1],
-                               kp[2] ? 0.0f : val[2], kp[3] ? 0.0f : val[3]};
-          if (a.aligned && (FULL || e0 + 4 <= n)) {
-            *reinterpret_cast<float4*>(arow + e0) = make_float4(ne[0], ne[1], ne[2], ne[3]);
-          } else {
+        __syncwarp();
+        pos += tr;
+      }
+    }
+    if (MODE != kPlain) {
+#pragma unroll
+      for (int v = 0; v < NVW; ++v) {
+        const int q = v * 32 + lane;
+        const int e0 = 4 * q;
+        const uint32_t nib = (km >> (4 * v)) & 0xfu;
+        if (FULL || e0 < n) {
+          const float4 s4 = value_of(v);
+          const float val[4] = {s4.x, s4.y, s4.z, s4.w};
+          if (MODE == kDelta && nib != 0) {  // state + d where kept
+            const float4 g = aux4(q);
+            const float st[4] = {g.x, g.y, g.z, g.w};
 #pragma unroll
             for (int i = 0; i < 4; ++i)
-              if (e0 + i < n) arow[e0 + i] = ne[i];
+              if ((nib >> i) & 1u) arow[e0 + i] = fadd(st[i], val[i]);
+          }
+          if (MODE == kEF) {  // err' = s - C(s): +0 where kept
+            const float ne[4] = {(nib & 1u) ? 0.0f : val[0], (nib & 2u) ? 0.0f : val[1],
+                                 (nib & 4u) ? 0.0f : val[2], (nib & 8u) ? 0.0f : val[3]};
+            if (a.aligned && (FULL || e0 + 4 <= n)) {
+              *reinterpret_cast<float4*>(arow + e0) = make_float4(ne[0], ne[1], ne[2], ne[3]);
+            } else {
+#pragma unroll
+              for (int i = 0; i < 4; ++i)
+                if (e0 + i < n) arow[e0 + i] = ne[i];
+            }
           }
         }
       }
@@ -1221,10 +1340,9 @@ __global__ void __launch_bounds__(32 * WPC) topk_warp_kernel(const TopkRowArgs a
 // ---------------------------------------------------------------------------
 template <int MODE, int NVW, bool FULL>
 cudaError_t run_warp(const TopkRowArgs& a, int num_sms, cudaStream_t s) {
-  // Eight warps per CTA, four when a warp's two row buffers exceed 12 KiB.
   constexpr int NBUF = warp_row_buffers(MODE, NVW);
   constexpr int WBYTES = 2 * 128 * NVW * 4 * NBUF;
-  constexpr int WPC = WBYTES > 12 * 1024 ? 4 : 8;
+  constexpr int WPC = warp_wpc(MODE, NVW);
   auto kernel = topk_warp_kernel<MODE, NVW, WPC, FULL>;
   const int smem = WPC * WBYTES;
   cudaError_t err = ensure_dynamic_smem(kernel, smem);
