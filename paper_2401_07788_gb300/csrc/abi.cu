@@ -122,7 +122,6 @@ mpc_status topk_compress_common(int mode, const float* x, float* aux, int64_t ro
   if (use_row_path(row_len)) {
     mpc::TopkRowArgs a = {};
     a.wide_cta = g_topk_path.load() != 3;
-  a.band = g_topk_path.load() != 4;
     a.band = g_topk_path.load() != 4;
     a.x = x;
     a.aux = aux;

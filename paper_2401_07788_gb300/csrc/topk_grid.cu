@@ -1,7 +1,10 @@
 // topk_grid.cu -- exact TopK (§2.3), with error feedback (§2.4) or the EF21
 // buffer update (§2.4), for rows longer than the on-chip row kernels take (up
 // to whole tensors of 2^31-1 entries), with the counters, lists and per-chunk
-// status words in a caller workspace; one row at a time.
+// status words in a caller workspace.  Rows go in batches of up to 64 (enough
+// for about 2^26 entries a batch): every launch below takes a batch, row
+// blockIdx.y of it, each row with a workspace slice of its own, so that a call
+// is 23 launches per batch whatever the number of rows.
 //
 // Per row, the selection by the band path (one read of the row), else by the
 // multi-pass path where the band path gave up, then the write: one more read
@@ -11,10 +14,10 @@
 // needed, so the host never waits.
 //
 // Band path:
-//   w_sample, w_spick  65536 entries spread over the row (one a thread over 64
-//             CTAs) give a band of keys [t_lo, t_hi) that holds the k-th
-//             largest magnitude unless the sample is 4 standard deviations
-//             off (as in topk_band.cuh);
+//   w_sample, w_spick  1/256 of the row's entries (1024 to 65536) spread
+//             over it (one a thread) give a band of keys [t_lo, t_hi) that
+//             holds the k-th largest magnitude unless the sample is 4
+//             standard deviations off (as in topk_band.cuh);
 //   w_pass1   one read of the row by persistent CTAs, 8192-entry chunks staged
 //             by double-buffered bulk copies: entries >= t_hi ("sure")
 //             counted; band entries (list mode: every entry >= t_lo) listed in
@@ -62,7 +65,6 @@ constexpr uint32_t kCandCap = 65536;     // candidate list capacity
 constexpr int kSamples = 4096;
 constexpr int kMaxRounds = 3;            // refinement rounds (11 bits each) reach one key
 constexpr int kWSamples = 65536;         // band path: sample entries
-constexpr int kWSCtas = kWSamples / 1024;  // band path: sampling CTAs (one entry a thread)
 constexpr int kWSBins = 32768;           // band path: sample bins, key >> 16 (1/128 octave)
 constexpr int kWSShift = 16;
 constexpr int kFBins = 256;              // band path: bins of the band histogram
@@ -119,6 +121,7 @@ struct WsLayout {
   int* c2key;       // kCand2Cap: keys of the chosen band bin
   uint32_t* nbc;    // kMaxBandCtas: band entries listed by each CTA of w_pass1
   uint32_t bcap;    // band list capacity (G regions of bcap / G entries, G the pass-1 grid)
+  uint32_t c2cap;   // c2key capacity: the chosen bin's entries are band-list entries
 };
 
 // CTAs of the persistent band-path kernels at most (each lists its band
@@ -138,6 +141,22 @@ uint32_t band_cap(int64_t L, int64_t k) {
 }
 
 size_t align256(size_t b) { return (b + 255) / 256 * 256; }
+
+uint32_t c2_cap(int64_t L, int64_t k) { return min(kCand2Cap, band_cap(L, k)); }
+
+// Band-path sample entries of a row: 1/256 of it (a multiple of 1024), at least
+// 1024 and at most kWSamples, so that the sample reads stay a few percent of
+// the row's sectors.
+int sample_count(int64_t L) {
+  return static_cast<int>(max64(1024, min64(kWSamples, L / 256 / 1024 * 1024)));
+}
+
+// Rows of one batch: enough rows for about 2^26 entries, at most 64.  Each row
+// of a batch has a workspace slice of its own.
+constexpr int64_t kMaxBatch = 64;
+int64_t grid_batch(int64_t rows, int64_t L) {
+  return max64(1, min64(min64(rows, kMaxBatch), (int64_t(1) << 26) / max64(L, 1)));
+}
 
 WsLayout layout(void* ws, int64_t L, int64_t k, int64_t nchunks) {
   WsLayout w;
@@ -163,8 +182,9 @@ WsLayout layout(void* ws, int64_t L, int64_t k, int64_t nchunks) {
   p += align256(kFBins * 4);
   w.shist = reinterpret_cast<uint32_t*>(p);
   p += align256(kWSBins * 4);
+  w.c2cap = c2_cap(L, k);
   w.c2key = reinterpret_cast<int*>(p);
-  p += align256(static_cast<size_t>(kCand2Cap) * 4);
+  p += align256(static_cast<size_t>(w.c2cap) * 4);
   w.nbc = reinterpret_cast<uint32_t*>(p);
   p += align256(kMaxBandCtas * 4);
   w.bcap = band_cap(L, k);
@@ -186,7 +206,7 @@ size_t ws_bytes_for(int64_t L, int64_t k) {
          2 * align256(static_cast<size_t>(((L + kWCH - 1) / kWCH + 1023) / 1024) * 4) +
          align256(kCandCap * 8) + align256(kCandCap * 4) + align256(kFBins * 4) +
          align256(kWSBins * 4) +
-         align256(static_cast<size_t>(kCand2Cap) * 4) + align256(kMaxBandCtas * 4) +
+         align256(static_cast<size_t>(c2_cap(L, k)) * 4) + align256(kMaxBandCtas * 4) +
          2 * align256(static_cast<size_t>(band_cap(L, k)) * 4);
 }
 
@@ -206,6 +226,13 @@ __device__ __forceinline__ float value_at(const float* xr, const float* ar, int6
   return xr[e];
 }
 
+// Rows are processed in batches, row blockIdx.y of a batch per launch: its
+// slice of the workspace lies wsr bytes after the previous row's.
+template <class T>
+__device__ __forceinline__ T* row_ws(T* p, size_t wsr) {
+  return reinterpret_cast<T*>(reinterpret_cast<uintptr_t>(p) + static_cast<uintptr_t>(blockIdx.y) * wsr);
+}
+
 __device__ __forceinline__ uint32_t block_sum(uint32_t v, uint32_t* red) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   v = __reduce_add_sync(kFull, v);
@@ -218,8 +245,13 @@ __device__ __forceinline__ uint32_t block_sum(uint32_t v, uint32_t* red) {
 }
 
 __global__ void g_init(GridMeta* meta, uint32_t* hist, uint32_t* shist, uint32_t* fhist,
-                       int64_t nchunks, int64_t L, int64_t k) {
+                       int64_t nchunks, int64_t L, int64_t k, size_t wsr) {
   pdl_begin();
+  pdl_end();  // light work: the next grid may be scheduled now
+  meta = row_ws(meta, wsr);
+  hist = row_ws(hist, wsr);
+  shist = row_ws(shist, wsr);
+  fhist = row_ws(fhist, wsr);
   for (int i = threadIdx.x; i < kGNB; i += blockDim.x) hist[i] = 0;
   for (int i = threadIdx.x; i < kWSBins; i += blockDim.x) shist[i] = 0;
   for (int i = threadIdx.x; i < kFBins; i += blockDim.x) fhist[i] = 0;
@@ -240,8 +272,12 @@ __global__ void g_init(GridMeta* meta, uint32_t* hist, uint32_t* shist, uint32_t
 
 template <int MODE>
 __global__ void __launch_bounds__(kGT) g_sample(const float* xr, const float* ar, int64_t L,
-                                                int64_t k, GridMeta* meta) {
+                                                int64_t k, GridMeta* meta, size_t wsr) {
   pdl_begin();
+  pdl_end();  // light work: the next grid may be scheduled now
+  xr += static_cast<int64_t>(blockIdx.y) * L;
+  if (MODE != kPlain) ar += static_cast<int64_t>(blockIdx.y) * L;
+  meta = row_ws(meta, wsr);
   __shared__ uint32_t red[kGT / 32];
   if (meta->resolved) return;  // the band path found T (or every entry is kept)
   int mx = -1;
@@ -270,8 +306,14 @@ __global__ void __launch_bounds__(kGT) g_sample(const float* xr, const float* ar
 // Later rounds: integer bins over the keys in [lo, hi].
 template <int MODE>
 __global__ void __launch_bounds__(kGT) g_hist(const float* xr, float* ar, int64_t L,
-                                              GridMeta* meta, uint32_t* hist, int first) {
+                                              GridMeta* meta, uint32_t* hist, int first,
+                                              size_t wsr) {
   pdl_begin();
+  pdl_end();  // light work: the next grid may be scheduled now
+  xr += static_cast<int64_t>(blockIdx.y) * L;
+  if (MODE != kPlain) ar += static_cast<int64_t>(blockIdx.y) * L;
+  meta = row_ws(meta, wsr);
+  hist = row_ws(hist, wsr);
   __shared__ uint32_t sh[kGNB];
   const GridMeta m = *meta;
   const bool bins = !m.resolved && m.m > kCandCap;
@@ -321,8 +363,11 @@ __device__ int first_key_of_bin(int b, float scale) {
 }
 
 // Pick the bin holding the kr-th entry and narrow [lo, hi] to it.
-__global__ void __launch_bounds__(kGT) g_pick(GridMeta* meta, uint32_t* hist) {
+__global__ void __launch_bounds__(kGT) g_pick(GridMeta* meta, uint32_t* hist, size_t wsr) {
   pdl_begin();
+  pdl_end();  // light work: the next grid may be scheduled now
+  meta = row_ws(meta, wsr);
+  hist = row_ws(hist, wsr);
   __shared__ uint32_t red[kGT / 32];
   __shared__ uint32_t pick_t, pick_excl;
   GridMeta m = *meta;
@@ -396,8 +441,16 @@ __global__ void __launch_bounds__(kGT) g_pick(GridMeta* meta, uint32_t* hist) {
 template <int MODE>
 __global__ void __launch_bounds__(kGT) g_count(const float* xr, const float* ar, int64_t L,
                                                GridMeta* meta, uint32_t* cgt, uint32_t* ceq,
-                                               int* ckey, int64_t* cidx) {
+                                               int* ckey, int64_t* cidx, size_t wsr) {
   pdl_begin();
+  pdl_end();  // light work: the next grid may be scheduled now
+  xr += static_cast<int64_t>(blockIdx.y) * L;
+  if (MODE != kPlain) ar += static_cast<int64_t>(blockIdx.y) * L;
+  meta = row_ws(meta, wsr);
+  cgt = row_ws(cgt, wsr);
+  ceq = row_ws(ceq, wsr);
+  ckey = row_ws(ckey, wsr);
+  cidx = row_ws(cidx, wsr);
   __shared__ uint32_t red[kGT / 32];
   const GridMeta m = *meta;
   if (m.counted) return;  // the band path has the counts
@@ -433,8 +486,14 @@ __global__ void __launch_bounds__(kGT) g_count(const float* xr, const float* ar,
 
 // T and need from the candidate list (one CTA), then the candidates' chunks.
 __global__ void __launch_bounds__(1024) g_select(GridMeta* meta, uint32_t* cgt, uint32_t* ceq,
-                                                 const int* ckey, const int64_t* cidx) {
+                                                 const int* ckey, const int64_t* cidx, size_t wsr) {
   pdl_begin();
+  pdl_end();  // light work: the next grid may be scheduled now
+  meta = row_ws(meta, wsr);
+  cgt = row_ws(cgt, wsr);
+  ceq = row_ws(ceq, wsr);
+  ckey = row_ws(ckey, wsr);
+  cidx = row_ws(cidx, wsr);
   __shared__ uint32_t hist[kRoundBins];
   __shared__ int s_lo, s_hi, s_T;
   __shared__ uint32_t s_kr, s_need, s_done;
@@ -524,19 +583,26 @@ __device__ __forceinline__ uint32_t excl_scan_1024(uint32_t v, uint32_t* red, ui
 // Band path
 // ===========================================================================
 
-// The band from a sample of the row.  w_sample: 65536 entries spread evenly
-// over the row, one a thread over kWSCtas CTAs, binned by magnitude key into
-// 32768 bins of 1/128 octave (key >> 16), and the largest finite sample key.
+// The band from a sample of the row.  w_sample: ns = sample_count(L) entries
+// spread evenly over the row, one a thread over ns / 1024 CTAs, binned by
+// magnitude key into 32768 bins of 1/128 octave (key >> 16), and the largest
+// finite sample key.
 // w_spick (one CTA): the band reaches 4 standard deviations of the sample count
 // on either side of the k-th entry; list mode when the sample's count at or
 // above t_lo, scaled to the row with a margin, fits the list.
 template <int MODE>
 __global__ void __launch_bounds__(1024) w_sample(const float* xr, const float* ar, int64_t L,
-                                                 GridMeta* meta, uint32_t* shist) {
+                                                 GridMeta* meta, uint32_t* shist, int ns,
+                                                 size_t wsr) {
   pdl_begin();
+  pdl_end();  // light work: the next grid may be scheduled now
+  xr += static_cast<int64_t>(blockIdx.y) * L;
+  if (MODE != kPlain) ar += static_cast<int64_t>(blockIdx.y) * L;
+  meta = row_ws(meta, wsr);
+  shist = row_ws(shist, wsr);
   if (meta->resolved) return;  // every entry is kept
   const int64_t s = static_cast<int64_t>(blockIdx.x) * 1024 + threadIdx.x;
-  const int64_t e = s * L / kWSamples;
+  const int64_t e = s * L / ns;
   const int key = mag_key(ranked<MODE>(xr[e], MODE != kPlain ? ar[e] : 0.0f));
   // lanes with the same bin add once
   const uint32_t bin = static_cast<uint32_t>(key) >> kWSShift;
@@ -547,8 +613,12 @@ __global__ void __launch_bounds__(1024) w_sample(const float* xr, const float* a
 }
 
 __global__ void __launch_bounds__(1024) w_spick(int64_t L, int64_t k, GridMeta* meta,
-                                                const uint32_t* shist, int list_ok, uint32_t bcap) {
+                                                const uint32_t* shist, int list_ok, uint32_t bcap,
+                                                int ns, size_t wsr) {
   pdl_begin();
+  pdl_end();  // light work: the next grid may be scheduled now
+  meta = row_ws(meta, wsr);
+  shist = row_ws(shist, wsr);
   // bins in rank order (largest keys first): warp w reads ranks [1024 w, 1024 w + 1024),
   // lane l the ranks 1024 w + 32 j + l (coalesced)
   constexpr int J = kWSBins / 1024;
@@ -560,8 +630,8 @@ __global__ void __launch_bounds__(1024) w_spick(int64_t L, int64_t k, GridMeta* 
   const int smax = meta->smax;
   if (smax <= 0) return;  // no finite non-zero magnitude in the sample: multi-pass path
   if (tid < 2) pick[tid] = -1;
-  if (tid == 0) s_ge = kWSamples;
-  const float mu = __fdividef(static_cast<float>(k) * static_cast<float>(kWSamples),
+  if (tid == 0) s_ge = ns;
+  const float mu = __fdividef(static_cast<float>(k) * static_cast<float>(ns),
                               static_cast<float>(L));
   const float sd = mu * rsqrtf(mu);
   const int r_hi = static_cast<int>(floorf(mu - kWZ * sd));
@@ -581,7 +651,7 @@ __global__ void __launch_bounds__(1024) w_spick(int64_t L, int64_t k, GridMeta* 
 #pragma unroll
   for (int q = 0; q < 2; ++q) {
     const int r = rs[q];
-    if (r >= 1 && r <= kWSamples && before < static_cast<uint32_t>(r) &&
+    if (r >= 1 && r <= ns && before < static_cast<uint32_t>(r) &&
         static_cast<uint32_t>(r) <= before + s) {
       // this warp's block holds the r-th largest: 32 bins at a time
       uint32_t run = before;
@@ -619,8 +689,8 @@ __global__ void __launch_bounds__(1024) w_spick(int64_t L, int64_t k, GridMeta* 
     meta->ncand2 = 0;
     meta->bin2 = 0;
     meta->band = 1;
-    const float est = static_cast<float>(pick[1] > 0 ? s_ge : kWSamples) *
-                      (static_cast<float>(L) / static_cast<float>(kWSamples));
+    const float est = static_cast<float>(pick[1] > 0 ? s_ge : ns) *
+                      (static_cast<float>(L) / static_cast<float>(ns));
     meta->lmode = list_ok && pick[1] > 0 && est * 1.25f + 65536.0f <= static_cast<float>(bcap);
   }
 }
@@ -643,6 +713,20 @@ __device__ __forceinline__ void issue_chunk(float* buf, const float* src, const 
   bulk_g2s(buf + p0, src + c0 + p0, bytes, &bars[lane]);
 }
 
+// L2 prefetch of chunk c of src, part w (1024 entries) by lane w of warp 0: the
+// chunk after the one whose bulk copies were just issued, so that each CTA has
+// two chunks on the way from HBM.
+template <int NW, int64_t CH>
+__device__ __forceinline__ void prefetch_chunk(const float* src, int64_t L, int64_t c, int lane) {
+  const int64_t c0 = c * CH;
+  if (c0 >= L) return;
+  const int n = static_cast<int>(min64(CH, L - c0));
+  const int p0 = 1024 * lane;
+  if (lane >= NW || p0 >= n) return;
+  const uint32_t bytes = static_cast<uint32_t>(min(1024, n - p0)) * 4u;
+  bulk_prefetch_l2(src + c0 + p0, bytes);
+}
+
 // One read of the row.  Persistent CTAs take chunks c, c + G, ... (G = the grid),
 // double-buffered: the next chunk's bulk copies are in flight while this one
 // is classified.  Thread t owns the 32 consecutive entries [32t, 32t + 32) of a
@@ -658,8 +742,19 @@ __global__ void __launch_bounds__(kGT) w_pass1(const float* xr, float* ar, int64
                                                uint32_t* cgt, uint32_t* ceq, int* bkey,
                                                uint32_t* bidx, uint32_t rcap, uint32_t* nbc,
                                                uint32_t* seg, uint32_t* segn, uint32_t* fhist,
-                                               uint32_t spin_limit, unsigned* status) {
+                                               uint32_t spin_limit, unsigned* status, size_t wsr) {
   pdl_begin();
+  xr += static_cast<int64_t>(blockIdx.y) * L;
+  if (MODE != kPlain) ar += static_cast<int64_t>(blockIdx.y) * L;
+  meta = row_ws(meta, wsr);
+  cgt = row_ws(cgt, wsr);
+  ceq = row_ws(ceq, wsr);
+  bkey = row_ws(bkey, wsr);
+  bidx = row_ws(bidx, wsr);
+  nbc = row_ws(nbc, wsr);
+  seg = row_ws(seg, wsr);
+  segn = row_ws(segn, wsr);
+  fhist = row_ws(fhist, wsr);
   constexpr int NW = kGT / 32;
   extern __shared__ __align__(16) float wbuf[];  // 2 x kCH
   __shared__ uint32_t fh[kFBins];
@@ -706,8 +801,12 @@ __global__ void __launch_bounds__(kGT) w_pass1(const float* xr, float* ar, int64
   static_assert(kCH == 2 * kWCH, "a pass-1 chunk is two write chunks");
   for (; c < nchunks; c += gridDim.x, b ^= 1) {
     const int64_t cn = c + gridDim.x;
-    if (aligned && warp == 0 && cn < nchunks)
+    if (aligned && warp == 0 && cn < nchunks) {
       issue_chunk<NW, kCH>(wbuf + (b ^ 1) * kCH, xr, pre, L, cn, bars[b ^ 1], lane);
+      // plain TopK only (measured: with the err row as well, and in the write
+      // pass, the deeper prefetch is slower)
+      if (MODE == kPlain) prefetch_chunk<NW, kCH>(xr, L, cn + gridDim.x, lane);
+    }
     if (tid == 0 && prev >= 0) put_sure(prev, b ^ 1);
     const int64_t c0 = c * kCH;
     const int n = static_cast<int>(min64(kCH, L - c0));
@@ -822,8 +921,12 @@ __global__ void __launch_bounds__(kGT) w_pass1(const float* xr, float* ar, int64
 }
 
 // The band bin holding the k-th entry, or the band path gives up (one warp).
-__global__ void __launch_bounds__(32) w_pick1(GridMeta* meta, const uint32_t* fhist, int64_t k) {
+__global__ void __launch_bounds__(32) w_pick1(GridMeta* meta, const uint32_t* fhist, int64_t k,
+                                              size_t wsr) {
   pdl_begin();
+  pdl_end();  // light work: the next grid may be scheduled now
+  meta = row_ws(meta, wsr);
+  fhist = row_ws(fhist, wsr);
   const GridMeta m = *meta;
   if (!m.band || m.resolved) return;
   const int lane = threadIdx.x & 31;
@@ -860,8 +963,14 @@ __global__ void __launch_bounds__(32) w_pick1(GridMeta* meta, const uint32_t* fh
 // The band entries of the chosen bin, listed: CTA r reads region r of the band
 // list (four loads in flight a thread; one atomic a warp).
 __global__ void __launch_bounds__(256) w_bin2(GridMeta* meta, const int* bkey, const uint32_t* nbc,
-                                              uint32_t rcap, int* c2key) {
+                                              uint32_t rcap, int* c2key, uint32_t c2cap,
+                                              size_t wsr) {
   pdl_begin();
+  pdl_end();  // light work: the next grid may be scheduled now
+  meta = row_ws(meta, wsr);
+  bkey = row_ws(bkey, wsr);
+  nbc = row_ws(nbc, wsr);
+  c2key = row_ws(c2key, wsr);
   const GridMeta m = *meta;
   if (!m.band || !m.bin2) return;
   const int lane = threadIdx.x & 31;
@@ -884,21 +993,25 @@ __global__ void __launch_bounds__(256) w_bin2(GridMeta* meta, const int* bkey, c
       if (lane == 0) base = atomicAdd(&meta->ncand2, static_cast<uint32_t>(__popc(bb)));
       base = __shfl_sync(kFull, base, 0);
       const uint32_t slot = base + __popc(bb & lt);
-      if (in && slot < kCand2Cap) c2key[slot] = key[q];
+      if (in && slot < c2cap) c2key[slot] = key[q];
     }
   }
 }
 
 // T and need among the chosen bin's entries, by integer rounds (one CTA).
-__global__ void __launch_bounds__(1024) w_select2(GridMeta* meta, const int* c2key) {
+__global__ void __launch_bounds__(1024) w_select2(GridMeta* meta, const int* c2key, uint32_t c2cap,
+                                                  size_t wsr) {
   pdl_begin();
+  pdl_end();  // light work: the next grid may be scheduled now
+  meta = row_ws(meta, wsr);
+  c2key = row_ws(c2key, wsr);
   __shared__ uint32_t hist[kRoundBins];
   __shared__ int s_lo, s_hi, s_T;
   __shared__ uint32_t s_kr, s_need, s_done;
   const GridMeta m = *meta;
   if (!m.band || !m.bin2) return;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  if (m.ncand2 > kCand2Cap) {
+  if (m.ncand2 > c2cap) {
     if (tid == 0) meta->band = 0;  // too crowded: the multi-pass path takes over
     return;
   }
@@ -961,8 +1074,15 @@ __global__ void __launch_bounds__(1024) w_select2(GridMeta* meta, const int* c2k
 // reads region r of the band list; lanes of a warp on the same chunk add once.
 __global__ void __launch_bounds__(256) w_mark(const GridMeta* meta, const int* bkey,
                                               const uint32_t* bidx, const uint32_t* nbc,
-                                              uint32_t rcap, uint32_t* cgt, uint32_t* ceq) {
+                                              uint32_t rcap, uint32_t* cgt, uint32_t* ceq, size_t wsr) {
   pdl_begin();
+  pdl_end();  // light work: the next grid may be scheduled now
+  meta = row_ws(meta, wsr);
+  bkey = row_ws(bkey, wsr);
+  bidx = row_ws(bidx, wsr);
+  nbc = row_ws(nbc, wsr);
+  cgt = row_ws(cgt, wsr);
+  ceq = row_ws(ceq, wsr);
   const GridMeta m = *meta;
   if (!m.band || !m.resolved) return;
   const int lane = threadIdx.x & 31;
@@ -996,8 +1116,13 @@ __global__ void __launch_bounds__(256) w_mark(const GridMeta* meta, const int* b
 // (one CTA) scans the totals.  The counts before chunk c are then
 // cgt[c] + tg[c / 1024] (and ceq[c] + te[c / 1024]).
 __global__ void __launch_bounds__(1024) w_scan1(uint32_t* cgt, uint32_t* ceq, uint32_t* tg,
-                                                uint32_t* te, int64_t nwch) {
+                                                uint32_t* te, int64_t nwch, size_t wsr) {
   pdl_begin();
+  pdl_end();  // light work: the next grid may be scheduled now
+  cgt = row_ws(cgt, wsr);
+  ceq = row_ws(ceq, wsr);
+  tg = row_ws(tg, wsr);
+  te = row_ws(te, wsr);
   __shared__ uint32_t red[32];
   const int64_t c = static_cast<int64_t>(blockIdx.x) * 1024 + threadIdx.x;
   const uint32_t g = c < nwch ? cgt[c] : 0u, q = c < nwch ? ceq[c] : 0u;
@@ -1014,8 +1139,11 @@ __global__ void __launch_bounds__(1024) w_scan1(uint32_t* cgt, uint32_t* ceq, ui
   }
 }
 
-__global__ void __launch_bounds__(1024) w_scan2(uint32_t* tg, uint32_t* te, int nblocks) {
+__global__ void __launch_bounds__(1024) w_scan2(uint32_t* tg, uint32_t* te, int nblocks, size_t wsr) {
   pdl_begin();
+  pdl_end();  // light work: the next grid may be scheduled now
+  tg = row_ws(tg, wsr);
+  te = row_ws(te, wsr);
   __shared__ uint32_t red[32];
   uint32_t carry_g = 0, carry_q = 0;
   for (int b0 = 0; b0 < nblocks; b0 += 1024) {
@@ -1059,8 +1187,17 @@ __global__ void __launch_bounds__(kWT) g_write3(const float* xr, float* ar, int6
                                                 const GridMeta* meta, const uint32_t* cgt,
                                                 const uint32_t* ceq, const uint32_t* tg,
                                                 const uint32_t* te, float* vals, int32_t* idx,
-                                                uint32_t spin_limit, unsigned* status) {
+                                                uint32_t spin_limit, unsigned* status, size_t wsr) {
   pdl_begin();
+  xr += static_cast<int64_t>(blockIdx.y) * L;
+  if (MODE != kPlain) ar += static_cast<int64_t>(blockIdx.y) * L;
+  meta = row_ws(meta, wsr);
+  cgt = row_ws(cgt, wsr);
+  ceq = row_ws(ceq, wsr);
+  tg = row_ws(tg, wsr);
+  te = row_ws(te, wsr);
+  vals += static_cast<int64_t>(blockIdx.y) * k;
+  idx += static_cast<int64_t>(blockIdx.y) * k;
   constexpr int NW = kWT / 32;
   extern __shared__ __align__(16) float wbuf[];  // 2 x kWCH values, then kWCH staged columns
   uint16_t* cols = reinterpret_cast<uint16_t*>(wbuf + 2 * kWCH);
@@ -1231,8 +1368,20 @@ __global__ void __launch_bounds__(256) g_wlist(float* ar, int64_t nchunks, uint3
                                                const uint32_t* seg, const uint32_t* segn,
                                                const uint32_t* cgt, const uint32_t* ceq,
                                                const uint32_t* tg, const uint32_t* te,
-                                               float* vals, int32_t* idx) {
+                                               float* vals, int32_t* idx, int64_t L, size_t wsr) {
   pdl_begin();
+  if (MODE != kPlain) ar += static_cast<int64_t>(blockIdx.y) * L;
+  meta = row_ws(meta, wsr);
+  bkey = row_ws(bkey, wsr);
+  bidx = row_ws(bidx, wsr);
+  seg = row_ws(seg, wsr);
+  segn = row_ws(segn, wsr);
+  cgt = row_ws(cgt, wsr);
+  ceq = row_ws(ceq, wsr);
+  tg = row_ws(tg, wsr);
+  te = row_ws(te, wsr);
+  vals += static_cast<int64_t>(blockIdx.y) * k;
+  idx += static_cast<int64_t>(blockIdx.y) * k;
   if (!(meta->band && meta->lmode)) return;
   const int T = meta->T;
   const uint32_t need = meta->need;
@@ -1276,9 +1425,10 @@ __global__ void __launch_bounds__(256) g_wlist(float* ar, int64_t nchunks, uint3
 // Persistent grids: the CTAs that fit on the GPU (and no more than the band
 // list has regions).
 template <class K>
-unsigned persistent_grid(K kernel, int threads, int smem, int num_sms, int64_t nchunks) {
+unsigned persistent_grid(K kernel, int threads, int smem, int num_sms, int64_t nchunks, int64_t batch) {
   const int occ = resident_blocks(kernel, threads, smem);
-  const int64_t g = min64(min64(static_cast<int64_t>(num_sms) * occ, kMaxBandCtas), nchunks);
+  const int64_t fit = (static_cast<int64_t>(num_sms) * occ + batch - 1) / batch;  // per row
+  const int64_t g = min64(min64(fit, kMaxBandCtas), nchunks);
   return static_cast<unsigned>(max64(g, 1));
 }
 
@@ -1289,7 +1439,9 @@ cudaError_t run_grid(const TopkGridArgs& a, int num_sms, cudaStream_t s) {
   const int64_t nwch = (L + kWCH - 1) / kWCH;
   const int nblk = static_cast<int>((nwch + 1023) / 1024);
   if (nchunks > 0x7fffffffLL) return cudaErrorInvalidValue;
-  const WsLayout w = layout(a.ws, L, a.k, nchunks);
+  const int64_t B = grid_batch(a.rows, L);
+  const size_t wsr = align256(ws_bytes_for(L, a.k));  // one row's workspace slice
+  const WsLayout w = layout(a.ws, L, a.k, nchunks);     // the first row's
   auto al16 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; };
   const int aligned = (L % 4 == 0) && al16(a.x) && (MODE == kPlain || al16(a.aux));
   constexpr int kP1Smem = 2 * kCH * 4;             // two chunk buffers
@@ -1299,56 +1451,64 @@ cudaError_t run_grid(const TopkGridArgs& a, int num_sms, cudaStream_t s) {
   cudaError_t err = ensure_dynamic_smem(p1, kP1Smem);
   if (err == cudaSuccess) err = ensure_dynamic_smem(wr, kWSmem);
   if (err != cudaSuccess) return err;
-  const unsigned g1 = persistent_grid(p1, kGT, kP1Smem, num_sms, nchunks);
-  const unsigned gw = persistent_grid(wr, kWT, kWSmem, num_sms, nwch);
+  // grids per row (the launches below take B rows, blockIdx.y the row)
+  const unsigned g1 = persistent_grid(p1, kGT, kP1Smem, num_sms, nchunks, B);
+  const unsigned gw = persistent_grid(wr, kWT, kWSmem, num_sms, nwch, B);
   const uint32_t rcap = w.bcap / g1;  // band-list region of one pass-1 CTA
+  const int ns = sample_count(L);
   // the list-mode write: a warp per pass-1 chunk
-  const unsigned gl = static_cast<unsigned>(min64((nchunks + 7) / 8, static_cast<int64_t>(num_sms) * 8));
+  const unsigned gl = static_cast<unsigned>(
+      max64(1, min64((nchunks + 7) / 8, (static_cast<int64_t>(num_sms) * 8 + B - 1) / B)));
   // the multi-pass kernels: a fixed grid striding over the chunks
-  const unsigned gm = static_cast<unsigned>(min64(nwch, static_cast<int64_t>(num_sms) * 8));
-  for (int64_t r = 0; r < a.rows; ++r) {
-    const float* xr = a.x + r * L;
-    float* ar = (MODE != kPlain) ? a.aux + r * L : nullptr;
-    float* vr = a.vals + r * a.k;
-    int32_t* ir = a.idx + r * a.k;
-    g_init<<<1, 1024, 0, s>>>(w.meta, w.hist, w.shist, w.fhist, nchunks, L, a.k);
+  const unsigned gm = static_cast<unsigned>(
+      max64(1, min64(nwch, (static_cast<int64_t>(num_sms) * 8 + B - 1) / B)));
+  // launches with programmatic dependent launch (the light kernels let the next
+  // grid be scheduled as soon as they start); the first error ends the call
+  auto go = [&](auto kernel, dim3 grid, int threads, int smem, auto... args) {
+    if (err == cudaSuccess) err = launch_kernel(kernel, grid, dim3(threads), smem, s, 0u, args...);
+  };
+  for (int64_t r0 = 0; r0 < a.rows && err == cudaSuccess; r0 += B) {
+    const unsigned nb = static_cast<unsigned>(min64(B, a.rows - r0));
+    const float* xr = a.x + r0 * L;
+    float* ar = (MODE != kPlain) ? a.aux + r0 * L : nullptr;
+    float* vr = a.vals + r0 * a.k;
+    int32_t* ir = a.idx + r0 * a.k;
+    auto G = [nb](unsigned x) { return dim3(x, nb); };
+    go(g_init, G(1), 1024, 0, w.meta, w.hist, w.shist, w.fhist, nchunks, L, a.k, wsr);
     // the band path
-    w_sample<MODE><<<kWSCtas, 1024, 0, s>>>(xr, ar, L, w.meta, w.shist);
-    w_spick<<<1, 1024, 0, s>>>(L, a.k, w.meta, w.shist, list_eligible(L, a.k) ? 1 : 0, w.bcap);
-    p1<<<g1, kGT, kP1Smem, s>>>(xr, ar, L, nchunks, aligned, w.meta, w.cgt, w.ceq, w.bkey, w.bidx,
-                                rcap, w.nbc, w.seg, w.segn, w.fhist, a.spin_limit, a.status);
-    w_pick1<<<1, 32, 0, s>>>(w.meta, w.fhist, a.k);
-    w_bin2<<<g1, 256, 0, s>>>(w.meta, w.bkey, w.nbc, rcap, w.c2key);
-    w_select2<<<1, 1024, 0, s>>>(w.meta, w.c2key);
-    w_mark<<<g1, 256, 0, s>>>(w.meta, w.bkey, w.bidx, w.nbc, rcap, w.cgt, w.ceq);
+    go(w_sample<MODE>, G(static_cast<unsigned>(ns / 1024)), 1024, 0, xr, ar, L, w.meta, w.shist, ns, wsr);
+    go(w_spick, G(1), 1024, 0, L, a.k, w.meta, w.shist, list_eligible(L, a.k) ? 1 : 0, w.bcap, ns, wsr);
+    go(p1, G(g1), kGT, kP1Smem, xr, ar, L, nchunks, aligned, w.meta, w.cgt, w.ceq, w.bkey, w.bidx,
+       rcap, w.nbc, w.seg, w.segn, w.fhist, a.spin_limit, a.status, wsr);
+    go(w_pick1, G(1), 32, 0, w.meta, w.fhist, a.k, wsr);
+    go(w_bin2, G(g1), 256, 0, w.meta, w.bkey, w.nbc, rcap, w.c2key, w.c2cap, wsr);
+    go(w_select2, G(1), 1024, 0, w.meta, w.c2key, w.c2cap, wsr);
+    go(w_mark, G(g1), 256, 0, w.meta, w.bkey, w.bidx, w.nbc, rcap, w.cgt, w.ceq, wsr);
     // the multi-pass path (each kernel returns at once when the band path resolved)
-    g_sample<MODE><<<1, kGT, 0, s>>>(xr, ar, L, a.k, w.meta);
-    g_hist<MODE><<<gm, kGT, 0, s>>>(xr, ar, L, w.meta, w.hist, 1);
-    g_pick<<<1, kGT, 0, s>>>(w.meta, w.hist);
+    go(g_sample<MODE>, G(1), kGT, 0, xr, ar, L, a.k, w.meta, wsr);
+    go(g_hist<MODE>, G(gm), kGT, 0, xr, ar, L, w.meta, w.hist, 1, wsr);
+    go(g_pick, G(1), kGT, 0, w.meta, w.hist, wsr);
     for (int i = 0; i < kMaxRounds; ++i) {
-      g_hist<MODE><<<gm, kGT, 0, s>>>(xr, ar, L, w.meta, w.hist, 0);
-      g_pick<<<1, kGT, 0, s>>>(w.meta, w.hist);
+      go(g_hist<MODE>, G(gm), kGT, 0, xr, ar, L, w.meta, w.hist, 0, wsr);
+      go(g_pick, G(1), kGT, 0, w.meta, w.hist, wsr);
     }
-    g_count<MODE><<<gm, kGT, 0, s>>>(xr, ar, L, w.meta, w.cgt, w.ceq, w.ckey, w.cidx);
-    g_select<<<1, 1024, 0, s>>>(w.meta, w.cgt, w.ceq, w.ckey, w.cidx);
+    go(g_count<MODE>, G(gm), kGT, 0, xr, ar, L, w.meta, w.cgt, w.ceq, w.ckey, w.cidx, wsr);
+    go(g_select, G(1), 1024, 0, w.meta, w.cgt, w.ceq, w.ckey, w.cidx, wsr);
     // both paths: positions per write chunk, then the payload (the second read)
-    w_scan1<<<nblk, 1024, 0, s>>>(w.cgt, w.ceq, w.tg, w.te, nwch);
-    w_scan2<<<1, 1024, 0, s>>>(w.tg, w.te, nblk);
-    wr<<<gw, kWT, kWSmem, s>>>(xr, ar, L, nwch, a.k, aligned, w.meta, w.cgt, w.ceq, w.tg, w.te,
-                               vr, ir, a.spin_limit, a.status);
-    g_wlist<MODE><<<gl, 256, 0, s>>>(ar, nchunks, g1, rcap, a.k, w.meta, w.bkey, w.bidx, w.seg,
-                                     w.segn, w.cgt, w.ceq, w.tg, w.te, vr, ir);
-    const cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
+    go(w_scan1, G(static_cast<unsigned>(nblk)), 1024, 0, w.cgt, w.ceq, w.tg, w.te, nwch, wsr);
+    go(w_scan2, G(1), 1024, 0, w.tg, w.te, nblk, wsr);
+    go(wr, G(gw), kWT, kWSmem, xr, ar, L, nwch, a.k, aligned, w.meta, w.cgt, w.ceq, w.tg, w.te, vr,
+       ir, a.spin_limit, a.status, wsr);
+    go(g_wlist<MODE>, G(gl), 256, 0, ar, nchunks, g1, rcap, a.k, w.meta, w.bkey, w.bidx, w.seg,
+       w.segn, w.cgt, w.ceq, w.tg, w.te, vr, ir, L, wsr);
   }
-  return cudaSuccess;
+  return err;
 }
 
 }  // namespace
 
 size_t topk_grid_workspace_bytes(int64_t rows, int64_t L, int64_t k) {
-  (void)rows;
-  return ws_bytes_for(L, k);
+  return static_cast<size_t>(grid_batch(rows, L)) * align256(ws_bytes_for(L, k));
 }
 
 cudaError_t launch_topk_grid(int mode, const TopkGridArgs& a, int num_sms, cudaStream_t s) {

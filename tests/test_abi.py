@@ -56,6 +56,17 @@ def test_sizes(lib):
     assert lib.mpc_quant_codes_words(1, 5, 17) == 0  # unsupported width
     assert lib.mpc_topk_workspace_bytes(128, 32768, 3276) == 0  # on-chip path
     assert lib.mpc_quant_workspace_bytes(128, 32768, 4) == 0
+    # rows longer than 65536 go through the grid path in batches of up to 64 rows (about
+    # 2^26 entries a batch), with a 256-byte-aligned workspace slice per row of a batch
+    one = lib.mpc_topk_workspace_bytes(1, 70000, 7000)
+    assert one > 0 and one % 256 == 0
+    assert lib.mpc_topk_workspace_bytes(2, 70000, 7000) == 2 * one
+    assert lib.mpc_topk_workspace_bytes(64, 70000, 7000) == 64 * one
+    assert lib.mpc_topk_workspace_bytes(1000, 70000, 7000) == 64 * one
+    big = lib.mpc_topk_workspace_bytes(1, 1 << 24, 1 << 20)
+    assert lib.mpc_topk_workspace_bytes(16, 1 << 24, 1 << 20) == 4 * big
+    whole = lib.mpc_topk_workspace_bytes(1, 1 << 30, 1 << 20)
+    assert lib.mpc_topk_workspace_bytes(3, 1 << 30, 1 << 20) == whole
 
 
 @pytest.mark.parametrize("args,code", [

@@ -137,10 +137,10 @@ def test_workspace_too_small_is_rejected(mpc):
 
 @pytest.mark.parametrize("L", [131072, 1000003])
 def test_sample_misled(mpc, L):
-    """A row whose sampled positions (16384 evenly spread) hold much larger magnitudes
-    than the rest: the sampled band misses the k-th entry after the first read, and the
-    multi-pass path finishes the selection (error feedback: with s already written into
-    err).  Plain, EF and EF21, against the oracle."""
+    """A row with 16384 evenly spread magnitudes much larger than the rest, which the
+    evenly spread sample over-represents: the sampled band misses the k-th entry after the
+    first read, and the multi-pass path finishes the selection (error feedback: with s
+    already written into err).  Plain, EF and EF21, against the oracle."""
     rng = np.random.default_rng(L)
     R = 1
     x = (rng.standard_normal((R, L)) * 1e-3).astype(np.float32)
@@ -167,3 +167,59 @@ def test_sample_misled(mpc, L):
     ov, oi = oracle.ef21_topk_compress(x, g_host, k)
     assert_bits_equal(i.cpu().numpy(), oi, "EF21 idx")
     assert_bits_equal(g_dev.cpu().numpy(), g_host, "EF21 g")
+
+
+@pytest.mark.parametrize("R,L", [(70, 70000), (9, 131073), (3, 1 << 20)])
+def test_many_long_rows(mpc, R, L):
+    """Several long rows in one call: the grid path takes up to 64 rows a batch (the row
+    in blockIdx.y, a workspace slice each), so 70 rows make a full batch and a partial
+    one.  Plain TopK at K = 1 / 10 / 50 % and two steps of error feedback, every row
+    against the oracle."""
+    rng = np.random.default_rng(7 * R + L)
+    x = rng.standard_normal((R, L)).astype(np.float32)
+    for k in sorted({max(1, L // 100), L // 10, L // 2}):
+        v, i = mpc.mpc_topk_compress(dev(x), k)
+        ok(mpc)
+        ov, oi = oracle.topk_compress(x, k)
+        assert_bits_equal(i.cpu().numpy(), oi, "idx R=%d L=%d k=%d" % (R, L, k))
+        assert_bits_equal(v.cpu().numpy(), ov, "vals R=%d L=%d k=%d" % (R, L, k))
+    k = L // 10
+    e_host = np.zeros((R, L), np.float32)
+    e_dev = torch.zeros((R, L), device="cuda")
+    for step in range(2):
+        v, i = mpc.mpc_ef_topk_compress(dev(x), e_dev, k)
+        ok(mpc)
+        ov, oi = oracle.ef_topk_compress(x, e_host, k)
+        assert_bits_equal(i.cpu().numpy(), oi, "EF idx step %d" % step)
+        assert_bits_equal(v.cpu().numpy(), ov, "EF vals step %d" % step)
+        assert_bits_equal(e_dev.cpu().numpy(), e_host, "EF err step %d" % step)
+        x = (x + 0.1 * rng.standard_normal((R, L))).astype(np.float32)
+
+
+def test_long_rows_of_every_kind_in_one_batch(mpc):
+    """One batch whose rows take different paths: rows the sampled band resolves next to
+    rows of equal values, zeros and few distinct magnitudes, and a row whose sampled
+    positions hold the largest magnitudes, which fall back to the multi-pass path.  Every
+    row against the oracle, plain and with error feedback."""
+    L = 100000
+    rows = [rows_of(kind, 1, L, seed=11 + n)[0].astype(np.float32) for n, kind in enumerate(KINDS)]
+    rng = np.random.default_rng(5)
+    misled = (rng.standard_normal(L) * 1e-3).astype(np.float32)
+    pos = (np.arange(1024, dtype=np.int64) * L) // 1024  # the sample of a row this long
+    misled[pos] = (1.0 + rng.random(1024)).astype(np.float32)
+    x = np.stack(rows + [misled])
+    R = x.shape[0]
+    for k in (L // 100, L // 4):
+        v, i = mpc.mpc_topk_compress(dev(x), k)
+        ok(mpc)
+        ov, oi = oracle.topk_compress(x, k)
+        assert_bits_equal(i.cpu().numpy(), oi, "idx k=%d" % k)
+        assert_bits_equal(v.cpu().numpy(), ov, "vals k=%d" % k)
+        e_host = (rng.standard_normal((R, L)) * 1e-4).astype(np.float32)
+        e_dev = dev(e_host.copy())
+        v, i = mpc.mpc_ef_topk_compress(dev(x), e_dev, k)
+        ok(mpc)
+        ov, oi = oracle.ef_topk_compress(x, e_host, k)
+        assert_bits_equal(i.cpu().numpy(), oi, "EF idx k=%d" % k)
+        assert_bits_equal(v.cpu().numpy(), ov, "EF vals k=%d" % k)
+        assert_bits_equal(e_dev.cpu().numpy(), e_host, "EF err k=%d" % k)
