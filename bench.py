@@ -25,7 +25,8 @@ Secondary keys: `cnn_boundary_step`, the CNN stage boundary [128,128,16,16] (EF-
 5/10/30 % and 2/4/8-bit quantisation, nearest and stochastic, with their
 decompressions; one CUDA graph per step); `whole_tensor`, whole-tensor rows of 2^27,
 2^28 and 2^29 entries; `operators`, every operator on its own workload (the small CNN,
-transformer and AQ-SGD boundaries, index reuse, EF-mixed, stochastic and 6-bit codes).
+transformer and AQ-SGD boundaries, index reuse, EF-mixed, stochastic and 6-bit codes, and
+256 rows of 2^20 entries through the grid path's batches of rows).
 
 `--impl reference` and `cpu_baseline` time the CPU oracle (single-threaded C) on a
 bounded sample of the same step: a few rows of each row length and a whole-tensor row of
@@ -1149,6 +1150,19 @@ def measure_operators(mpc, synth, device, stream, peak):
                     algorithmic_bytes(Rs, Ls, bits=6, op="dequant"))
                 del ys
             del cq, sq, mq
+    # many long rows (256 rows of 2^20 entries): the grid path's batches of rows
+    Ll = 1 << 20
+    Rl = N // Ll
+    xl2 = xs.view(Rl, Ll)
+    kl2 = synth.k_of(Ll, 10)
+    wsl = torch.empty(mpc.mpc_topk_workspace_bytes(Rl, Ll, kl2), dtype=torch.uint8, device=device)
+    vl2, il2 = mpc.mpc_topk_compress(xl2, kl2, ws=wsl)
+    rec("topk_compress 2^28 L=2^20 K=10%", time_op(lambda: mpc.mpc_topk_compress(xl2, kl2, vl2, il2, wsl), stream, flush),
+        algorithmic_bytes(Rl, Ll, k=kl2, op="topk"))
+    el2 = torch.zeros_like(xl2)
+    rec("ef_topk_compress 2^28 L=2^20 K=10%", time_op(lambda: mpc.mpc_ef_topk_compress(xl2, el2, kl2, vl2, il2, wsl), stream, flush),
+        algorithmic_bytes(Rl, Ll, k=kl2, op="ef_topk"))
+    del vl2, il2, el2, wsl, xl2
     del xs
     torch.cuda.empty_cache()
     st = mpc.mpc_get_status(stream)

@@ -769,6 +769,7 @@ __global__ void __launch_bounds__(kQNT) quant_minmax_kernel(const float* x, int6
 
 __global__ void minmax_init_kernel(uint32_t* mm, int64_t rows) {
   pdl_begin();
+  pdl_end();  // light work: the min/max pass may be scheduled now
   for (int64_t r = blockIdx.x * blockDim.x + threadIdx.x; r < rows;
        r += static_cast<int64_t>(gridDim.x) * blockDim.x) {
     mm[2 * r] = 0xffffffffu;
@@ -1062,12 +1063,13 @@ cudaError_t run_quant_bits(const QuantArgs& a0, int num_sms, cudaStream_t s) {
     spr = (L + kQSCAP - 1) / kQSCAP;
     if (a.rows > 0x7fffffffLL / spr) return cudaErrorInvalidValue;  // before any launch
     uint32_t* mm = static_cast<uint32_t*>(a.ws);
-    minmax_init_kernel<<<static_cast<unsigned>(min64((a.rows + 255) / 256, 1024)), 256, 0, s>>>(mm, a.rows);
+    err = launch_kernel(minmax_init_kernel, dim3(static_cast<unsigned>(min64((a.rows + 255) / 256, 1024))),
+                        dim3(256), 0, s, 0u, mm, a.rows);
+    if (err != cudaSuccess) return err;
     const int occ = resident_blocks(quant_minmax_kernel, kQNT, 0);
     const int64_t mgrid = min64(a.rows * spr, static_cast<int64_t>(num_sms) * occ);
-    quant_minmax_kernel<<<static_cast<unsigned>(mgrid), kQNT, 0, s>>>(
-        a.x, L, a.rows, static_cast<int>(spr), a.slice, a.aligned, mm);
-    err = cudaGetLastError();
+    err = launch_kernel(quant_minmax_kernel, dim3(static_cast<unsigned>(mgrid)), dim3(kQNT), 0, s, 0u,
+                        a.x, L, a.rows, static_cast<int>(spr), a.slice, a.aligned, mm);
     if (err != cudaSuccess) return err;
   }
   const int64_t blocks = a.rows * spr;
