@@ -28,9 +28,10 @@
 //     (coalesced), error feedback zeroes err' and EF21 / AQ-SGD update the state
 //     at the kept columns.  Two-pass mode: a second pass over the row (from
 //     L2), each warp on its own sub-chunks with no block barrier: the kept
-//     entries (|s| > T, and the sub-chunk's quota of ties) of each 128-entry
-//     group staged in shared memory in index order and written out with
-//     coalesced stores (a sub-chunk with nothing kept is not read again); error
+//     entries (|s| > T, and the sub-chunk's quota of ties) of two 128-entry
+//     groups at a time staged in shared memory in index order by predicated
+//     stores and written out with coalesced stores (a sub-chunk with nothing
+//     kept is not read again); error
 //     feedback rewrites err' (+0 where kept), EF21 / AQ-SGD the state (state + d
 //     where kept), a 16-byte group at a time.
 //
@@ -560,8 +561,9 @@ __global__ void __launch_bounds__(NT, 2) topk_lrow_kernel(const TopkRowArgs a) {
   // ---- two-pass mode: the second pass ------------------------------------------------
   // Each warp on its own sub-chunks: kept entries |s| > T (all finite entries when T
   // is -1), and the sub-chunk's quota of ties |s| == T, first in index order.
-  float* ov = reinterpret_cast<float*>(stage) + warp * 256;  // this warp's output buffer
-  int* oc = reinterpret_cast<int*>(ov + 128);
+  // this warp's share of the stage: (value, column) pairs of two 128-entry groups
+  const uint2* op = reinterpret_cast<const uint2*>(stage) + warp * 256;
+  const uint32_t op_s = static_cast<uint32_t>(__cvta_generic_to_shared(op));
   const float tf = T >= 0 ? __uint_as_float(static_cast<uint32_t>(T)) : -1.0f;
   for (int c = 0; c < nch; ++c) {
     const int sc = c * NW + warp;
@@ -623,39 +625,44 @@ __global__ void __launch_bounds__(NT, 2) topk_lrow_kernel(const TopkRowArgs a) {
     const uint32_t ik = warp_inclusive_scan(pk, lane);
     const uint32_t tk = __shfl_sync(kFull, ik, 31);
 #pragma unroll
-    for (int u = 0; u < kU; ++u) {
-      const uint32_t nib = (kw >> (4 * u)) & 0xfu;
-      const uint32_t tu = fld(tk, u);
-      const int col0 = sb + u * 128 + lane * 4;
-      if (tu != 0) {
-        uint32_t p = fld(ik, u) - fld(pk, u);
-        if (nib & 1u) { ov[p] = v[u].x; oc[p] = col0; ++p; }
-        if (nib & 2u) { ov[p] = v[u].y; oc[p] = col0 + 1; ++p; }
-        if (nib & 4u) { ov[p] = v[u].z; oc[p] = col0 + 2; ++p; }
-        if (nib & 8u) { ov[p] = v[u].w; oc[p] = col0 + 3; }
+    for (int u0 = 0; u0 < kU; u0 += 2) {
+      // the kept entries of groups u0 and u0 + 1 staged in index order by
+      // predicated stores, then out with coalesced stores
+      const uint32_t ta = fld(tk, u0), tr = ta + fld(tk, u0 + 1);
+      if (tr != 0) {
+        uint32_t at = op_s + 8u * (fld(ik, u0) - fld(pk, u0));
+        stage_kept4((kw >> (4 * u0)) & 0xfu, at, v[u0], sb + u0 * 128 + lane * 4);
+        at = op_s + 8u * (ta + fld(ik, u0 + 1) - fld(pk, u0 + 1));
+        stage_kept4((kw >> (4 * (u0 + 1))) & 0xfu, at, v[u0 + 1], sb + (u0 + 1) * 128 + lane * 4);
         __syncwarp();
-        for (uint32_t i = lane; i < tu; i += 32) {
-          const uint32_t pos = ubase + i;
-          if (pos < static_cast<uint32_t>(k)) {
-            st_f32(vrow + pos, ov[i], drop);
-            st_s32(irow + pos, oc[i], drop);
-          }
+        const uint32_t lim = static_cast<int64_t>(ubase) < k
+                                 ? static_cast<uint32_t>(min(static_cast<int64_t>(tr), k - ubase))
+                                 : 0u;
+        for (uint32_t i = lane; i < lim; i += 32) {
+          const uint2 e = op[i];
+          st_f32(vrow + ubase + i, __uint_as_float(e.x), drop);
+          st_s32(irow + ubase + i, static_cast<int32_t>(e.y), drop);
         }
         __syncwarp();
-        ubase += tu;
+        ubase += tr;
       }
-      if (MODE != kPlain && nib != 0) {
-        float4 w4;
-        if (MODE == kEF) {  // err' = s - C(s): +0 where sent
-          w4 = make_float4((nib & 1u) ? 0.0f : v[u].x, (nib & 2u) ? 0.0f : v[u].y,
-                           (nib & 4u) ? 0.0f : v[u].z, (nib & 8u) ? 0.0f : v[u].w);
-        } else {  // state + d where sent
-          w4 = make_float4((nib & 1u) ? fadd(g[u].x, v[u].x) : g[u].x,
-                           (nib & 2u) ? fadd(g[u].y, v[u].y) : g[u].y,
-                           (nib & 4u) ? fadd(g[u].z, v[u].z) : g[u].z,
-                           (nib & 8u) ? fadd(g[u].w, v[u].w) : g[u].w);
+#pragma unroll
+      for (int u = u0; u < u0 + 2; ++u) {
+        const uint32_t nib = (kw >> (4 * u)) & 0xfu;
+        const int col0 = sb + u * 128 + lane * 4;
+        if (MODE != kPlain && nib != 0) {
+          float4 w4;
+          if (MODE == kEF) {  // err' = s - C(s): +0 where sent
+            w4 = make_float4((nib & 1u) ? 0.0f : v[u].x, (nib & 2u) ? 0.0f : v[u].y,
+                             (nib & 4u) ? 0.0f : v[u].z, (nib & 8u) ? 0.0f : v[u].w);
+          } else {  // state + d where sent
+            w4 = make_float4((nib & 1u) ? fadd(g[u].x, v[u].x) : g[u].x,
+                             (nib & 2u) ? fadd(g[u].y, v[u].y) : g[u].y,
+                             (nib & 4u) ? fadd(g[u].z, v[u].z) : g[u].z,
+                             (nib & 8u) ? fadd(g[u].w, v[u].w) : g[u].w);
+          }
+          st_f4(arow + col0, w4, drop);
         }
-        st_f4(arow + col0, w4, drop);
       }
     }
   }

@@ -902,26 +902,6 @@ __device__ __forceinline__ void or_if_key_gt(uint32_t& w, int key, int t, uint32
   asm("{\n .reg .pred p;\n setp.gt.s32 p, %1, %2;\n @p or.b32 %0, %0, %3;\n}" : "+r"(w) : "r"(key), "r"(t), "r"(bit));
 }
 
-// Appends the kept ones of four entries (bits of nib) to a warp's write stage
-// as (value bits, column) pairs from shared byte address `at` on, and advances
-// it: predicated stores, no branch.
-__device__ __forceinline__ void stage_kept4(uint32_t nib, uint32_t& at, float4 v, int col0) {
-  asm volatile(
-      "{\n .reg .pred p;\n .reg .b32 t;\n"
-      " and.b32 t, %1, 1;\n setp.ne.b32 p, t, 0;\n"
-      " @p st.shared.v2.b32 [%0], {%2, %6};\n @p add.u32 %0, %0, 8;\n"
-      " and.b32 t, %1, 2;\n setp.ne.b32 p, t, 0;\n"
-      " @p st.shared.v2.b32 [%0], {%3, %7};\n @p add.u32 %0, %0, 8;\n"
-      " and.b32 t, %1, 4;\n setp.ne.b32 p, t, 0;\n"
-      " @p st.shared.v2.b32 [%0], {%4, %8};\n @p add.u32 %0, %0, 8;\n"
-      " and.b32 t, %1, 8;\n setp.ne.b32 p, t, 0;\n"
-      " @p st.shared.v2.b32 [%0], {%5, %9};\n @p add.u32 %0, %0, 8;\n}"
-      : "+r"(at)
-      : "r"(nib), "r"(__float_as_uint(v.x)), "r"(__float_as_uint(v.y)), "r"(__float_as_uint(v.z)),
-        "r"(__float_as_uint(v.w)), "r"(col0), "r"(col0 + 1), "r"(col0 + 2), "r"(col0 + 3)
-      : "memory");
-}
-
 // Row of the error / state buffer for a logical row (nullptr for plain TopK);
 // *ok = false for an AQ-SGD sample id out of range.
 template <int MODE>
