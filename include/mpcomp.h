@@ -75,8 +75,11 @@ int mpc_version(void);
 /* ------------------------------------------------------------------------ */
 
 /* Bytes of device workspace the TopK compress calls below need for this
- * shape (0 when none).  Rows longer than the on-chip path handles use a
- * multi-pass path that keeps counters and candidates in the workspace. */
+ * shape (0 when none).  Rows longer than the on-chip path handles (65536
+ * entries) use a multi-pass path that keeps counters, lists and candidates
+ * in the workspace; it takes the rows in batches of up to 64 (about 2^26
+ * entries a batch), one 256-byte-aligned slice of the workspace per row of a
+ * batch, so the size grows with min(rows, batch) rather than with rows. */
 size_t mpc_topk_workspace_bytes(int64_t rows, int64_t row_len, int64_t k);
 
 /* TopK compress (§2.3: keep the K% entries of each row with the largest
