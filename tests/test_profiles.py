@@ -63,3 +63,43 @@ def test_step_branch_layouts():
         assert sorted(set(got)) == list(range(nb)), (nb, got)
         assert nb in b.BRANCH_TEXT
     assert set(b.BRANCH_OF[1](i, None if i < 3 else False) for i in range(9)) == {0}
+
+
+def test_algorithmic_bytes():
+    """Minimum HBM bytes per call: TopK 4N + 8kR, error feedback / EF21 / AQ-SGD
+    12N + 8kR, decompression 8kR + 4N, (de)quantisation 4N + ceil(N b / 8) + 8R."""
+    b = _bench()
+    R, L, k = 2, 10, 3
+    assert b.algorithmic_bytes(R, L, k=k, op="topk") == 4 * 20 + 8 * 3 * 2
+    assert b.algorithmic_bytes(R, L, k=k, op="ef_topk") == 12 * 20 + 8 * 3 * 2
+    assert b.algorithmic_bytes(R, L, k=k, op="delta_topk") == 12 * 20 + 8 * 3 * 2
+    assert b.algorithmic_bytes(R, L, k=k, op="topk_decompress") == 8 * 3 * 2 + 4 * 20
+    assert b.algorithmic_bytes(R, L, bits=3, op="quant") == 4 * 20 + 8 + 8 * 2  # 60 bits -> 8 B
+    assert b.algorithmic_bytes(R, L, bits=4, op="dequant") == 4 * 20 + 10 + 8 * 2
+    # the headline at 2^30: a whole-tensor error-feedback TopK at K = 50 % is 17.2 GB
+    N = 1 << 30
+    assert b.algorithmic_bytes(1, N, k=N // 2, op="ef_topk") == 12 * N + 4 * N
+
+
+def test_kernels_of_name_library_kernels():
+    """Every kernel bench.py attributes a headline call's launches to is a __global__
+    function of the library's sources (the traffic table and the launch list map ncu's
+    launches to calls through these lists)."""
+    import re
+
+    b = _bench()
+    csrc = os.path.join(ROOT, "paper_2401_07788_gb300", "csrc")
+    text = "".join(open(os.path.join(csrc, f)).read() for f in os.listdir(csrc)
+                   if f.endswith((".cu", ".cuh")))
+    bounds = r"__launch_bounds__\((?:[^()]|\([^()]*\))*\)\s*"  # one level of nesting
+    globals_ = set(re.findall(r"__global__\s+void\s+(?:%s)?(\w+)\s*\(" % bounds, text))
+    N = 1 << b.LOG2N
+    for op in ("topk", "ef_topk", "topk_decompress", "quant", "dequant"):
+        for L in (768, 4096, 65536, N):
+            ks = b.kernels_of(op, L)
+            assert ks, (op, L)
+            for kname in ks:
+                assert kname in globals_, (op, L, kname)
+    # a whole-tensor TopK is one batch of 23 launches, a whole-tensor quantisation 3
+    assert len(b.kernels_of("topk", N)) == 23
+    assert len(b.kernels_of("quant", N)) == 3
